@@ -1,0 +1,453 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each check_* raises AssertionError on a mismatch; tests/test_oracle_pins.py runs
+them on the oracle, tests/test_oracle_mutations.py plants plausible mistakes in
+the oracle and asserts that some check catches each one.  Nothing here calls the
+CUDA path.
+"""
+from __future__ import annotations
+
+import itertools
+import os
+
+import numpy as np
+import scipy.special
+
+import oracle.cast_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def read_golden(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                rows.append(line.split())
+    return rows
+
+
+# ---------------------------------------------------------------------------
+# DFT (Section 4.3, App. A.2)
+# ---------------------------------------------------------------------------
+
+
+def check_dft_matches_library():
+    """The naive DFT equals numpy's orthonormal rfft2 for every tile shape up to 8x8."""
+    r = _rng(0)
+    for h in range(1, 9):
+        for w in range(1, 9):
+            x = r.standard_normal((3, h, w))
+            assert np.allclose(O.rfft2_ortho(x), np.fft.rfft2(x, norm="ortho"), atol=1e-12)
+
+
+def check_dft_round_trip_and_parseval():
+    """irfft2(rfft2(x)) = x and sum kappa |F|^2 = sum x^2 (real-FFT multiplicities)."""
+    r = _rng(1)
+    for h, w in [(8, 8), (4, 8), (8, 4), (6, 8), (5, 7), (3, 3), (1, 8), (8, 1), (2, 2)]:
+        x = r.standard_normal((4, h, w))
+        F = O.rfft2_ortho(x)
+        assert np.allclose(O.irfft2_ortho(F, w), x, atol=1e-12)
+        b = O.tile_bins(h, w)
+        assert np.allclose(np.sum(b.kappa * np.abs(F) ** 2, axis=(-2, -1)),
+                           np.sum(x ** 2, axis=(-2, -1)), rtol=1e-12)
+
+
+def check_bin_structure():
+    """Mirrors hold the conjugate of their representative for real input; self-conjugate
+    bins are real; every stored bin's (ky, kx) radius is within [0, 1] after normalisation."""
+    r = _rng(2)
+    for h in range(1, 9):
+        for w in range(1, 9):
+            x = r.standard_normal((h, w))
+            F = np.fft.rfft2(x, norm="ortho")
+            b = O.tile_bins(h, w)
+            ry, rx = b.rep[..., 0], b.rep[..., 1]
+            assert np.allclose(F[b.mirror], np.conj(F[ry, rx][b.mirror]), atol=1e-12)
+            assert np.allclose(F[b.selfconj].imag, 0.0, atol=1e-12)
+            assert b.nu.min() >= 0.0 and b.nu.max() <= 1.0 + 1e-15
+            if h % 2 == 0 and w % 2 == 0:
+                assert b.selfconj.sum() == 4
+                assert abs(b.nu[h // 2, w // 2] - 1.0) < 1e-15
+
+
+# ---------------------------------------------------------------------------
+# PAR (Section 4.3, Eq. fcpasm; App. A.2)
+# ---------------------------------------------------------------------------
+
+
+def _assign(mask):
+    return O.skipped_assignment(mask)
+
+
+def check_interval_coefficients_closed_form():
+    """Sums of (1-a)^2, a^2, a(1-a) over an interval's skipped frames (Eq. abc) with the
+    alphas of Eq. (block) equal the printed closed forms of Eq. (abcclosed)."""
+    for n, A_ref, C_ref in read_golden("abc_closed_form.txt"):
+        n = int(n)
+        mask = np.zeros(n + 1, dtype=np.uint8)
+        mask[0] = mask[n] = 1
+        al = np.array([a for (_, _, _, a) in _assign(mask)]) if n > 1 else np.zeros(0)
+        assert abs(np.sum((1 - al) ** 2) - float(A_ref)) < 1e-12
+        assert abs(np.sum(al ** 2) - float(A_ref)) < 1e-12
+        assert abs(np.sum(al * (1 - al)) - float(C_ref)) < 1e-12
+
+
+def check_assignment_boundaries():
+    """Frames outside the anchor span extrapolate from the two nearest anchors (Eq. block)."""
+    got = {t: (a, b, al) for (t, a, b, al) in _assign([0, 1, 0, 1, 0, 0])}
+    assert got[0] == (1, 3, -0.5)
+    assert got[2] == (1, 3, 0.5)
+    assert got[4] == (1, 3, 1.5) and got[5] == (1, 3, 2.0)
+    assert _assign([1, 1, 1]) == []
+
+
+def _par(R, mask, **kw):
+    wch = kw.pop("wch", None)
+    return O.par_reconstruct(R, np.asarray(mask, dtype=np.uint8), wch, O.ParParams(**kw))
+
+
+def check_par_identical_anchors():
+    """R_a = R_b: theta = 0, every reconstruction returns the anchor (interpolation and
+    extrapolation, every gate mode, ragged edge tiles)."""
+    r = _rng(3)
+    base = r.standard_normal((11, 13, 5))
+    R = np.stack([base] * 6)
+    R[[1, 2, 4, 5]] = r.standard_normal((4, 11, 13, 5))   # skipped rows: overwritten
+    for mode in ("paper", "zero", "one"):
+        out = _par(R, [1, 0, 0, 1, 0, 0], gate_mode=mode)
+        for t in (1, 2, 4, 5):
+            assert np.allclose(out[t], base, atol=1e-12)
+
+
+def check_par_gate_zero_is_linear():
+    """g = 0 gives direct value interpolation / extrapolation (1-a) R_a + a R_b."""
+    r = _rng(4)
+    R = r.standard_normal((7, 10, 12, 6))
+    mask = [0, 1, 0, 0, 1, 0, 0]
+    out = _par(R, mask, gate_mode="zero")
+    for (t, a, b, al) in _assign(mask):
+        assert np.allclose(out[t], (1 - al) * R[a] + al * R[b], atol=1e-12)
+    for (t, a, b, al) in _assign(mask):   # band radius 0 keeps only DC -> also linear
+        out2 = _par(R, mask, band_radius=0.0)
+        assert np.allclose(out2[t], (1 - al) * R[a] + al * R[b], atol=1e-12)
+
+
+def check_par_endpoints():
+    """alpha = 0 reproduces R_a and alpha = 1 reproduces R_b exactly (Section 4.3)."""
+    r = _rng(5)
+    F_a = O.rfft2_ortho(r.standard_normal((3, 8, 8)))
+    F_b = O.rfft2_ortho(r.standard_normal((3, 8, 8)))
+    th = r.uniform(-np.pi, np.pi, (8, 5))
+    g = r.uniform(0, 1, (8, 5))
+    assert np.allclose(O.blend(F_a, F_b, th, g, 0.0), F_a, atol=1e-14)
+    assert np.allclose(O.blend(F_a, F_b, th, g, 1.0), F_b, atol=1e-14)
+
+
+def _bandlimited_tile(r, C, h, w, keep):
+    """Real [C, h, w] fields whose spectrum lives on the bins where keep(ky_s, kx) holds."""
+    F = np.fft.rfft2(r.standard_normal((C, h, w)), norm="ortho")
+    ky = np.fft.fftfreq(h, 1.0 / h)[:, None]
+    kx = np.arange(w // 2 + 1)[None, :]
+    F = F * keep(ky, kx)
+    return np.fft.irfft2(F, s=(h, w), norm="ortho")
+
+
+def check_par_translation_identity():
+    """Eq. (exacttranslation): with g = 1, a band-limited circular translation by d between
+    the anchors reconstructs to the translation by alpha*d, also for alpha outside [0, 1]."""
+    r = _rng(6)
+    # shift along W by 2: energy only at |kx| <= 1 so that |omega . d| < pi
+    x = _bandlimited_tile(r, 3, 8, 8, lambda ky, kx: (kx <= 1))
+    R = np.zeros((5, 8, 8, 3))
+    R[0] = np.moveaxis(x, 0, -1)
+    R[2] = np.roll(R[0], 2, axis=1)
+    out = _par(R, [1, 0, 1, 0, 0], gate_mode="one")
+    assert np.allclose(out[1], np.roll(R[0], 1, axis=1), atol=1e-10)      # alpha = 1/2
+    assert np.allclose(out[4], np.roll(R[0], 4, axis=1), atol=1e-10)      # alpha = 2
+    # shift along H by 2 (tests the mirrored kx = 0 column): energy at |ky| <= 1
+    y = _bandlimited_tile(r, 3, 8, 8, lambda ky, kx: (np.abs(ky) <= 1) + 0 * kx)
+    R = np.zeros((4, 8, 8, 3))
+    R[1] = np.moveaxis(y, 0, -1)
+    R[3] = np.roll(R[1], 2, axis=0)
+    out = _par(R, [0, 1, 0, 1], gate_mode="one")
+    assert np.allclose(out[2], np.roll(R[1], 1, axis=0), atol=1e-10)      # alpha = 1/2
+    assert np.allclose(out[0], np.roll(R[1], -1, axis=0), atol=1e-10)     # alpha = -1/2
+    # diagonal shift (1, 1) with energy in the low band: alpha = 3 extrapolates by (3, 3)
+    z = _bandlimited_tile(r, 2, 8, 8, lambda ky, kx: (np.abs(ky) <= 1) & (kx <= 1))
+    R = np.zeros((5, 8, 8, 2))
+    R[0] = np.moveaxis(z, 0, -1)
+    R[1] = np.roll(R[0], (1, 1), axis=(0, 1))
+    out = _par(R, [1, 1, 0, 0, 0], gate_mode="one")
+    assert np.allclose(out[3], np.roll(R[0], (3, 3), axis=(0, 1)), atol=1e-10)
+
+
+def check_par_confidence_closed_form():
+    """Two channels carrying one spatial frequency, translated by d1 and d2: the pooled
+    resultant length gives c = |cos(omega.(d1 - d2)/2)|; a pure translation gives c = 1."""
+    h = w = 8
+    yy, xx = np.meshgrid(np.arange(h), np.arange(w), indexing="ij")
+    k = (0, 1)                      # one bin pair
+    om = 2 * np.pi * np.array([k[0] / h, k[1] / w])
+    base = np.cos(om[0] * yy + om[1] * xx + 0.3)
+    for d1, d2 in [((0, 1), (0, 1)), ((0, 1), (0, 3)), ((0, 0), (0, 2)), ((0, 2), (0, 3))]:
+        A = np.stack([base, base])
+        B = np.stack([np.roll(base, d1, axis=(0, 1)), np.roll(base, d2, axis=(0, 1))])
+        Fa, Fb = O.rfft2_ortho(A), O.rfft2_ortho(B)
+        tt = O.tile_transport(Fa, Fb, None, O.ParParams(), O.tile_bins(h, w))
+        delta = om @ (np.array(d1) - np.array(d2))
+        assert abs(tt.c - abs(np.cos(delta / 2))) < 1e-9, (d1, d2, tt.c)
+    # content at (1, 0) (kappa = 1, stored with its mirror) and at (0, 1) (kappa = 2) with
+    # coherence 1 and |cos(pi/4)|: c weighs every bin of the full spectrum equally
+    om1, om2 = 2 * np.pi / h, 2 * np.pi / w
+    f1 = np.cos(om1 * yy + 0.2)
+    f2 = np.cos(om2 * xx + 0.7)
+    A = np.stack([f1 + f2, f1 + f2])
+    B = np.stack([np.roll(f1, 1, axis=0) + np.roll(f2, 1, axis=1),
+                  np.roll(f1, 1, axis=0) + np.roll(f2, 3, axis=1)])
+    tt = O.tile_transport(O.rfft2_ortho(A), O.rfft2_ortho(B), None, O.ParParams(),
+                          O.tile_bins(h, w))
+    assert abs(tt.c - (1.0 + abs(np.cos(np.pi / 4))) / 2.0) < 1e-9, tt.c
+    # random content with independent random circular shifts per channel: 0 <= c <= 1
+    r = _rng(7)
+    A = r.standard_normal((64, 8, 8))
+    B = np.stack([np.roll(a, tuple(r.integers(0, 8, 2)), axis=(0, 1)) for a in A])
+    tt = O.tile_transport(O.rfft2_ortho(A), O.rfft2_ortho(B), None, O.ParParams(),
+                          O.tile_bins(8, 8))
+    assert 0.0 <= tt.c <= 0.6
+
+
+def check_par_gate_at_threshold():
+    """Eq. (gate): where c equals tau(nu) the gate is exactly 1/2; the printed constants
+    (tau_low, tau_high, q, T) of Tab. config_cast fix tau at nu = 0 and nu = 1."""
+    consts = {k: float(v) for k, v in read_golden("par_constants.txt")}
+    p = O.ParParams()
+    for k in ("tau_low", "tau_high", "q", "T", "eta_rel", "eta_abs", "eps"):
+        assert getattr(p, k) == consts[k], k
+    assert (p.tile_h, p.tile_w) == (int(consts["tile_h"]), int(consts["tile_w"]))
+    h = w = 8
+    b = O.tile_bins(h, w)
+    yy, xx = np.meshgrid(np.arange(h), np.arange(w), indexing="ij")
+    # bin (0, 1): nu = (1/8) / sqrt(0.5); tau = 0.25 + 0.5 nu^2 = 0.265625
+    nu = b.nu[0, 1]
+    tau = consts["tau_low"] + (consts["tau_high"] - consts["tau_low"]) * nu ** consts["q"]
+    assert abs(tau - 0.265625) < 1e-15
+    # two channels at frequency (0,1) with translations differing by delta along W give
+    # c = |cos(delta * pi / 8)|; pick delta so that c = tau
+    delta = 8.0 / np.pi * np.arccos(tau)
+    om = 2 * np.pi / w
+    base = np.cos(om * xx + 0.1)
+    A = np.stack([base, base])
+    B = np.stack([np.cos(om * (xx - 0.0) + 0.1), np.cos(om * (xx - delta) + 0.1)])
+    tt = O.tile_transport(O.rfft2_ortho(A), O.rfft2_ortho(B), None, p, b)
+    assert abs(tt.c - tau) < 1e-9
+    assert abs(tt.g[0, 1] - 0.5) < 1e-7
+
+
+def check_par_frozen_transport_bound():
+    """Prop. 1 (Eq. bound) and the extrapolation amplification bound |1-a| + |a| (App. A.2):
+    with U and g frozen, perturbations of the anchors move the reconstruction by at most
+    the stated amounts."""
+    r = _rng(8)
+    h = w = 8
+    b = O.tile_bins(h, w)
+    Ra, Rb = r.standard_normal((2, 4, h, w))
+    tt = O.tile_transport(O.rfft2_ortho(Ra), O.rfft2_ortho(Rb), None, O.ParParams(), b)
+    for n in (2, 3, 5):
+        alphas = np.arange(1, n) / n
+        va, vb = r.standard_normal((2, 4, h, w))
+        Fa, Fb = O.rfft2_ortho(va), O.rfft2_ortho(vb)
+        lhs = sum(np.sum(O.irfft2_ortho(O.blend(Fa, Fb, tt.theta, tt.g, al), w) ** 2)
+                  for al in alphas)
+        A = np.sum((1 - alphas) ** 2)
+        B = np.sum(alphas ** 2)
+        C = np.sum(alphas * (1 - alphas))
+        na, nb = np.linalg.norm(va), np.linalg.norm(vb)
+        assert lhs <= A * na ** 2 + B * nb ** 2 + 2 * C * na * nb + 1e-9
+        # frozen transport is norm preserving per anchor (Parseval)
+        one_a = O.irfft2_ortho(O.blend(Fa, 0 * Fb, tt.theta, tt.g, 0.5), w) / 0.5
+        assert abs(np.linalg.norm(one_a) - na) < 1e-9
+    for al in (-1.0, -0.5, 1.5, 2.0):
+        va, vb = r.standard_normal((2, 4, h, w))
+        out = O.irfft2_ortho(O.blend(O.rfft2_ortho(va), O.rfft2_ortho(vb), tt.theta, tt.g, al), w)
+        assert np.linalg.norm(out) <= (abs(1 - al) + abs(al)) * max(
+            np.linalg.norm(va), np.linalg.norm(vb)) + 1e-9
+
+
+def check_par_unreliable_bins_interpolate():
+    """A bin with no energy in one anchor fails the reliability threshold and keeps U = 1."""
+    h = w = 8
+    r = _rng(9)
+    A = _bandlimited_tile(r, 2, h, w, lambda ky, kx: (kx <= 2))
+    B = _bandlimited_tile(r, 2, h, w, lambda ky, kx: (kx <= 1))     # kx = 2 empty in B
+    tt = O.tile_transport(O.rfft2_ortho(A), O.rfft2_ortho(B), None, O.ParParams(),
+                          O.tile_bins(h, w))
+    assert not tt.reliable[:, 2].any()
+    assert np.all(tt.theta[:, 2] == 0.0)
+    assert not tt.reliable[0, 0] or tt.theta[0, 0] == 0.0
+
+
+def check_par_weights_scale_invariant():
+    """Scaling every channel weight by a constant leaves the reconstruction unchanged;
+    unit weights equal the unweighted paper form."""
+    r = _rng(10)
+    R = r.standard_normal((3, 8, 16, 6))
+    mask = [1, 0, 1]
+    wc = r.uniform(0.1, 1.0, 6)
+    a = _par(R, mask, wch=wc)
+    b = _par(R, mask, wch=3.0 * wc)
+    c = _par(R, mask, wch=np.ones(6))
+    d = _par(R, mask)
+    assert np.allclose(a, b, atol=1e-9)
+    assert np.allclose(c, d, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Routing (Section 4.4, Eqs. pooled, omission; App. B.1 Eq. omissionexact)
+# ---------------------------------------------------------------------------
+
+
+def _routing_inputs(seed, N=3, S=5, H=2, d=4, M=6, Bv=3):
+    r = _rng(seed)
+    q = r.standard_normal((N, S, H, d)) + r.standard_normal((N, 1, H, d))
+    k = r.standard_normal((M, Bv, H, d)) + r.standard_normal((M, 1, H, d))
+    v = r.standard_normal((M, Bv, H, d)) + r.standard_normal((M, 1, H, d))
+    return q, k, v
+
+
+def check_omission_identity():
+    """Eq. (omissionexact): with eps = 0, delta_m equals the change of the pooled output when
+    block m is dropped and the remaining weights are renormalised (brute force)."""
+    q, k, v = _routing_inputs(11)
+    anchors = [0, 2]
+    rt = O.pooled_routing(q, anchors, k, v, eps=0.0)
+    M, H, d = k.shape[0], k.shape[2], k.shape[3]
+    for i, a in enumerate(anchors):
+        for h in range(H):
+            qb = q[a, :, h].mean(axis=0)
+            kb = k[:, :, h].mean(axis=1)
+            vb = v[:, :, h].mean(axis=1)
+            s = kb @ qb / np.sqrt(d)
+            full = scipy.special.softmax(s) @ vb
+            assert np.allclose(rt.obar[i, h], full, atol=1e-12)
+            for m in range(M):
+                keep = [j for j in range(M) if j != m]
+                drop = scipy.special.softmax(s[keep]) @ vb[keep]
+                assert np.allclose(rt.delta[i, h, m], drop - full, atol=1e-10)
+
+
+def check_omission_projection():
+    """u = ||P delta||^2: P = I gives ||delta||^2, an orthogonal P leaves u unchanged, P = 2I
+    multiplies it by 4, and u equals delta^T (P^T P) delta (the Gram form)."""
+    q, k, v = _routing_inputs(12)
+    H, d = q.shape[2], q.shape[3]
+    r = _rng(13)
+    base = O.pooled_routing(q, [1], k, v)
+    Qm = np.stack([np.linalg.qr(r.standard_normal((d, d)))[0] for _ in range(H)])
+    rot = O.pooled_routing(q, [1], k, v, proj=Qm)
+    two = O.pooled_routing(q, [1], k, v, proj=2 * np.stack([np.eye(d)] * H))
+    assert np.allclose(base.u, np.sum(base.delta ** 2, axis=-1), rtol=1e-12)
+    assert np.allclose(rot.u, base.u, rtol=1e-10)
+    assert np.allclose(two.u, 4 * base.u, rtol=1e-12)
+    P = r.standard_normal((H, 7, d))
+    pr = O.pooled_routing(q, [1], k, v, proj=P)
+    gram = np.einsum("hod,hoe->hde", P, P)
+    assert np.allclose(pr.u, np.einsum("ihmd,hde,ihme->ihm", pr.delta, gram, pr.delta),
+                       rtol=1e-10)
+
+
+def check_pooled_scores():
+    """s = q.k/sqrt(d) on token means, softmax over blocks sums to one, scores permute with
+    the blocks (Eq. pooled)."""
+    q, k, v = _routing_inputs(14)
+    rt = O.pooled_routing(q, [0, 1], k, v)
+    d = q.shape[-1]
+    assert np.allclose(rt.pi.sum(-1), 1.0)
+    for i, a in enumerate([0, 1]):
+        for h in range(q.shape[2]):
+            for m in range(k.shape[0]):
+                qs = sum(q[a, s, h] for s in range(q.shape[1])) / q.shape[1]
+                ks = sum(k[m, j, h] for j in range(k.shape[1])) / k.shape[1]
+                assert abs(rt.s[i, h, m] - float(qs @ ks) / np.sqrt(d)) < 1e-12
+    perm = _rng(15).permutation(k.shape[0])
+    rp = O.pooled_routing(q, [0, 1], k[perm], v[perm])
+    assert np.allclose(rp.u, rt.u[..., perm], rtol=1e-12)
+
+
+def check_topk():
+    """TopK keeps the K largest (the subset of maximal sum when scores are distinct), ties
+    go to the lower block index, output ascending; K >= M keeps every block."""
+    r = _rng(16)
+    for _ in range(20):
+        M, K = 7, 3
+        u = r.standard_normal(M)
+        best = max(itertools.combinations(range(M), K), key=lambda c: sum(u[list(c)]))
+        assert list(O.topk_blocks(u[None], K)[0]) == sorted(best)
+    u = np.array([1.0, 3.0, 2.0, 3.0, 2.0, 0.5])
+    assert list(O.topk_blocks(u[None], 3)[0]) == [1, 2, 3]
+    assert list(O.topk_blocks(u[None], 2)[0]) == [1, 3]
+    assert list(O.topk_blocks(u[None], 9)[0]) == list(range(6))
+    assert O.topk_blocks(np.zeros((1, 0)), 3).shape == (1, 0)
+
+
+# ---------------------------------------------------------------------------
+# Routed attention (Eq. block; App. B.4)
+# ---------------------------------------------------------------------------
+
+
+def _attn_inputs(seed, N=3, S=4, H=2, d=8, M=3, Bv=5):
+    r = _rng(seed)
+    return (r.standard_normal((N, S, H, d)), r.standard_normal((N, S, H, d)),
+            r.standard_normal((N, S, H, d)), r.standard_normal((M, Bv, H, d)),
+            r.standard_normal((M, Bv, H, d)))
+
+
+def check_attention_brute_force():
+    """Pure-Python loops of softmax attention over the current chunk followed by the routed
+    blocks equal the oracle on tiny inputs."""
+    q, kc, vc, kh, vh = _attn_inputs(17)
+    N, S, H, d = q.shape
+    anchors = [0, 2]
+    idx = np.array([[[0, 2], [1, 2]], [[1, 2], [0, 1]]])
+    out = O.routed_attention(q, kc, vc, kh, vh, anchors, idx)
+    sc = 1 / np.sqrt(d)
+    for i, a in enumerate(anchors):
+        for h in range(H):
+            keys = [kc[f, s, h] for f in range(N) for s in range(S)]
+            vals = [vc[f, s, h] for f in range(N) for s in range(S)]
+            for m in idx[i, h]:
+                keys += [kh[m, j, h] for j in range(kh.shape[1])]
+                vals += [vh[m, j, h] for j in range(kh.shape[1])]
+            for s in range(S):
+                lg = [float(q[a, s, h] @ kk) * sc for kk in keys]
+                mx = max(lg)
+                e = [np.exp(x - mx) for x in lg]
+                z = sum(e)
+                o = sum(ej / z * vv for ej, vv in zip(e, vals))
+                assert np.allclose(out[i, s, h], o, atol=1e-12)
+
+
+def check_attention_dense_limit():
+    """Routing every history block equals dense softmax attention over current plus all
+    history (library softmax), and permuting the routed blocks changes nothing."""
+    q, kc, vc, kh, vh = _attn_inputs(18)
+    N, S, H, d = q.shape
+    M = kh.shape[0]
+    anchors = [1]
+    idx = np.tile(np.arange(M), (1, H, 1))
+    out = O.routed_attention(q, kc, vc, kh, vh, anchors, idx)
+    for h in range(H):
+        K = np.concatenate([kc[:, :, h].reshape(-1, d), kh[:, :, h].reshape(-1, d)])
+        V = np.concatenate([vc[:, :, h].reshape(-1, d), vh[:, :, h].reshape(-1, d)])
+        ref = scipy.special.softmax(q[1, :, h] @ K.T / np.sqrt(d), axis=1) @ V
+        assert np.allclose(out[0, :, h], ref, atol=1e-12)
+    perm = idx[..., ::-1]
+    assert np.allclose(O.routed_attention(q, kc, vc, kh, vh, anchors, perm), out, atol=1e-12)
+
+
+ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

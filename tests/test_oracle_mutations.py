@@ -1,0 +1,112 @@
+"""Plant plausible mistakes in the CPU oracle and check that its pins catch every one.
+
+Each mutation replaces one oracle function (on the CPU, for the duration of the
+test) with a subtly wrong variant: a flipped sign, a dropped term, a transposed
+operand, a wrong multiplicity or tie rule.  At least one pin must then fail.
+"""
+import numpy as np
+import pytest
+
+import oracle.cast_oracle as O
+from tests import oracle_checks as C
+
+_orig_blend = O.blend
+_orig_bins = O.tile_bins
+_orig_pooled = O.pooled_routing
+_orig_transport = O.tile_transport
+
+
+def _blend_sign(Fa, Fb, th, g, al):
+    return (1 - al) * Fa * np.exp(-1j * g * al * th) + al * Fb * np.exp(1j * g * (1 - al) * th)
+
+
+def _blend_swapped(Fa, Fb, th, g, al):
+    return al * Fa * np.exp(1j * g * al * th) + (1 - al) * Fb * np.exp(-1j * g * (1 - al) * th)
+
+
+def _blend_no_gate(Fa, Fb, th, g, al):
+    return (1 - al) * Fa * np.exp(1j * al * th) + al * Fb * np.exp(-1j * (1 - al) * th)
+
+
+def _rfft2_transposed(x):
+    h, w = x.shape[-2:]
+    ey = O.dft_matrix(h, -1).T.conj().T        # = ey
+    ex = O.dft_matrix(w, +1)[:, : w // 2 + 1]  # wrong sign of the exponent
+    return (ey @ x @ ex) / np.sqrt(h * w)
+
+
+def _transport_mirror_same_sign(Fa, Fb, wch, p, bins, amb_tol=1e-5):
+    tt = _orig_transport(Fa, Fb, wch, p, bins, amb_tol)
+    tt.theta = np.where(bins.mirror, -tt.theta, tt.theta)      # mirror copies +theta_rep
+    return tt
+
+
+def _bins_kappa_one(h, w):
+    b = _orig_bins(h, w)
+    b.kappa = np.ones_like(b.kappa)
+    return b
+
+
+def _bins_nu_unnormalised(h, w):
+    b = _orig_bins(h, w)
+    ky = np.arange(h)[:, None]
+    kx = np.arange(w // 2 + 1)[None, :]
+    ky_s = np.where(ky <= (h - 1) // 2, ky, ky - h)
+    b.nu = np.sqrt((ky_s / h) ** 2 + (kx / w) ** 2)
+    return b
+
+
+def _pooled_no_renorm(q, anchors, k, v, proj=None, eps=1e-8):
+    rt = _orig_pooled(q, anchors, k, v, proj=proj, eps=eps)
+    rt.delta = rt.delta * (1.0 - rt.pi[..., None] + eps)        # drops 1/(1 - pi + eps)
+    rt.u = np.sum(rt.delta ** 2, axis=-1)
+    return rt
+
+
+def _topk_high_ties(score, K):
+    M = score.shape[-1]
+    keff = min(K, M)
+    if M == 0:
+        return np.zeros(score.shape[:-1] + (0,), dtype=np.int64)
+    flat = score.reshape(-1, M)
+    out = [np.sort(np.lexsort((-np.arange(M), -r))[:keff]) for r in flat]
+    return np.array(out).reshape(score.shape[:-1] + (keff,))
+
+
+def _attn_ignores_history(q, kc, vc, kh, vh, anchors, idx, **kw):
+    return _orig_attn(q, kc, vc, kh, vh, anchors, None if idx is None else idx[..., :0], **kw)
+
+
+_orig_attn = O.routed_attention
+
+
+def _attn_no_scale(q, kc, vc, kh, vh, anchors, idx, scale=None, **kw):
+    return _orig_attn(q, kc, vc, kh, vh, anchors, idx, scale=1.0, **kw)
+
+
+MUTATIONS = {
+    "blend_phase_sign": ("blend", _blend_sign),
+    "blend_weights_swapped": ("blend", _blend_swapped),
+    "blend_gate_dropped": ("blend", _blend_no_gate),
+    "dft_exponent_sign": ("rfft2_ortho", _rfft2_transposed),
+    "mirror_not_negated": ("tile_transport", _transport_mirror_same_sign),
+    "kappa_dropped": ("tile_bins", _bins_kappa_one),
+    "nu_not_normalised": ("tile_bins", _bins_nu_unnormalised),
+    "omission_renorm_dropped": ("pooled_routing", _pooled_no_renorm),
+    "topk_ties_high": ("topk_blocks", _topk_high_ties),
+    "attention_history_dropped": ("routed_attention", _attn_ignores_history),
+    "attention_scale_dropped": ("routed_attention", _attn_no_scale),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_mutation(name, monkeypatch):
+    attr, fn = MUTATIONS[name]
+    monkeypatch.setattr(O, attr, fn)
+    caught = []
+    for check in C.ALL_CHECKS:
+        try:
+            check()
+        except (AssertionError, ValueError, IndexError):
+            caught.append(check.__name__)
+    assert caught, f"no pin catches the planted mistake {name}"
