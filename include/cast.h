@@ -1,0 +1,241 @@
+/*
+ * cast.h - C ABI of the CAST per-block anchor/skip step on one GB300 (sm_103a).
+ *
+ * CAST (reconstruction-coupled acceleration of interactive world models) computes,
+ * at each eligible residual site of a transformer block, the update of the
+ * anchor frames directly and reconstructs the residual of every skipped frame
+ * from the two anchors that bracket it (Section 4.1, Eq. block).  This library
+ * runs the data-parallel hot path of that step:
+ *
+ *   cast_route_topk        pooled historical scoring and one-block omission
+ *                          scores, TopK of K history blocks per (anchor, head)
+ *                          (Section 4.4, Eqs. pooled, omission, topk)
+ *   cast_anchor_attention  anchor queries attend to the whole current chunk plus
+ *                          their routed history blocks (Eq. block, App. B.4)
+ *   cast_par_reconstruct   Phase-Aware Reconstruction of the skipped frames
+ *                          (Section 4.3, Eqs. cross, confidence, gate, fcpasm;
+ *                          App. A.2)
+ *   cast_block_step        the three in order at one attention residual site
+ *
+ * Conventions shared by every entry point
+ *   - Tensor pointers are DEVICE pointers owned by the caller; `anchors` and
+ *     `anchor_mask` are HOST arrays read during the call only.  The library
+ *     allocates no device memory: scratch comes from the caller's workspace,
+ *     sized by the matching cast_*_workspace_size() and at least 256-byte aligned.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL = the
+ *     legacy default stream).  No call synchronises the host with the device.
+ *   - Every call validates its arguments before launching anything.  On an
+ *     error nothing is written and a cast_status other than CAST_OK is
+ *     returned; cast_last_error_detail() gives a message for the calling thread.
+ *     CAST_ERR_CUDA reports a launch or runtime error seen after enqueuing.
+ *   - Kernels never wait without bound.  A wait that exceeds its limit makes the
+ *     kernel record an error word and return; the next call on this device that
+ *     finds the word set returns CAST_ERR_DEVICE_TIMEOUT (cast_check_device()
+ *     polls it explicitly; it synchronises `stream`).
+ *   - Layouts are row-major.  Token tensors are [frames, S, H, d] with d
+ *     contiguous and S = Hg * Wg tokens of a frame's latent grid in row-major
+ *     (y, x) order; the token row stride (elements between consecutive tokens)
+ *     must be >= H*d and a multiple of 8.  Residuals are channels-last
+ *     [F, Hg, Wg, C] (the attention output viewed per frame).
+ *   - bf16 is IEEE bfloat16 (round-to-nearest-even on output); f32 is IEEE float.
+ */
+#ifndef CAST_H_
+#define CAST_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int cast_status;
+#define CAST_OK 0
+#define CAST_ERR_INVALID_ARG 1     /* a shape, pointer, alignment or value is wrong */
+#define CAST_ERR_UNSUPPORTED 2     /* valid but outside what the kernels implement */
+#define CAST_ERR_CUDA 3            /* the CUDA runtime reported an error */
+#define CAST_ERR_DEVICE_TIMEOUT 4  /* a kernel gave up on a bounded wait */
+
+#define CAST_F32 0
+#define CAST_BF16 1
+
+#define CAST_ROUTE_OMISSION 0     /* TopK on u = ||P delta||^2 (Eq. omission), the paper's */
+#define CAST_ROUTE_SIMILARITY 1   /* TopK on the pooled similarity s (Eq. pooled) */
+
+#define CAST_GATE_PAPER 0         /* g from Eq. (gate) */
+#define CAST_GATE_ZERO 1          /* g = 0: direct value interpolation / extrapolation */
+#define CAST_GATE_ONE 2           /* g = 1: full endpoint phase transport */
+
+#define CAST_MAX_FRAMES 256       /* frames of one chunk (anchors + skipped) */
+#define CAST_MAX_ANCHORS 64
+
+/* ------------------------------------------------------------------------ */
+/* Routing: Section 4.4, Eqs. (pooled), (omission), (topk); App. B.1.        */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  /* queries of the current chunk, [n_frames, S, H, d]; only anchor frames are read */
+  const void* q;
+  int64_t q_row_stride;
+  int32_t n_frames, S, H, d;      /* d in {64, 128} */
+  int32_t dtype;                  /* dtype of q, k_hist, v_hist: CAST_BF16 or CAST_F32 */
+  const int32_t* anchors;         /* HOST, n_anchors strictly ascending frame indices */
+  int32_t n_anchors;
+  /* history blocks, [M, B_v, H, d]: block m is rows m*B_v .. m*B_v+B_v-1 */
+  const void* k_hist;
+  const void* v_hist;
+  int64_t hist_row_stride;
+  int32_t M, B_v;
+  /* Gram matrices G_h = P_h^T P_h of the output-projection head slices P = W_O^(h),
+     device f32 [H, d, d]; NULL means P = I (u = ||delta||^2) */
+  const float* gram;
+  int32_t K;                      /* budget K_KV; K_eff = min(K, M) blocks are kept */
+  float eps;                      /* stabiliser of Eq. (omission); 1e-8 by default */
+  int32_t mode;                   /* CAST_ROUTE_OMISSION | CAST_ROUTE_SIMILARITY */
+  /* outputs (device unless noted) */
+  int32_t* idx;                   /* [n_anchors, H, K_eff] ascending block indices */
+  float* u;                       /* optional [n_anchors, H, M] routing scores used for TopK */
+  float* qbar;                    /* optional [n_anchors, H, d] pooled queries */
+  float* kbar;                    /* optional [M, H, d] pooled keys */
+  float* vbar;                    /* optional [M, H, d] pooled values */
+  int32_t* k_eff;                 /* optional HOST: receives K_eff */
+} cast_route_args;
+
+/* Pooled mean statistics q_bar, k_bar, v_bar (mean over a frame's S tokens and over a
+ * block's B_v tokens, f32 accumulation), scores s = q_bar.k_bar / sqrt(d), pi = softmax
+ * over blocks, o_bar = sum pi v_bar, delta = pi/(1-pi+eps) (o_bar - v_bar),
+ * u = delta^T G delta; then per (anchor, head) the K_eff largest scores (ties to the
+ * lower block index), written in ascending block order.  K >= M keeps every block and
+ * M == 0 writes nothing (routing bypass, App. B.3).
+ * Errors: INVALID_ARG for NULL required pointers, n_anchors < 1 or > CAST_MAX_ANCHORS,
+ * anchors not ascending / out of range, K < 0, M < 0, B_v < 1 with M > 0, bad strides,
+ * a workspace smaller than cast_route_workspace_size(); UNSUPPORTED for d not 64/128. */
+cast_status cast_route_topk(const cast_route_args* args, void* workspace,
+                            size_t workspace_bytes, void* stream);
+size_t cast_route_workspace_size(const cast_route_args* args);
+
+/* ------------------------------------------------------------------------ */
+/* Routed anchor attention: Eq. (block), App. B.4, App. B.5.                 */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  const void* q;                  /* bf16 [n_frames, S, H, d], anchor rows are read */
+  const void* k_cur;              /* bf16 [n_frames, S, H, d] keys of the whole current chunk */
+  const void* v_cur;              /* bf16 [n_frames, S, H, d] */
+  int64_t q_row_stride, cur_row_stride;
+  int32_t n_frames, S, H, d;      /* d in {64, 128} */
+  const int32_t* anchors;         /* HOST, strictly ascending */
+  int32_t n_anchors;
+  const void* k_hist;             /* bf16 [M, B_v, H, d] */
+  const void* v_hist;
+  int64_t hist_row_stride;
+  int32_t M, B_v;
+  const int32_t* idx;             /* device [n_anchors, H, K_eff] routed blocks (any order) */
+  int32_t K_eff;                  /* 0 = current chunk only */
+  float scale;                    /* softmax scale; <= 0 means 1/sqrt(d) */
+  void* o;                        /* device [n_anchors, S, H*d], dtype o_dtype */
+  int32_t o_dtype;                /* CAST_BF16 or CAST_F32 */
+  float* lse;                     /* optional device f32 [n_anchors, H, S]: natural-log
+                                     log-sum-exp of the scaled logits of each query row */
+} cast_attn_args;
+
+/* O[i, s, h, :] = sum_j softmax_j(scale * q_i,s,h . k_j) v_j, where j runs over every
+ * token of the current chunk (no causal mask inside the chunk) and every token of the
+ * history blocks idx[i, h, :].  bf16 operands, f32 softmax and accumulation (Tab. config).
+ * Errors: INVALID_ARG for NULL pointers, bad shapes or strides, anchors not ascending,
+ * K_eff > 0 with M == 0; UNSUPPORTED for d not 64/128 or S*n_frames >= 2^31.
+ * Block indices outside [0, M) make the kernel record an error and skip that block. */
+cast_status cast_anchor_attention(const cast_attn_args* args, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* Phase-Aware Reconstruction: Section 4.3, Eqs. (cross), (confidence),      */
+/* (gate), (fcpasm); App. A.2.                                               */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  int32_t tile_h, tile_w;         /* disjoint spatial tiles, 1..8 tokens; 8x8 in the paper */
+  float tau_low, tau_high, q, T;  /* gate of Eq. (gate); (0.25, 0.75, 2, 0.10) in the paper */
+  float eps;                      /* 1e-8, Eq. (confidence) */
+  float eta_rel, eta_abs;         /* reliability threshold eta = eta_rel max W + eta_abs */
+  float band_radius;              /* < 0: every bin gated as in the paper; >= 0: bins whose
+                                     radius in 8x8-tile bin units exceeds it get g = 0 */
+  int32_t gate_mode;              /* CAST_GATE_PAPER | CAST_GATE_ZERO | CAST_GATE_ONE */
+} cast_par_params;
+
+/* Fills the paper's defaults (Tab. config_cast, App. A.2). */
+void cast_par_params_default(cast_par_params* p);
+
+typedef struct {
+  void* r;                        /* device [F, Hg, Wg, C] in/out: anchor frames read,
+                                     skipped frames overwritten */
+  int32_t dtype;                  /* CAST_F32 or CAST_BF16 */
+  int32_t F, Hg, Wg, C;           /* C a multiple of 8 */
+  const uint8_t* anchor_mask;     /* HOST [F]: nonzero = anchor */
+  const float* channel_weight;    /* optional device [C], >= 0; NULL = 1 */
+  cast_par_params params;
+} cast_par_args;
+
+/* For every skipped frame t with bracketing anchors (a, b) (frames outside the anchor
+ * span use the two nearest anchors and alpha < 0 or > 1), alpha = (t-a)/(b-a); per tile
+ * and channel F = RFFT2_ortho(R), Z = sum_c w_c F_b conj(F_a), W = sum_c w_c |F_b||F_a|,
+ * reliable bins W > eta and |Z| > eta, theta = Arg Z in (-pi, pi] on representatives
+ * (mirrors negated, self-conjugate bins 0), c = sum kappa|Z| / (sum kappa W + eps) over the
+ * reliable non-DC bins, g = sigmoid((c - tau(nu)) / T), and
+ * R_t = IRFFT2_ortho((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
+ * All frames anchors: nothing to do.  Errors: INVALID_ARG when a frame is skipped and
+ * fewer than two anchors exist, bad shapes or pointers, a short workspace;
+ * UNSUPPORTED for tile sides outside 1..8 or C not a multiple of 8. */
+cast_status cast_par_reconstruct(const cast_par_args* args, void* workspace,
+                                 size_t workspace_bytes, void* stream);
+size_t cast_par_workspace_size(const cast_par_args* args);
+
+/* ------------------------------------------------------------------------ */
+/* One block step at an attention residual site: Eq. (block), App. B.4.      */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  const void* q;                  /* bf16 [n_frames, S, H, d] */
+  const void* k_cur;
+  const void* v_cur;
+  int64_t q_row_stride, cur_row_stride;
+  int32_t n_frames, Hg, Wg, H, d; /* S = Hg * Wg */
+  const int32_t* anchors;         /* HOST, strictly ascending; n_anchors >= 2 unless
+                                     every frame is an anchor */
+  int32_t n_anchors;
+  const void* k_hist;             /* bf16 [M, B_v, H, d] */
+  const void* v_hist;
+  int64_t hist_row_stride;
+  int32_t M, B_v;
+  const float* gram;              /* optional, as in cast_route_args */
+  int32_t K;
+  float route_eps;
+  int32_t route_mode;
+  float scale;                    /* <= 0: 1/sqrt(d) */
+  void* r_out;                    /* device [n_frames, S, H*d]: anchor rows = attention
+                                     output, skipped rows = PAR reconstruction */
+  int32_t r_dtype;                /* CAST_BF16 or CAST_F32 */
+  void* x;                        /* optional device [n_frames, S, H*d] of r_dtype: x += r_out */
+  int32_t* idx_out;               /* optional device [n_anchors, H, min(K, M)] */
+  const float* channel_weight;    /* optional device [H*d] PAR channel weights */
+  cast_par_params par;
+} cast_block_args;
+
+/* route_topk -> anchor_attention -> par_reconstruct on one stream, then the optional
+ * residual update x += r_out.  Errors: those of the three steps. */
+cast_status cast_block_step(const cast_block_args* args, void* workspace,
+                            size_t workspace_bytes, void* stream);
+size_t cast_block_workspace_size(const cast_block_args* args);
+
+/* ------------------------------------------------------------------------ */
+/* Status                                                                    */
+/* ------------------------------------------------------------------------ */
+const char* cast_status_string(cast_status s);
+/* Message of the last error on the calling thread ("" if none). */
+const char* cast_last_error_detail(void);
+/* Synchronises `stream`, then reports CAST_ERR_DEVICE_TIMEOUT if a kernel on the current
+ * device recorded a bounded-wait timeout (and clears the record), CAST_ERR_CUDA on a
+ * pending CUDA error, CAST_OK otherwise. */
+cast_status cast_check_device(void* stream);
+/* Library version, "major.minor.patch". */
+const char* cast_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CAST_H_ */

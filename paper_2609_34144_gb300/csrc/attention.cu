@@ -1,0 +1,472 @@
+// Routed anchor attention on sm_103a tensor cores (Eq. block, App. B.4, App. B.5).
+//
+// One CTA computes a 128-row query tile of one (anchor i, head h):
+//   O = softmax(scale Q K^T) V over every token of the current chunk followed by the tokens
+//   of the routed history blocks idx[i, h, :].
+// Warp roles (192 threads):
+//   warp 0       TMA producer: Q once, then K / V tiles of 128 tokens into a 2-stage ring
+//                (128-byte swizzle, 64-element boxes), current-chunk tiles from a 2-D map,
+//                history tiles from a 3-D map [block, token, channel] so a tile never reads
+//                past its block (out-of-range rows arrive as zeros and are masked).
+//   warp 1       TMEM owner and single-thread UMMA issuer: S_j = Q K_j^T (M=128, N=128,
+//                kind::f16, f32 accumulate) into one of two TMEM S buffers, then
+//                O += P_{j-1} V_{j-1} (V read MN-major) into a TMEM O accumulator.
+//   warps 2..5   one query row per thread: tcgen05.ld of the S row, masking, online softmax
+//                in the exp2 domain with lazy rescaling (O and l are rescaled only when the
+//                running max grows by more than 8 = log2 256), P written to shared memory as
+//                bf16 in the 128-byte-swizzled K-major layout the UMMA reads, and the epilogue
+//                O / l (+ log-sum-exp).
+// Every wait is bounded; on a timeout the CTA records an error word and leaves.
+#include <cuda_bf16.h>
+
+#include <cmath>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace cast {
+namespace {
+
+__device__ unsigned int g_attn_error;
+
+constexpr int BM = 128, BN = 128, KST = 2;
+constexpr int kThreads = 192;
+constexpr float kRescaleThreshold = 8.f;
+
+template <int HD>
+struct Cfg {
+  static constexpr int Q_BYTES = BM * HD * 2;
+  static constexpr int KV_BYTES = BN * HD * 2;
+  static constexpr int P_BYTES = BM * BN * 2;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
+  static constexpr int OFF_P = OFF_V + KST * KV_BYTES;
+  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;   // + barriers + alignment slack
+};
+
+struct AttnKArgs {
+  int S, H, n_qt, n_anchors, n_cur_tiles, tiles_per_block, K_eff, M, cur_rows, B_v;
+  const int* idx;
+  void* o;
+  int o_f32;
+  float* lse;
+  float scale_log2;
+  unsigned long long wait_ns;
+  int q_frame[CAST_MAX_ANCHORS];
+  int o_frame[CAST_MAX_ANCHORS];
+};
+
+struct Bars {
+  uint64_t q_full;
+  uint64_t k_full[KST], k_empty[KST], v_full[KST], v_empty[KST];
+  uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
+  uint64_t fin;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ bool aborted(const Bars* b) {
+  return *reinterpret_cast<const volatile int*>(&b->abort) != 0;
+}
+__device__ __forceinline__ void set_abort(Bars* b) {
+  atomicExch(&b->abort, 1);
+  atomicExch(&g_attn_error, 1u);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_attn(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
+           const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kh,
+           const __grid_constant__ CUtensorMap tm_vh, const __grid_constant__ AttnKArgs a) {
+  using C = Cfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  uint8_t* sQ = smem + C::OFF_Q;
+  uint8_t* sK = smem + C::OFF_K;
+  uint8_t* sV = smem + C::OFF_V;
+  uint8_t* sP = smem + C::OFF_P;
+  Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // head slowest: CTAs resident together share the head's current-chunk K/V in L2
+  const int lin = blockIdx.x;
+  const int qt = lin % a.n_qt;
+  const int rest = lin / a.n_qt;
+  const int i = rest % a.n_anchors;
+  const int h = rest / a.n_anchors;
+  const int n_tiles = a.n_cur_tiles + a.K_eff * a.tiles_per_block;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bars->q_full, 1);
+    for (int s = 0; s < KST; ++s) {
+      mbar_init(&bars->k_full[s], 1);
+      mbar_init(&bars->k_empty[s], 1);
+      mbar_init(&bars->v_full[s], 1);
+      mbar_init(&bars->v_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bars->s_full[s], 1);
+      mbar_init(&bars->s_empty[s], 128);
+      mbar_init(&bars->p_full[s], 128);
+      mbar_init(&bars->p_empty[s], 1);
+    }
+    mbar_init(&bars->fin, 1);
+    bars->abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem_base, 512);
+    tmem_relinquish();
+    tc_fence_before();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  const uint64_t lim = a.wait_ns;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_kc);
+      tma_prefetch_desc(&tm_vc);
+      tma_prefetch_desc(&tm_kh);
+      tma_prefetch_desc(&tm_vh);
+      mbar_arrive_expect_tx(&bars->q_full, C::Q_BYTES);
+#pragma unroll
+      for (int b = 0; b < HD / 64; ++b)
+        tma_load_3d(sQ + b * BM * 128, &tm_q, &bars->q_full, h * HD + b * 64, qt * BM,
+                    a.q_frame[i]);
+      for (int j = 0; j < n_tiles; ++j) {
+        const bool cur = j < a.n_cur_tiles;
+        int y = 0, z = 0;
+        if (cur) {
+          y = j * BN;
+        } else {
+          const int jj = j - a.n_cur_tiles;
+          const int blk = jj / a.tiles_per_block;
+          y = (jj - blk * a.tiles_per_block) * BN;
+          z = a.idx[((int64_t)i * a.H + h) * a.K_eff + blk];
+          if (z < 0 || z >= a.M) {
+            atomicExch(&g_attn_error, 2u);
+            z = 0;
+          }
+        }
+        const int s = j % KST;
+        const uint32_t ph = (uint32_t)(j / KST) & 1u;
+        if (aborted(bars) || !mbar_wait(&bars->k_empty[s], ph ^ 1u, lim)) { set_abort(bars); break; }
+        mbar_arrive_expect_tx(&bars->k_full[s], C::KV_BYTES);
+#pragma unroll
+        for (int b = 0; b < HD / 64; ++b) {
+          uint8_t* dst = sK + s * C::KV_BYTES + b * BN * 128;
+          if (cur) tma_load_2d(dst, &tm_kc, &bars->k_full[s], h * HD + b * 64, y);
+          else tma_load_3d(dst, &tm_kh, &bars->k_full[s], h * HD + b * 64, y, z);
+        }
+        if (aborted(bars) || !mbar_wait(&bars->v_empty[s], ph ^ 1u, lim)) { set_abort(bars); break; }
+        mbar_arrive_expect_tx(&bars->v_full[s], C::KV_BYTES);
+#pragma unroll
+        for (int b = 0; b < HD / 64; ++b) {
+          uint8_t* dst = sV + s * C::KV_BYTES + b * BN * 128;
+          if (cur) tma_load_2d(dst, &tm_vc, &bars->v_full[s], h * HD + b * 64, y);
+          else tma_load_3d(dst, &tm_vh, &bars->v_full[s], h * HD + b * 64, y, z);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ UMMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, HD, false, true);
+      const uint32_t q_addr = smem_u32(sQ), k_addr = smem_u32(sK), v_addr = smem_u32(sV),
+                     p_addr = smem_u32(sP);
+      bool ok = mbar_wait(&bars->q_full, 0, lim);
+      if (!ok) set_abort(bars);
+      tc_fence_after();
+      auto issue_pv = [&](int jp) -> bool {
+        const int pb = jp & 1;
+        const int vs = jp % KST;
+        if (aborted(bars) || !mbar_wait(&bars->p_full[pb], (uint32_t)(jp >> 1) & 1u, lim)) return false;
+        if (!mbar_wait(&bars->v_full[vs], (uint32_t)(jp / KST) & 1u, lim)) return false;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const uint64_t ad =
+              sdesc_sw128(p_addr + pb * C::P_BYTES + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd = sdesc_sw128(v_addr + vs * C::KV_BYTES + kk * 16 * 128, BN * 128, 1024);
+          umma_bf16_ss(tmem + 256, ad, bd, idesc_pv, (jp > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&bars->v_empty[vs]);
+        umma_commit(&bars->p_empty[pb]);   // also signals "O includes P_jp V_jp"
+        return true;
+      };
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int sb = j & 1;
+        const int ks = j % KST;
+        if (aborted(bars) || !mbar_wait(&bars->s_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, lim) ||
+            !mbar_wait(&bars->k_full[ks], (uint32_t)(j / KST) & 1u, lim)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint64_t ad = sdesc_sw128(q_addr + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd =
+              sdesc_sw128(k_addr + ks * C::KV_BYTES + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024);
+          umma_bf16_ss(tmem + sb * BN, ad, bd, idesc_qk, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&bars->s_full[sb]);
+        umma_commit(&bars->k_empty[ks]);
+        if (j > 0 && !issue_pv(j - 1)) { ok = false; break; }
+      }
+      if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
+      if (!ok) set_abort(bars);
+      // drain: every issued UMMA has completed before TMEM is released
+      umma_commit(&bars->fin);
+      mbar_wait(&bars->fin, 0, lim);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax + epilogue
+    const int q4 = warp & 3;
+    const int row = q4 * 32 + lane;
+    const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n_tiles; ++j) {
+      const int sb = j & 1;
+      bool w = !aborted(bars) && mbar_wait(&bars->s_full[sb], (uint32_t)(j >> 1) & 1u, lim);
+      if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
+      tc_fence_after();
+      uint32_t sr[BN];
+      tmem_ld_x64(tl + sb * BN, sr);
+      tmem_ld_x64(tl + sb * BN + 64, sr + 64);
+      tc_fence_before();
+      mbar_arrive(&bars->s_empty[sb]);
+      int valid;
+      if (j < a.n_cur_tiles) {
+        valid = min(BN, a.cur_rows - j * BN);
+      } else {
+        const int jj = j - a.n_cur_tiles;
+        valid = min(BN, a.B_v - (jj % a.tiles_per_block) * BN);
+      }
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < BN; ++c) {
+        const float v = c < valid ? __uint_as_float(sr[c]) * a.scale_log2 : -INFINITY;
+        sr[c] = __float_as_uint(v);
+        mx = fmaxf(mx, v);
+      }
+      const bool need = mx > m_ref + kRescaleThreshold;
+      float corr = 1.f;
+      if (need) {
+        corr = exp2f(m_ref - mx);   // 0 on the first tile (m_ref = -inf)
+        m_ref = mx;
+        l *= corr;
+      }
+      if (j > 0 && __any_sync(0xffffffffu, need)) {
+        // O holds P_0..P_{j-1} V once PV_{j-1} has completed; its commit is the
+        // ((j-1)/2)-th completion of p_empty[(j-1)&1] (tracked phase by phase, never stale)
+        w = !aborted(bars) &&
+            mbar_wait(&bars->p_empty[(j - 1) & 1], (uint32_t)((j - 1) >> 1) & 1u, lim);
+        if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int half = 0; half < HD / 64; ++half) {
+          uint32_t orr[64];
+          tmem_ld_x64(tl + 256 + half * 64, orr);
+#pragma unroll
+          for (int c = 0; c < 64; ++c) orr[c] = __float_as_uint(__uint_as_float(orr[c]) * corr);
+          tmem_st_x64(tl + 256 + half * 64, orr);
+        }
+      }
+      // P buffer sb is free once PV_{j-2} has completed
+      w = !aborted(bars) && mbar_wait(&bars->p_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, lim);
+      if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
+      float sum = 0.f;
+      uint8_t* prow = sP + sb * C::P_BYTES + row * 128;
+#pragma unroll
+      for (int c16 = 0; c16 < BN / 8; ++c16) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float p0 = exp2f(__uint_as_float(sr[c16 * 8 + 2 * e]) - m_ref);
+          const float p1 = exp2f(__uint_as_float(sr[c16 * 8 + 2 * e + 1]) - m_ref);
+          sum += p0 + p1;
+          __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
+          pk[e] = *reinterpret_cast<uint32_t*>(&b2);
+        }
+        const int blk = c16 >> 3, c = c16 & 7;
+        *reinterpret_cast<uint4*>(prow + blk * (BM * 128) + ((c ^ (row & 7)) << 4)) =
+            make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+      l += sum;
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&bars->p_full[sb]);
+    }
+    if (ok && n_tiles > 0) {
+      const int jl = n_tiles - 1;
+      bool w = !aborted(bars) &&
+               mbar_wait(&bars->p_empty[jl & 1], (uint32_t)(jl >> 1) & 1u, lim);
+      ok = __all_sync(0xffffffffu, w);
+    }
+    if (!ok) {
+      set_abort(bars);
+    } else {
+      tc_fence_after();
+      const int s = qt * BM + row;
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      const int64_t D = (int64_t)a.H * HD;
+      const int64_t off = ((int64_t)a.o_frame[i] * a.S + s) * D + (int64_t)h * HD;
+#pragma unroll
+      for (int half = 0; half < HD / 64; ++half) {
+        uint32_t orr[64];
+        tmem_ld_x64(tl + 256 + half * 64, orr);   // warp-collective: every lane loads
+        if (s < a.S) {
+          if (a.o_f32) {
+            float* dst = static_cast<float*>(a.o) + off + half * 64;
+#pragma unroll
+            for (int c = 0; c < 64; c += 4)
+              *reinterpret_cast<float4*>(dst + c) =
+                  make_float4(__uint_as_float(orr[c]) * inv, __uint_as_float(orr[c + 1]) * inv,
+                              __uint_as_float(orr[c + 2]) * inv, __uint_as_float(orr[c + 3]) * inv);
+          } else {
+            __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(a.o) + off + half * 64;
+#pragma unroll
+            for (int c = 0; c < 64; c += 8) {
+              uint32_t pk4[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(orr[c + 2 * e]) * inv,
+                                                          __uint_as_float(orr[c + 2 * e + 1]) * inv);
+                pk4[e] = *reinterpret_cast<uint32_t*>(&b2);
+              }
+              *reinterpret_cast<uint4*>(dst + c) = make_uint4(pk4[0], pk4[1], pk4[2], pk4[3]);
+            }
+          }
+        }
+      }
+      {
+        if (a.lse && s < a.S)
+          a.lse[((int64_t)i * a.H + h) * a.S + s] = (m_ref + log2f(l)) * 0.69314718055994531f;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// bf16 tensor [depth][rows][inner] (rank 2 when depth == 0), box 64 x 128 (x 1), 128-B swizzle
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows,
+              uint64_t row_stride_bytes, uint64_t depth, uint64_t depth_stride_bytes) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {inner, rows, depth};
+  cuuint64_t strides[2] = {row_stride_bytes, depth_stride_bytes};
+  cuuint32_t box[3] = {64, 128, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  const cuuint32_t rank = depth ? 3 : 2;
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box,
+            es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int HD>
+cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream_t st) {
+  using C = Cfg<HD>;
+  const int D = a.H * HD;
+  CUtensorMap mq, mkc, mvc, mkh, mvh;
+  const uint64_t cur_rows = (uint64_t)a.n_frames * a.S;
+  bool ok = make_map(&mq, a.q, D, a.S, a.q_row_stride * 2, a.n_frames, (uint64_t)a.S * a.q_row_stride * 2) &&
+            make_map(&mkc, a.k_cur, D, cur_rows, a.cur_row_stride * 2, 0, 0) &&
+            make_map(&mvc, a.v_cur, D, cur_rows, a.cur_row_stride * 2, 0, 0);
+  if (ok && a.M > 0) {
+    ok = make_map(&mkh, a.k_hist, D, a.B_v, a.hist_row_stride * 2, a.M,
+                  (uint64_t)a.B_v * a.hist_row_stride * 2) &&
+         make_map(&mvh, a.v_hist, D, a.B_v, a.hist_row_stride * 2, a.M,
+                  (uint64_t)a.B_v * a.hist_row_stride * 2);
+  } else if (ok) {
+    mkh = mkc;
+    mvh = mvc;
+  }
+  if (!ok) return fail(CAST_ERR_CUDA, "attention: cuTensorMapEncodeTiled failed");
+  AttnKArgs k{};
+  k.S = a.S;
+  k.H = a.H;
+  k.n_qt = (a.S + BM - 1) / BM;
+  k.n_anchors = a.n_anchors;
+  k.n_cur_tiles = (int)((cur_rows + BN - 1) / BN);
+  k.tiles_per_block = a.M > 0 ? (a.B_v + BN - 1) / BN : 0;
+  k.K_eff = a.M > 0 ? a.K_eff : 0;
+  k.M = a.M;
+  k.cur_rows = (int)cur_rows;
+  k.B_v = a.B_v;
+  k.idx = a.idx;
+  k.o = a.o;
+  k.o_f32 = a.o_dtype == CAST_F32;
+  k.lse = a.lse;
+  const float scale = a.scale > 0.f ? a.scale : 1.f / sqrtf((float)HD);
+  k.scale_log2 = scale * 1.4426950408889634f;
+  k.wait_ns = 2000000000ull;
+  for (int j = 0; j < a.n_anchors; ++j) {
+    k.q_frame[j] = a.anchors[j];
+    k.o_frame[j] = o_frame_of_anchor ? a.anchors[j] : j;
+  }
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(k_attn<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
+        cudaSuccess)
+      return check_launch("attention smem attribute");
+    attr_set = true;
+  }
+  const int grid = k.n_qt * a.n_anchors * a.H;
+  k_attn<HD><<<grid, kThreads, C::SMEM, st>>>(mq, mkc, mvc, mkh, mvh, k);
+  return check_launch("attention kernel");
+}
+
+}  // namespace
+
+cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, cudaStream_t st) {
+  if (a.d == 128) return launch_hd<128>(a, o_frame_of_anchor, st);
+  return launch_hd<64>(a, o_frame_of_anchor, st);
+}
+
+unsigned int attention_error_word(cudaStream_t st, bool clear) {
+  unsigned int v = 0;
+  cudaMemcpyFromSymbolAsync(&v, g_attn_error, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  cudaStreamSynchronize(st);
+  if (clear && v) {
+    const unsigned int z = 0;
+    cudaMemcpyToSymbolAsync(g_attn_error, &z, sizeof(z), 0, cudaMemcpyHostToDevice, st);
+    cudaStreamSynchronize(st);
+  }
+  return v;
+}
+
+}  // namespace cast

@@ -1,0 +1,52 @@
+// Internal declarations shared by the translation units of libcast.
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "cast.h"
+
+namespace cast {
+
+// Records a printf-style message for cast_last_error_detail() and returns `s`.
+cast_status fail(cast_status s, const char* fmt, ...);
+// Converts a pending launch error into CAST_ERR_CUDA.
+cast_status check_launch(const char* what);
+
+constexpr size_t kWsAlign = 256;
+inline size_t align_up(size_t x, size_t a = kWsAlign) { return (x + a - 1) / a * a; }
+
+// ------------------------------------------------------------------ routing
+struct RoutePlan {
+  int n_seg;        // n_anchors + 2 M pooled segments
+  int nsplit;       // row splits per segment
+  size_t partial_bytes, pooled_bytes, total_bytes;
+};
+RoutePlan route_plan(const cast_route_args& a);
+// Arguments must have been validated; ws holds at least route_plan(a).total_bytes.
+cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st);
+
+// ------------------------------------------------------------------ attention
+// o_frame_of_anchor: 0 -> output frame i for anchor i (o is [n_anchors, S, H*d]);
+//                    1 -> output frame anchors[i] (o is [n_frames, S, H*d], block step).
+cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, cudaStream_t st);
+unsigned int attention_error_word(cudaStream_t st, bool clear);
+
+// ------------------------------------------------------------------ PAR
+struct ParPlan {
+  int n_anchor, n_pair, n_target;
+  int tiles_y, tiles_x, n_tile;
+  int chunk;        // channels per work item (= threads per CTA)
+  int n_chunk;
+  int slab_tiles, n_slab;
+  size_t partial_bytes, counter_bytes, total_bytes;
+};
+ParPlan par_plan(const cast_par_args& a);
+cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st);
+unsigned int par_error_word(cudaStream_t st, bool clear);
+
+// ------------------------------------------------------------------ residual update
+cast_status launch_residual_add(void* x, const void* r, int dtype, size_t n, cudaStream_t st);
+
+}  // namespace cast

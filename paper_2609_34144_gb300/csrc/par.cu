@@ -1,0 +1,499 @@
+// Phase-Aware Reconstruction of skipped frames (Section 4.3, Eqs. cross, confidence, gate,
+// fcpasm; App. A.2), one fused persistent kernel.
+//
+// Work is split into items (spectral tile p, channel chunk of 128 channels); one thread owns
+// one channel of the tile and keeps the 2-D spectrum of its h x w tokens in registers.
+//   stats item  : walks the anchors in order, forms each anchor's spectrum once, and for every
+//                 adjacent anchor pair with targets reduces Z = sum_c w_c F_b conj(F_a) and
+//                 W = sum_c w_c |F_b||F_a| over the chunk's channels into a partial record.
+//   recon item  : waits until every chunk of its tile has published its partials, walks the
+//                 anchors again (re-read mostly from L2), sums the partial records of each pair
+//                 in a fixed order, derives eta, reliability, principal phases, the tile
+//                 confidence c and the gate g, and for every target t of the pair writes
+//                 R_t = IRFFT2((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
+// Items are claimed from a ticket counter in an order where every stats item of a tile is
+// claimed before any recon item of that tile, so a waiting recon item only ever waits on
+// items already held by running CTAs (no deadlock); the wait is also bounded in time.
+#include <cuda_bf16.h>
+
+#include <cmath>
+
+#include "dft.cuh"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace cast {
+namespace {
+
+constexpr int kThreads = 128;      // channels per item
+constexpr int kNB = 40;            // stored bins of an 8-wide tile: 8 x 5
+constexpr int kNV = 3 * kNB;       // Re Z, Im Z, W per bin
+constexpr int kMaxSeg = 128;
+constexpr int kCoefBatch = 8;
+
+__device__ unsigned int g_par_error;   // nonzero: a recon item gave up waiting
+
+struct ParKArgs {
+  char* r;
+  const float* wch;
+  int dtype, F, Hg, Wg, C;
+  int th, tw, tiles_x, n_tile, n_chunk;
+  int n_anchor;
+  int anchor_frame[CAST_MAX_ANCHORS];
+  int pair_tbeg[CAST_MAX_ANCHORS + 1];   // targets of pair j (anchors j-1, j) in [tbeg[j], tbeg[j+1])
+  int target_frame[CAST_MAX_FRAMES];
+  float target_alpha[CAST_MAX_FRAMES];
+  int n_seg;
+  int seg_first[kMaxSeg + 1];            // first ticket of each segment
+  int seg_tile0[kMaxSeg];                // first tile of the segment's slab
+  unsigned char seg_recon[kMaxSeg];
+  int total_tickets;
+  float tau_low, tau_high, q, T, eps, eta_rel, eta_abs, band;
+  int gate_mode;
+  unsigned long long wait_ns;
+};
+
+__device__ __forceinline__ float ld_elem(const char* base, int64_t off, int dtype) {
+  if (dtype == CAST_BF16) {
+    const unsigned short b = __ldg(reinterpret_cast<const unsigned short*>(base) + off);
+    return __uint_as_float(((unsigned)b) << 16);
+  }
+  return __ldg(reinterpret_cast<const float*>(base) + off);
+}
+__device__ __forceinline__ void st_elem(char* base, int64_t off, int dtype, float v) {
+  if (dtype == CAST_BF16) {
+    __stcs(reinterpret_cast<__nv_bfloat16*>(base) + off, __float2bfloat16_rn(v));
+  } else {
+    __stcs(reinterpret_cast<float*>(base) + off, v);
+  }
+}
+
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+struct TileGeom {
+  int y0, x0, h, w;
+};
+
+__device__ __forceinline__ TileGeom tile_geom(const ParKArgs& a, int tile) {
+  TileGeom g;
+  const int ty = tile / a.tiles_x, tx = tile - ty * a.tiles_x;
+  g.y0 = ty * a.th;
+  g.x0 = tx * a.tw;
+  g.h = min(a.th, a.Hg - g.y0);
+  g.w = min(a.tw, a.Wg - g.x0);
+  return g;
+}
+
+// Loads one channel of an h x w tile of frame f (zeros outside the tile or channel range).
+__device__ __forceinline__ void load_tile(const ParKArgs& a, int f, const TileGeom& g, int c,
+                                          bool active, float (&x)[8][8]) {
+  const int64_t rowC = (int64_t)a.Wg * a.C;
+  const int64_t base = ((int64_t)f * a.Hg + g.y0) * rowC + (int64_t)g.x0 * a.C + c;
+#pragma unroll
+  for (int y = 0; y < 8; ++y)
+#pragma unroll
+    for (int xx = 0; xx < 8; ++xx)
+      x[y][xx] = (active && y < g.h && xx < g.w) ? ld_elem(a.r, base + y * rowC + xx * a.C, a.dtype)
+                                                 : 0.f;
+}
+
+// Warp transpose-reduction of 32 values: lane l returns the warp sum of v[l].
+__device__ __forceinline__ float warp_transpose_sum(float (&v)[32], int lane) {
+#pragma unroll
+  for (int off = 16, n = 16; off > 0; off >>= 1, n >>= 1) {
+    const bool hi = (lane & off) != 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (i < n) {
+        const float send = hi ? v[i] : v[i + n];
+        const float keep = hi ? v[i + n] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+      }
+    }
+  }
+  return v[0];
+}
+
+// value index vi in [0, 120): component vi / 40 (0: Re Z, 1: Im Z, 2: W) of bin vi % 40
+__device__ __forceinline__ float stat_value(int vi, float wc, const float* fa, const float* fb,
+                                            int tid) {
+  const int comp = vi / kNB, b = vi % kNB;
+  const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
+  const float br = fb[(2 * b) * kThreads + tid], bi = fb[(2 * b + 1) * kThreads + tid];
+  if (comp == 0) return wc * (br * ar + bi * ai);
+  if (comp == 1) return wc * (bi * ar - br * ai);
+  return wc * sqrtf((ar * ar + ai * ai) * (br * br + bi * bi));
+}
+
+// Per-tile transport of one anchor pair (warp 0): theta and g per stored bin.
+__device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float* zw, float* th,
+                               float* gate, float* own_th, int* own_rel, int lane) {
+  const float inv_hw = 1.f / (float)(g.h * g.w);
+  const int hw2 = g.w / 2;
+  float Zr[2], Zi[2], Wv[2], Za[2];
+  bool valid[2];
+  float wmax = 0.f;
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    const int b = lane + 32 * s;
+    const int ky = b / 5, kx = b % 5;
+    valid[s] = b < kNB && ky < g.h && kx <= hw2;
+    Zr[s] = valid[s] ? zw[b] * inv_hw : 0.f;
+    Zi[s] = valid[s] ? zw[kNB + b] * inv_hw : 0.f;
+    Wv[s] = valid[s] ? zw[2 * kNB + b] * inv_hw : 0.f;
+    Za[s] = sqrtf(Zr[s] * Zr[s] + Zi[s] * Zi[s]);
+    if (valid[s]) wmax = fmaxf(wmax, Wv[s]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) wmax = fmaxf(wmax, __shfl_xor_sync(0xffffffffu, wmax, o));
+  const float eta = a.eta_rel * wmax + a.eta_abs;
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    const int b = lane + 32 * s;
+    if (b < kNB) {
+      float t = atan2f(Zi[s], Zr[s]);
+      if (t <= -3.14159265358979f) t = 3.14159265358979f;   // principal branch (-pi, pi]
+      own_th[b] = t;
+      own_rel[b] = valid[s] && Wv[s] > eta && Za[s] > eta;
+    }
+  }
+  __syncwarp();
+  float num = 0.f, den = 0.f;
+  int any = 0;
+  float thv[2];
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    const int b = lane + 32 * s;
+    const int ky = b / 5, kx = b % 5;
+    const bool edge = kx == 0 || ((g.w % 2 == 0) && kx == hw2);
+    const bool selfc = edge && (ky == 0 || ((g.h % 2 == 0) && 2 * ky == g.h));
+    const bool mirror = edge && !selfc && 2 * ky > g.h;
+    const int rep = mirror ? (g.h - ky) * 5 + kx : b;
+    const bool rel = valid[s] && b < kNB && own_rel[rep < kNB ? rep : 0];
+    float t = (b < kNB) ? own_th[rep < kNB ? rep : 0] : 0.f;
+    if (mirror) t = -t;
+    if (!rel || selfc) t = 0.f;
+    thv[s] = t;
+    if (rel && b != 0) {
+      const float kap = edge ? 1.f : 2.f;
+      num += kap * Za[s];
+      den += kap * Wv[s];
+      any = 1;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    num += __shfl_xor_sync(0xffffffffu, num, o);
+    den += __shfl_xor_sync(0xffffffffu, den, o);
+    any |= __shfl_xor_sync(0xffffffffu, any, o);
+  }
+  const float c = any ? num / (den + a.eps) : 0.f;
+  const float hh = (float)(g.h / 2) / (float)g.h, ww = (float)hw2 / (float)g.w;
+  const float rmax = sqrtf(hh * hh + ww * ww);
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    const int b = lane + 32 * s;
+    if (b >= kNB) continue;
+    const int ky = b / 5, kx = b % 5;
+    const int kys = ky <= (g.h - 1) / 2 ? ky : ky - g.h;
+    const float fy = (float)kys / (float)g.h, fx = (float)kx / (float)g.w;
+    const float nu = rmax > 0.f ? sqrtf(fy * fy + fx * fx) / rmax : 0.f;
+    const float tau = a.tau_low + (a.tau_high - a.tau_low) * powf(nu, a.q);
+    float gv = 1.f / (1.f + expf(-(c - tau) / a.T));
+    if (a.gate_mode == CAST_GATE_ZERO) gv = 0.f;
+    if (a.gate_mode == CAST_GATE_ONE) gv = 1.f;
+    if (a.band >= 0.f) {
+      const float ry = (float)kys * 8.f / (float)g.h, rx = (float)kx * 8.f / (float)g.w;
+      if (sqrtf(ry * ry + rx * rx) > a.band) gv = 0.f;
+    }
+    th[b] = any ? thv[s] : 0.f;
+    gate[b] = gv;
+  }
+}
+
+constexpr int kSpecFloats = 2 * kNB * kThreads;   // one spectrum per thread, [value][thread]
+constexpr size_t kParDynSmem = 2 * kSpecFloats * sizeof(float);
+
+__global__ void __launch_bounds__(kThreads, 2)
+    k_par(const __grid_constant__ ParKArgs a, float* __restrict__ partial,
+          unsigned* __restrict__ counters) {
+  extern __shared__ float s_spec[];   // spectra of anchors j-1 and j: s_spec[(j & 1) * kSpecFloats + ...]
+  __shared__ float s_red[kThreads / 32][128];
+  __shared__ float s_zw[kNV];
+  __shared__ float s_th[kNB], s_g[kNB], s_own_th[kNB];
+  __shared__ int s_own_rel[kNB];
+  __shared__ float4 s_coef[kCoefBatch][kNB];
+  __shared__ int s_ticket;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+  for (;;) {
+    if (tid == 0) s_ticket = (int)atomicAdd(&counters[0], 1u);
+    __syncthreads();
+    const int t = s_ticket;
+    __syncthreads();
+    if (t >= a.total_tickets) break;
+    int q = 0;
+    while (q + 1 < a.n_seg && a.seg_first[q + 1] <= t) ++q;
+    const int local = t - a.seg_first[q];
+    const int tile = a.seg_tile0[q] + local / a.n_chunk;
+    const int chunk = local % a.n_chunk;
+    const bool recon = a.seg_recon[q] != 0;
+    const TileGeom g = tile_geom(a, tile);
+    const int c = chunk * kThreads + tid;
+    const bool active = c < a.C;
+    const float wc = active ? (a.wch ? __ldg(a.wch + c) : 1.f) : 0.f;
+
+    if (recon) {
+      // wait (bounded) until every chunk of this tile has published its partials
+      if (tid == 0) {
+        const uint64_t t0 = global_ns();
+        while (ld_acquire(&counters[1 + tile]) < (unsigned)a.n_chunk) {
+          if (global_ns() - t0 > a.wait_ns) {
+            atomicExch(&g_par_error, 1u);
+            break;
+          }
+          __nanosleep(128);
+        }
+      }
+      __syncthreads();
+    }
+
+    for (int j = 0; j < a.n_anchor; ++j) {
+      float* fb = s_spec + (j & 1) * kSpecFloats;        // this anchor (thread-private column)
+      const float* fa = s_spec + ((j + 1) & 1) * kSpecFloats;   // previous anchor
+      {
+        float x[8][8], re[8][5], im[8][5];
+        load_tile(a, a.anchor_frame[j], g, c, active, x);
+        dft::fwd2d(x, g.h, g.w, re, im);
+#pragma unroll
+        for (int b = 0; b < kNB; ++b) {
+          fb[(2 * b) * kThreads + tid] = re[b / 5][b % 5];
+          fb[(2 * b + 1) * kThreads + tid] = im[b / 5][b % 5];
+        }
+      }
+      const bool has_targets = j > 0 && a.pair_tbeg[j + 1] > a.pair_tbeg[j];
+      if (has_targets && !recon) {
+        // ---- partial Z, W of pair (j-1, j) over this chunk's channels
+#pragma unroll
+        for (int grp = 0; grp < 4; ++grp) {
+          float v[32];
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const int vi = grp * 32 + e;
+            v[e] = vi < kNV ? stat_value(vi, wc, fa, fb, tid) : 0.f;
+          }
+          s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
+        }
+        __syncthreads();
+        if (tid < kNV) {
+          float s = 0.f;
+#pragma unroll
+          for (int w = 0; w < kThreads / 32; ++w) s += s_red[w][tid];
+          partial[(((int64_t)j * a.n_tile + tile) * a.n_chunk + chunk) * kNV + tid] = s;
+        }
+        __syncthreads();
+      } else if (has_targets && recon) {
+        // ---- transport of pair (j-1, j) on this tile
+        if (tid < kNV) {
+          float s = 0.f;
+          const float* p = partial + ((int64_t)j * a.n_tile + tile) * a.n_chunk * kNV + tid;
+          for (int k = 0; k < a.n_chunk; ++k) s += __ldcg(p + (int64_t)k * kNV);
+          s_zw[tid] = s;
+        }
+        __syncthreads();
+        if (warp == 0) tile_transport(a, g, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
+        __syncthreads();
+        const float inv_hw = 1.f / (float)(g.h * g.w);
+        for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += kCoefBatch) {
+          const int nt = min(kCoefBatch, a.pair_tbeg[j + 1] - t0);
+          for (int e = tid; e < nt * kNB; e += kThreads) {
+            const int k = e / kNB, b = e % kNB;
+            const float al = a.target_alpha[t0 + k];
+            float sa, ca, sb, cb;
+            sincosf(s_g[b] * al * s_th[b], &sa, &ca);
+            sincosf(-s_g[b] * (1.f - al) * s_th[b], &sb, &cb);
+            const float fa = (1.f - al) * inv_hw, fb = al * inv_hw;
+            s_coef[k][b] = make_float4(fa * ca, fa * sa, fb * cb, fb * sb);
+          }
+          __syncthreads();
+          for (int k = 0; k < nt; ++k) {
+            float hr[8][5], hi[8][5];
+#pragma unroll
+            for (int b = 0; b < kNB; ++b) {
+              const int ky = b / 5, kx = b % 5;
+              const float4 cf = s_coef[k][b];
+              const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
+              const float br = fb[(2 * b) * kThreads + tid], bi = fb[(2 * b + 1) * kThreads + tid];
+              hr[ky][kx] = cf.x * ar - cf.y * ai + cf.z * br - cf.w * bi;
+              hi[ky][kx] = cf.x * ai + cf.y * ar + cf.z * bi + cf.w * br;
+            }
+            float y[8][8];
+            dft::inv2d(hr, hi, g.h, g.w, y);
+            if (active) {
+              const int tf = a.target_frame[t0 + k];
+              const int64_t rowC = (int64_t)a.Wg * a.C;
+              const int64_t base = ((int64_t)tf * a.Hg + g.y0) * rowC + (int64_t)g.x0 * a.C + c;
+#pragma unroll
+              for (int yy = 0; yy < 8; ++yy)
+#pragma unroll
+                for (int xx = 0; xx < 8; ++xx)
+                  if (yy < g.h && xx < g.w) st_elem(a.r, base + yy * rowC + xx * a.C, a.dtype, y[yy][xx]);
+            }
+          }
+          __syncthreads();
+        }
+      }
+    }
+    if (!recon) {
+      __syncthreads();
+      if (tid == 0) {
+        __threadfence();
+        atomicAdd(&counters[1 + tile], 1u);
+      }
+    }
+  }
+}
+
+}  // namespace
+
+ParPlan par_plan(const cast_par_args& a) {
+  ParPlan p{};
+  int na = 0;
+  for (int f = 0; f < a.F; ++f) na += a.anchor_mask[f] ? 1 : 0;
+  p.n_anchor = na;
+  p.n_pair = na > 0 ? na - 1 : 0;
+  p.n_target = a.F - na;
+  const int th = a.params.tile_h, tw = a.params.tile_w;
+  p.tiles_y = (a.Hg + th - 1) / th;
+  p.tiles_x = (a.Wg + tw - 1) / tw;
+  p.n_tile = p.tiles_y * p.tiles_x;
+  p.chunk = kThreads;
+  p.n_chunk = (a.C + kThreads - 1) / kThreads;
+  // slab: tiles whose anchor bytes stay well inside L2 between the stats and recon passes
+  const double elt = a.dtype == CAST_BF16 ? 2.0 : 4.0;
+  const double tile_bytes = (double)na * th * tw * a.C * elt;
+  int slab = (int)(24.0e6 / (tile_bytes > 1 ? tile_bytes : 1));
+  if (slab < 1) slab = 1;
+  if (slab > p.n_tile) slab = p.n_tile;
+  while ((p.n_tile + slab - 1) / slab > kMaxSeg / 2) ++slab;
+  p.slab_tiles = slab;
+  p.n_slab = (p.n_tile + slab - 1) / slab;
+  p.partial_bytes = align_up((size_t)(na > 0 ? na : 1) * p.n_tile * p.n_chunk * kNV * sizeof(float));
+  p.counter_bytes = align_up((size_t)(1 + p.n_tile) * sizeof(unsigned));
+  p.total_bytes = p.partial_bytes + p.counter_bytes;
+  return p;
+}
+
+cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
+  const ParPlan p = par_plan(a);
+  if (p.n_target == 0) return CAST_OK;   // every frame is an anchor: reconstruction bypassed
+  ParKArgs k{};
+  k.r = static_cast<char*>(a.r);
+  k.wch = a.channel_weight;
+  k.dtype = a.dtype;
+  k.F = a.F;
+  k.Hg = a.Hg;
+  k.Wg = a.Wg;
+  k.C = a.C;
+  k.th = a.params.tile_h;
+  k.tw = a.params.tile_w;
+  k.tiles_x = p.tiles_x;
+  k.n_tile = p.n_tile;
+  k.n_chunk = p.n_chunk;
+  int anchors[CAST_MAX_FRAMES];
+  int na = 0;
+  for (int f = 0; f < a.F; ++f)
+    if (a.anchor_mask[f]) anchors[na++] = f;
+  k.n_anchor = na;
+  for (int j = 0; j < na; ++j) k.anchor_frame[j] = anchors[j];
+  // targets grouped by pair j (anchors j-1, j), j = 1..na-1 (Eq. block)
+  int nt = 0;
+  for (int j = 0; j <= na; ++j) k.pair_tbeg[j] = 0;
+  for (int j = 1; j < na; ++j) {
+    k.pair_tbeg[j] = nt;
+    const int a0 = anchors[j - 1], a1 = anchors[j];
+    auto add = [&](int t) {
+      k.target_frame[nt] = t;
+      k.target_alpha[nt] = (float)((double)(t - a0) / (double)(a1 - a0));
+      ++nt;
+    };
+    if (j == 1)
+      for (int t = 0; t < a0; ++t) add(t);
+    for (int t = a0 + 1; t < a1; ++t) add(t);
+    if (j == na - 1)
+      for (int t = a1 + 1; t < a.F; ++t) add(t);
+  }
+  k.pair_tbeg[na] = nt;
+  k.pair_tbeg[0] = 0;
+  // ticket schedule: S(0), S(1), R(0), S(2), R(1), ..., R(n-1)
+  int nseg = 0, ticket = 0;
+  auto seg = [&](int slab, bool recon) {
+    const int t0 = slab * p.slab_tiles;
+    const int nt_ = (t0 + p.slab_tiles <= p.n_tile ? p.slab_tiles : p.n_tile - t0);
+    k.seg_first[nseg] = ticket;
+    k.seg_tile0[nseg] = t0;
+    k.seg_recon[nseg] = recon ? 1 : 0;
+    ticket += nt_ * p.n_chunk;
+    ++nseg;
+  };
+  seg(0, false);
+  for (int s = 1; s < p.n_slab; ++s) {
+    seg(s, false);
+    seg(s - 1, true);
+  }
+  seg(p.n_slab - 1, true);
+  k.n_seg = nseg;
+  k.seg_first[nseg] = ticket;
+  k.total_tickets = ticket;
+  const cast_par_params& pp = a.params;
+  k.tau_low = pp.tau_low;
+  k.tau_high = pp.tau_high;
+  k.q = pp.q;
+  k.T = pp.T;
+  k.eps = pp.eps;
+  k.eta_rel = pp.eta_rel;
+  k.eta_abs = pp.eta_abs;
+  k.band = pp.band_radius;
+  k.gate_mode = pp.gate_mode;
+  k.wait_ns = 2000000000ull;
+
+  char* w = static_cast<char*>(ws);
+  float* partial = reinterpret_cast<float*>(w);
+  unsigned* counters = reinterpret_cast<unsigned*>(w + p.partial_bytes);
+  if (cudaMemsetAsync(counters, 0, (size_t)(1 + p.n_tile) * sizeof(unsigned), st) != cudaSuccess)
+    return check_launch("PAR counter reset");
+  int dev = 0, nsm = 0, occ = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(k_par, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kParDynSmem) !=
+        cudaSuccess)
+      return check_launch("PAR smem attribute");
+    attr_set = true;
+  }
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_par, kThreads, kParDynSmem);
+  if (occ < 1) occ = 1;
+  int grid = nsm * occ;
+  if (grid > ticket) grid = ticket;
+  k_par<<<grid, kThreads, kParDynSmem, st>>>(k, partial, counters);
+  return check_launch("PAR kernel");
+}
+
+unsigned int par_error_word(cudaStream_t st, bool clear) {
+  unsigned int v = 0;
+  cudaMemcpyFromSymbolAsync(&v, g_par_error, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  cudaStreamSynchronize(st);
+  if (clear && v) {
+    const unsigned int z = 0;
+    cudaMemcpyToSymbolAsync(g_par_error, &z, sizeof(z), 0, cudaMemcpyHostToDevice, st);
+    cudaStreamSynchronize(st);
+  }
+  return v;
+}
+
+}  // namespace cast

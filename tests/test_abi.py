@@ -1,0 +1,152 @@
+"""The C ABI on the CPU: the library loads, exports every function include/cast.h declares, and
+rejects bad arguments with the documented status before any CUDA call (no GPU needed)."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "cast.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    names = re.findall(r"\b(cast_[a-z_]+)\s*\(", src)
+    return sorted(set(names))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_34144_gb300 import native
+    return native
+
+
+def test_header_declares_the_entry_points():
+    d = _declared()
+    for n in ("cast_route_topk", "cast_anchor_attention", "cast_par_reconstruct", "cast_block_step"):
+        assert n in d
+
+
+def test_every_declared_symbol_is_exported(lib):
+    so = lib.library()
+    for name in _declared():
+        assert hasattr(so, name), name
+    assert set(_declared()) <= set(lib.EXPORTED) | {"cast_version"}
+
+
+def test_status_strings(lib):
+    so = lib.library()
+    assert so.cast_status_string(0) == b"CAST_OK"
+    assert so.cast_status_string(4) == b"CAST_ERR_DEVICE_TIMEOUT"
+
+
+def test_default_params_are_the_papers(lib):
+    p = lib.default_par_params()
+    assert (p.tile_h, p.tile_w) == (8, 8)
+    assert abs(p.tau_low - 0.25) < 1e-7 and abs(p.tau_high - 0.75) < 1e-7
+    assert abs(p.q - 2.0) < 1e-7 and abs(p.T - 0.10) < 1e-7
+    assert abs(p.eta_rel - 1e-6) < 1e-12 and abs(p.eta_abs - 1e-8) < 1e-14
+    assert p.band_radius < 0 and p.gate_mode == lib.GATE_PAPER
+
+
+def _fake(addr=0x10000):
+    return C.c_void_p(addr)
+
+
+def _route(lib, **kw):
+    a = lib.RouteArgs()
+    a.q = _fake()
+    a.q_row_stride = 256
+    a.n_frames, a.S, a.H, a.d = 3, 16, 2, 128
+    a.dtype = lib.BF16
+    anchors = kw.pop("anchors", [0, 2])
+    a._an = (C.c_int32 * len(anchors))(*anchors)
+    a.anchors = C.cast(a._an, C.POINTER(C.c_int32))
+    a.n_anchors = len(anchors)
+    a.k_hist, a.v_hist = _fake(0x20000), _fake(0x30000)
+    a.hist_row_stride = 256
+    a.M, a.B_v, a.K, a.eps, a.mode = 4, 8, 2, 1e-8, 0
+    a.idx = _fake(0x40000)
+    for k, v in kw.items():
+        setattr(a, k, v)
+    return a
+
+
+@pytest.mark.parametrize("bad,status", [
+    ({"anchors": [2, 0]}, 1),
+    ({"anchors": [0, 5]}, 1),
+    ({"d": 96}, 2),
+    ({"q_row_stride": 100}, 1),
+    ({"q": _fake(0x10008)}, 1),
+    ({"K": -1}, 1),
+    ({"mode": 7}, 1),
+])
+def test_route_validation(lib, bad, status):
+    a = _route(lib, **bad)
+    ws = C.create_string_buffer(16)
+    assert lib.library().cast_route_topk(C.byref(a), ws, 0, None) == status
+    assert lib.library().cast_last_error_detail() != b""
+
+
+def test_route_short_workspace_is_rejected(lib):
+    a = _route(lib)
+    need = lib.library().cast_route_workspace_size(C.byref(a))
+    assert need > 0
+    assert lib.library().cast_route_topk(C.byref(a), _fake(0x100000), need - 1, None) == 1
+
+
+def _par(lib, mask, **kw):
+    a = lib.ParArgs()
+    a.r = _fake()
+    a.dtype = lib.F32
+    a.F, a.Hg, a.Wg, a.C = len(mask), 16, 16, 64
+    a._m = (C.c_uint8 * len(mask))(*mask)
+    a.anchor_mask = C.cast(a._m, C.POINTER(C.c_uint8))
+    a.params = lib.default_par_params()
+    for k, v in kw.items():
+        if k.startswith("p_"):
+            setattr(a.params, k[2:], v)
+        else:
+            setattr(a, k, v)
+    return a
+
+
+@pytest.mark.parametrize("mask,kw,status", [
+    ([1, 0, 0], {}, 1),                   # one anchor with skipped frames (Eq. block needs two)
+    ([1, 0, 1], {"C": 60}, 2),            # channels not a multiple of 8
+    ([1, 0, 1], {"p_tile_h": 9}, 2),      # tile side above 8
+    ([1, 0, 1], {"p_T": 0.0}, 1),         # gate temperature must be positive
+    ([1, 0, 1], {"p_gate_mode": 5}, 1),
+    ([1, 0, 1], {"dtype": 9}, 1),
+])
+def test_par_validation(lib, mask, kw, status):
+    a = _par(lib, mask, **kw)
+    assert lib.library().cast_par_reconstruct(C.byref(a), _fake(0x100000), 1 << 30, None) == status
+
+
+def test_par_all_anchors_needs_nothing(lib):
+    a = _par(lib, [1, 1, 1])
+    # nothing to reconstruct: returns OK before touching the device
+    assert lib.library().cast_par_reconstruct(C.byref(a), None, 0, None) == 0
+
+
+def test_par_workspace_grows_with_channels(lib):
+    s1 = lib.library().cast_par_workspace_size(C.byref(_par(lib, [1, 0, 1])))
+    s2 = lib.library().cast_par_workspace_size(C.byref(_par(lib, [1, 0, 1], C=512)))
+    assert 0 < s1 < s2
+
+
+def test_attention_validation(lib):
+    a = lib.AttnArgs()
+    a.q = a.k_cur = a.v_cur = _fake()
+    a.q_row_stride = a.cur_row_stride = 256
+    a.n_frames, a.S, a.H, a.d = 2, 16, 2, 128
+    an = (C.c_int32 * 1)(1)
+    a.anchors = C.cast(an, C.POINTER(C.c_int32))
+    a.n_anchors = 1
+    a.M, a.B_v, a.K_eff = 0, 1, 1          # routed blocks without history
+    a.o, a.o_dtype = _fake(), lib.BF16
+    assert lib.library().cast_anchor_attention(C.byref(a), None) == 1
+    a.K_eff, a.d = 0, 80
+    assert lib.library().cast_anchor_attention(C.byref(a), None) == 2

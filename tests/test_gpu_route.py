@@ -1,0 +1,124 @@
+"""Routing kernels (cast_route_topk) against the CPU oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle.cast_oracle as O
+from synthetic import generators as G
+from synthetic import workloads as W
+from tests.gpu_util import TOPK_GAP, to_dev, to_host
+
+pytestmark = pytest.mark.gpu
+
+
+def _inputs(seed, N, S, H, d, M, Bv, dtype):
+    ss = np.random.SeedSequence(seed)
+    a, b, c = ss.spawn(3)
+    q = G.tokens_with_offsets(a, N, S, H, d, 1.0)
+    k = G.tokens_with_offsets(b, M, Bv, H, d, 1.0)
+    v = G.tokens_with_offsets(c, M, Bv, H, d, 1.0)
+    if dtype == "bf16":
+        q, k, v = G.round_bf16(q), G.round_bf16(k), G.round_bf16(v)
+    return q, k, v
+
+
+def check_idx(idx_gpu, score_ref, K):
+    """Sets match wherever the oracle's relative gap at the K boundary exceeds TOPK_GAP;
+    elsewhere only blocks outside the ambiguous band must agree.  Returns #ambiguous."""
+    ref = O.topk_blocks(score_ref, K)
+    gap = O.topk_margin(score_ref, K)
+    amb = 0
+    for r in np.ndindex(ref.shape[:-1]):
+        g = idx_gpu[r]
+        assert np.all(np.diff(g) > 0), "indices not strictly ascending"
+        if gap[r] > TOPK_GAP:
+            assert np.array_equal(g, ref[r]), (r, g, ref[r])
+        else:
+            amb += 1
+            s = score_ref[r]
+            kth = np.sort(s)[::-1][K - 1]
+            lo, hi = kth - TOPK_GAP * abs(kth), kth + TOPK_GAP * abs(kth)
+            assert set(np.flatnonzero(s > hi)) <= set(g.tolist())
+            assert not (set(np.flatnonzero(s < lo)) & set(g.tolist()))
+    return amb
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("d", [64, 128])
+def test_route_small(lib, dtype, d):
+    N, S, H, M, Bv, K = 3, 50, 3, 7, 37, 3
+    q, k, v = _inputs(10 + d, N, S, H, d, M, Bv, dtype)
+    anchors = [0, 2]
+    idx, u, (qb, kb, vb) = lib.cast_route_topk(to_dev(q, dtype), anchors, to_dev(k, dtype),
+                                                to_dev(v, dtype), K, want_u=True, want_pooled=True)
+    torch.cuda.synchronize()
+    rt = O.pooled_routing(q, anchors, k, v)
+    np.testing.assert_allclose(to_host(qb), rt.qbar, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(to_host(kb), rt.kbar, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(to_host(vb), rt.vbar, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(to_host(u), rt.u, rtol=2e-4, atol=1e-7 * rt.u.max())
+    amb = check_idx(idx.cpu().numpy(), rt.u, K)
+    assert amb == 0
+
+
+def test_route_gram_projection(lib):
+    """GPU with G = P^T P equals the oracle's literal ||P delta||^2 (Eq. omission)."""
+    N, S, H, d, M, Bv, K = 2, 64, 2, 64, 9, 40, 4
+    q, k, v = _inputs(21, N, S, H, d, M, Bv, "bf16")
+    P = np.random.default_rng(5).standard_normal((H, d, d)) / np.sqrt(d)
+    gram = np.einsum("hod,hoe->hde", P, P).astype(np.float32)
+    idx, u = lib.cast_route_topk(to_dev(q, "bf16"), [1], to_dev(k, "bf16"), to_dev(v, "bf16"), K,
+                                 gram=torch.from_numpy(gram).cuda(), want_u=True)
+    torch.cuda.synchronize()
+    rt = O.pooled_routing(q, [1], k, v, proj=P)
+    np.testing.assert_allclose(to_host(u), rt.u, rtol=5e-4, atol=1e-7 * rt.u.max())
+    check_idx(idx.cpu().numpy(), rt.u, K)
+
+
+def test_route_similarity_mode(lib):
+    N, S, H, d, M, Bv, K = 2, 33, 2, 128, 11, 20, 5
+    q, k, v = _inputs(22, N, S, H, d, M, Bv, "bf16")
+    idx, s = lib.cast_route_topk(to_dev(q, "bf16"), [0, 1], to_dev(k, "bf16"), to_dev(v, "bf16"), K,
+                                 mode=lib.ROUTE_SIMILARITY, want_u=True)
+    torch.cuda.synchronize()
+    rt = O.pooled_routing(q, [0, 1], k, v)
+    np.testing.assert_allclose(to_host(s), rt.s, rtol=1e-4, atol=1e-5)
+    check_idx(idx.cpu().numpy(), rt.s, K)
+
+
+def test_route_bypass_keeps_all_blocks(lib):
+    q, k, v = _inputs(23, 2, 16, 2, 64, 5, 8, "bf16")
+    idx = lib.cast_route_topk(to_dev(q, "bf16"), [0, 1], to_dev(k, "bf16"), to_dev(v, "bf16"), 9)
+    torch.cuda.synchronize()
+    assert idx.shape == (2, 2, 5)
+    assert np.array_equal(idx.cpu().numpy(), np.broadcast_to(np.arange(5), (2, 2, 5)))
+
+
+@pytest.mark.parametrize("K", [4, 8, 16, 32])
+def test_route_stress_full_size(lib, K, stress_inputs):
+    """Long-history stress workload at full size (128 blocks of 3520 tokens, 24 heads)."""
+    inp = stress_inputs
+    idx, u = lib.cast_route_topk(inp["dev"]["q"], list(inp["anchors"]), inp["dev"]["k_hist"],
+                                 inp["dev"]["v_hist"], K, want_u=True)
+    torch.cuda.synchronize()
+    u_ref = inp["routing"].u
+    np.testing.assert_allclose(to_host(u), u_ref, rtol=1e-3, atol=1e-6 * u_ref.max())
+    amb = check_idx(idx.cpu().numpy(), u_ref, K)
+    if K <= 8:
+        assert amb == 0
+
+
+@pytest.fixture(scope="module")
+def stress_inputs():
+    import oracle.cast_oracle as O  # noqa: F811
+    w = W.STRESS
+    inp = W.stress_inputs(w)
+    dev = {k: to_dev(inp[k], "bf16") for k in ("q", "k_hist", "v_hist")}
+    anchors = [int(a) for a in inp["anchors"]]
+    # oracle pooled statistics block by block (float64), then Eqs. pooled / omission
+    q = inp["q"]
+    qbar = np.stack([q[a].astype(np.float64).mean(axis=0) for a in anchors])
+    kbar = np.stack([inp["k_hist"][m].astype(np.float64).mean(axis=0) for m in range(w.M)])
+    vbar = np.stack([inp["v_hist"][m].astype(np.float64).mean(axis=0) for m in range(w.M)])
+    rt = O.pooled_routing(qbar[:, None], list(range(len(anchors))), kbar[:, None], vbar[:, None])
+    return {"dev": dev, "anchors": anchors, "routing": rt}
