@@ -1,0 +1,373 @@
+"""Benchmark of the CAST block step on GB300: prints one JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Workload: the Matrix-Game-3.0-shaped bf16 block step (8 current latent frames of 30x52 tokens,
+12 heads x 128, 16 history blocks of 1560 tokens, K = 4, anchors every second frame).
+A step is cast_block_step: routing -> routed anchor attention -> PAR.
+  value   frames/s with inputs resident in HBM (CUDA events around each step, L2 flushed
+          between steps outside the timed events)
+  e2e     frames/s through the same C call with the inputs copied from pinned host memory
+          and r_out copied back, copies inside the timed region
+  roofline  the dominant kernel (routed attention): algorithmic FLOP per launch / its average
+          CUDA-event duration (stages launched through their own entry points, same kernels
+          and launch configuration as inside the block step) against the measured bf16 peak
+  cpu_baseline  the CPU oracle timed on a bounded sample of the same workload
+Under torchrun each rank runs its own block step (independent chunks, no collective): weak
+scaling, value = frames of all ranks / max over ranks of the timed region.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from synthetic import generators as G  # noqa: E402
+from synthetic import workloads as W  # noqa: E402
+
+METRIC = "block-step frames/s; routed-attn TFLOP/s & PAR GB/s as % of GB300 peak"
+WL = W.MG
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), d.get("bf16_tflops", 1900.0), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def algorithmic_work(wl):
+    S, D = wl.S, wl.H * wl.d
+    keff = min(wl.K, wl.M)
+    Kf = len(wl.anchors)
+    attn_flop = 4.0 * Kf * S * (wl.n_cur * S + keff * wl.B_v) * wl.d * wl.H
+    route_bytes = (Kf * S + 2 * wl.M * wl.B_v) * D * 2.0
+    par_bytes = wl.n_cur * S * D * 2.0   # anchors read once + skipped frames written once (bf16)
+    return attn_flop, route_bytes, par_bytes
+
+
+# ------------------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev_index):
+        self.proc = None
+        self.dev = dev_index
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.dev)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[3:7]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------------------ GPU arm
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_34144_gb300 import native as lib
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    wl = WL
+    inp = W.block_step_inputs(wl)
+
+    def to_bf16_host(x):
+        return torch.from_numpy(G.bf16_bits(x).view(np.int16)).view(torch.bfloat16)
+
+    names = ("q", "k_cur", "v_cur", "k_hist", "v_hist")
+    host = {k: to_bf16_host(inp[k]).pin_memory() for k in names}
+    d = {k: host[k].to(dev) for k in names}
+    N, S, H, dh = inp["q"].shape
+    anchors = list(wl.anchors)
+    keff = min(wl.K, wl.M)
+    r_out = torch.empty((N, S, H * dh), dtype=torch.bfloat16, device=dev)
+    idx = torch.empty((len(anchors), H, keff), dtype=torch.int32, device=dev)
+    params = lib.par_params(band_radius=wl.band_radius)
+    bargs = lib.block_args(d["q"], d["k_cur"], d["v_cur"], anchors, d["k_hist"], d["v_hist"],
+                           wl.K, wl.grid, r_out, idx_out=idx, params=params)
+    ws = torch.empty(max(lib.block_workspace_size(bargs), 256), dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        lib.cast_block_step_args(bargs, ws)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    lib.cast_check_device()
+
+    # ---------------- timed region: device-resident inputs
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.25)
+    for k in range(args.steps):
+        flush.fill_(k & 0xFF)   # L2 flush, outside the step's events
+        ev[k][0].record(stream)
+        step()
+        ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    lib.cast_check_device()
+    ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = world * N * args.steps / (total_ms / 1e3)
+
+    # ---------------- per-stage breakdown (same kernels through the stage entry points)
+    o_att = torch.empty((len(anchors), S, H * dh), dtype=torch.bfloat16, device=dev)
+    r_par = torch.empty_like(r_out)
+    r_par.copy_(r_out)
+    mask = W.anchor_mask(N, anchors)
+    rws = torch.empty(max(lib.route_workspace_size(d["q"], anchors, d["k_hist"], d["v_hist"], wl.K), 256),
+                      dtype=torch.uint8, device=dev)
+    pws = torch.empty(max(lib.par_workspace_size(r_par.view(N, wl.grid[0], wl.grid[1], H * dh), mask,
+                                                 params), 256), dtype=torch.uint8, device=dev)
+    nb = max(20, args.steps // 4)
+    st_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(nb)]
+    rp = r_par.view(N, wl.grid[0], wl.grid[1], H * dh)
+    for k in range(nb + 3):
+        flush.fill_(k & 0xFF)
+        e = st_ev[k - 3] if k >= 3 else None
+        if e:
+            e[0].record(stream)
+        lib.cast_route_topk(d["q"], anchors, d["k_hist"], d["v_hist"], wl.K, workspace=rws)
+        if e:
+            e[1].record(stream)
+        lib.cast_anchor_attention(d["q"], d["k_cur"], d["v_cur"], anchors, d["k_hist"], d["v_hist"],
+                                  idx, out=o_att)
+        if e:
+            e[2].record(stream)
+        lib.cast_par_reconstruct(rp, mask, None, params, workspace=pws)
+        if e:
+            e[3].record(stream)
+    torch.cuda.synchronize()
+    t_route = statistics.mean(e[0].elapsed_time(e[1]) for e in st_ev)
+    t_attn = statistics.mean(e[1].elapsed_time(e[2]) for e in st_ev)
+    t_par = statistics.mean(e[2].elapsed_time(e[3]) for e in st_ev)
+
+    # ---------------- end to end through the C call with host buffers
+    h_out = torch.empty((N, S, H * dh), dtype=torch.bfloat16).pin_memory()
+    ne = max(10, args.steps // 4)
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(ne)]
+    for k in range(ne + 2):
+        flush.fill_(k & 0xFF)
+        e = e2e_ev[k - 2] if k >= 2 else None
+        if e:
+            e[0].record(stream)
+        for nm in names:
+            d[nm].copy_(host[nm], non_blocking=True)
+        step()
+        h_out.copy_(r_out, non_blocking=True)
+        if e:
+            e[1].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
+    h2d = sum(host[nm].numel() * host[nm].element_size() for nm in names)
+    d2h = h_out.numel() * h_out.element_size()
+
+    if rank == 0:
+        hbm, bf16, src = _peaks()
+        attn_flop, route_bytes, par_bytes = algorithmic_work(wl)
+        achieved = attn_flop / (t_attn / 1e3) / 1e12
+        traffic = _captured_traffic()
+        line = {
+            "metric": METRIC, "value": round(value, 3), "unit": "frames/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": wl.name, "frames_per_step": N, "grid": list(wl.grid),
+                       "heads": H, "head_dim": dh, "history_blocks": wl.M, "block_tokens": wl.B_v,
+                       "K": wl.K, "anchors": anchors, "global_batch": world,
+                       "l2": "flushed (256 MiB write) between timed steps, outside the events",
+                       "parallelism": f"replicas x{world} (independent chunks, no collective)"},
+            "roofline": {"bound": "tensor", "kernel": "k_attn<128> (routed anchor attention)",
+                         "achieved": round(achieved, 2), "peak": bf16, "unit": "TFLOP/s",
+                         "frac": round(achieved / bf16, 4), "peak_source": f"{src} bf16 burst",
+                         "traffic": traffic, "flop_per_launch": attn_flop,
+                         "launch_ms": round(t_attn, 5)},
+            "breakdown": {
+                "route": {"ms": round(t_route, 5), "GB/s": round(route_bytes / t_route / 1e6, 1),
+                          "frac_hbm": round(route_bytes / t_route / 1e6 / hbm, 4),
+                          "bytes": route_bytes, "kernels": 3},
+                "attention": {"ms": round(t_attn, 5), "TFLOP/s": round(achieved, 2),
+                              "frac_bf16": round(achieved / bf16, 4)},
+                "par": {"ms": round(t_par, 5), "GB/s": round(par_bytes / t_par / 1e6, 1),
+                        "frac_hbm": round(par_bytes / t_par / 1e6 / hbm, 4), "bytes": par_bytes},
+                "hbm_peak_gbs": hbm},
+            "e2e": {"value": round(N / (e2e_ms / 1e3) * world, 3), "unit": "frames/s",
+                    "ms_per_step": round(e2e_ms, 4), "h2d_bytes_per_step": int(h2d),
+                    "d2h_bytes_per_step": int(d2h)},
+            "gpu_launches": 5 * args.steps,
+            "clocks": clk,
+        }
+        if not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline(wl)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _captured_traffic():
+    """DRAM bytes per attention launch from the committed ncu summary, if it is current."""
+    p = os.path.join(ROOT, "profiles", "attention_traffic.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("dram_bytes_per_launch")
+    return None
+
+
+# ------------------------------------------------------------------------------ CPU oracle
+def _oracle_sample(wl, inp, R, heads, row_stride, tiles):
+    """One bounded sample of the block step in the CPU oracle: routing and attention on the
+    first `heads` heads (attention on every `row_stride`-th query row), PAR on the first
+    `tiles` tiles (pooled over every channel).  Returns (seconds for the whole workload
+    scaled from the sample, description of the sample)."""
+    import oracle.cast_oracle as O
+    anchors = list(wl.anchors)
+    hs = slice(0, heads)
+    t0 = time.perf_counter()
+    rt = O.pooled_routing(inp["q"][:, :, hs], anchors, inp["k_hist"][:, :, hs],
+                          inp["v_hist"][:, :, hs])
+    idx = O.topk_blocks(rt.u, wl.K)
+    t1 = time.perf_counter()
+    rows = np.arange(0, wl.S, row_stride)
+    O.routed_attention(inp["q"][:, :, hs], inp["k_cur"][:, :, hs], inp["v_cur"][:, :, hs],
+                       inp["k_hist"][:, :, hs], inp["v_hist"][:, :, hs], anchors, idx, rows=rows)
+    t2 = time.perf_counter()
+    n_tiles = len(O.tiles_of(wl.grid[0], wl.grid[1], 8, 8))
+    O.par_reconstruct(R, W.anchor_mask(wl.n_cur, anchors), None,
+                      O.ParParams(band_radius=wl.band_radius), tiles=range(tiles))
+    t3 = time.perf_counter()
+    hf = wl.H / heads
+    est = (t1 - t0) * hf + (t2 - t1) * hf * (wl.S / len(rows)) + (t3 - t2) * (n_tiles / tiles)
+    desc = (f"routing on {heads}/{wl.H} heads (all tokens, all blocks), attention on those heads "
+            f"for {len(rows)}/{wl.S} query rows of every anchor, PAR on {tiles}/{n_tiles} tiles; "
+            f"each stage scaled to the full workload by its share of the work")
+    return est, desc
+
+
+def _par_input(wl):
+    return np.random.default_rng(0).standard_normal(
+        (wl.n_cur, wl.grid[0], wl.grid[1], wl.H * wl.d)).astype(np.float32)
+
+
+def cpu_baseline(wl):
+    inp = W.block_step_inputs(wl)
+    R = _par_input(wl)
+    cores = len(os.sched_getaffinity(0))
+    n_tiles = (wl.grid[0] + 7) // 8 * ((wl.grid[1] + 7) // 8)
+    est, desc = _oracle_sample(wl, inp, R, heads=wl.H, row_stride=16, tiles=n_tiles)
+    return {"value": round(wl.n_cur / est, 6), "unit": "frames/s", "cores": cores, "kind": "oracle",
+            "sample": desc, "est_seconds_per_step": round(est, 3)}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    wl = WL
+    inp = W.block_step_inputs(wl)
+    R = _par_input(wl)
+    cores = len(os.sched_getaffinity(0))
+    for _ in range(args.warmup):
+        _oracle_sample(wl, inp, R, heads=1, row_stride=wl.S // 8, tiles=1)
+    total, desc = 0.0, ""
+    for _ in range(args.steps):
+        est, desc = _oracle_sample(wl, inp, R, heads=1, row_stride=wl.S // 8, tiles=1)
+        total += est
+    value = wl.n_cur * args.steps / total
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "frames/s",
+            "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 2),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": wl.name},
+            "cpu_baseline": {"value": round(value, 6), "unit": "frames/s", "cores": cores,
+                             "kind": "oracle", "sample": desc},
+            "e2e": {"value": round(value, 6), "unit": "frames/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

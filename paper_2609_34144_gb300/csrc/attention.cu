@@ -67,6 +67,13 @@ struct Bars {
   int abort;
 };
 
+// 2^x in one MUFU op (flush-to-zero; 2^-inf = 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ bool aborted(const Bars* b) {
   return *reinterpret_cast<const volatile int*>(&b->abort) != 0;
 }
@@ -252,20 +259,43 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int jj = j - a.n_cur_tiles;
         valid = min(BN, a.B_v - (jj % a.tiles_per_block) * BN);
       }
-      float mx = -INFINITY;
+      // raw-logit max over the valid columns (scale > 0 commutes with max)
+      float mxr = -INFINITY;
 #pragma unroll
       for (int c = 0; c < BN; ++c) {
-        const float v = c < valid ? __uint_as_float(sr[c]) * a.scale_log2 : -INFINITY;
-        sr[c] = __float_as_uint(v);
-        mx = fmaxf(mx, v);
+        if (c >= valid) sr[c] = __float_as_uint(-INFINITY);
+        mxr = fmaxf(mxr, __uint_as_float(sr[c]));
       }
+      const float mx = mxr * a.scale_log2;
       const bool need = mx > m_ref + kRescaleThreshold;
       float corr = 1.f;
       if (need) {
-        corr = exp2f(m_ref - mx);   // 0 on the first tile (m_ref = -inf)
+        corr = ex2_approx(m_ref - mx);   // 0 on the first tile (m_ref = -inf)
         m_ref = mx;
         l *= corr;
       }
+      // P buffer sb is free once PV_{j-2} has completed
+      w = !aborted(bars) && mbar_wait(&bars->p_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, lim);
+      if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
+      float sum = 0.f;
+      uint8_t* prow = sP + sb * C::P_BYTES + row * 128;
+      const float nm = -m_ref;
+#pragma unroll
+      for (int c16 = 0; c16 < BN / 8; ++c16) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c16 * 8 + 2 * e]), a.scale_log2, nm));
+          const float p1 = ex2_approx(fmaf(__uint_as_float(sr[c16 * 8 + 2 * e + 1]), a.scale_log2, nm));
+          sum += p0 + p1;
+          __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
+          pk[e] = *reinterpret_cast<uint32_t*>(&b2);
+        }
+        const int blk = c16 >> 3, c = c16 & 7;
+        *reinterpret_cast<uint4*>(prow + blk * (BM * 128) + ((c ^ (row & 7)) << 4)) =
+            make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+      l += sum;
       if (j > 0 && __any_sync(0xffffffffu, need)) {
         // O holds P_0..P_{j-1} V once PV_{j-1} has completed; its commit is the
         // ((j-1)/2)-th completion of p_empty[(j-1)&1] (tracked phase by phase, never stale)
@@ -282,27 +312,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_st_x64(tl + 256 + half * 64, orr);
         }
       }
-      // P buffer sb is free once PV_{j-2} has completed
-      w = !aborted(bars) && mbar_wait(&bars->p_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, lim);
-      if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
-      float sum = 0.f;
-      uint8_t* prow = sP + sb * C::P_BYTES + row * 128;
-#pragma unroll
-      for (int c16 = 0; c16 < BN / 8; ++c16) {
-        uint32_t pk[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float p0 = exp2f(__uint_as_float(sr[c16 * 8 + 2 * e]) - m_ref);
-          const float p1 = exp2f(__uint_as_float(sr[c16 * 8 + 2 * e + 1]) - m_ref);
-          sum += p0 + p1;
-          __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
-          pk[e] = *reinterpret_cast<uint32_t*>(&b2);
-        }
-        const int blk = c16 >> 3, c = c16 & 7;
-        *reinterpret_cast<uint4*>(prow + blk * (BM * 128) + ((c ^ (row & 7)) << 4)) =
-            make_uint4(pk[0], pk[1], pk[2], pk[3]);
-      }
-      l += sum;
       fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(&bars->p_full[sb]);

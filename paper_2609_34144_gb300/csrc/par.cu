@@ -299,10 +299,18 @@ __global__ void __launch_bounds__(kThreads, 2)
       } else if (has_targets && recon) {
         // ---- transport of pair (j-1, j) on this tile
         if (tid < kNV) {
-          float s = 0.f;
+          // fixed-order sum over the chunks, 4 independent loads in flight
           const float* p = partial + ((int64_t)j * a.n_tile + tile) * a.n_chunk * kNV + tid;
-          for (int k = 0; k < a.n_chunk; ++k) s += __ldcg(p + (int64_t)k * kNV);
-          s_zw[tid] = s;
+          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+          int k = 0;
+          for (; k + 3 < a.n_chunk; k += 4) {
+            s0 += __ldcg(p + (int64_t)k * kNV);
+            s1 += __ldcg(p + (int64_t)(k + 1) * kNV);
+            s2 += __ldcg(p + (int64_t)(k + 2) * kNV);
+            s3 += __ldcg(p + (int64_t)(k + 3) * kNV);
+          }
+          for (; k < a.n_chunk; ++k) s0 += __ldcg(p + (int64_t)k * kNV);
+          s_zw[tid] = (s0 + s1) + (s2 + s3);
         }
         __syncthreads();
         if (warp == 0) tile_transport(a, g, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
