@@ -113,6 +113,22 @@ cast_status cast_route_topk(const cast_route_args* args, void* workspace,
                             size_t workspace_bytes, void* stream);
 size_t cast_route_workspace_size(const cast_route_args* args);
 
+/* cast_route_topk for callers that cannot allocate device memory.  The paper has no
+ * counterpart: this is a deployment convenience.  Plugins inside a host framework that owns
+ * all device allocations, real-time loops that must not take an allocator's locks or its
+ * implicit synchronisation, and fixed-budget embedded runtimes can call this instead of
+ * providing a workspace.  The scratch is a 16 MiB array that the library reserves in device
+ * memory on every GPU where it is loaded, until the process exits.
+ *   - Problems needing more than 16 MiB of scratch (cast_route_workspace_size() > 16 MiB)
+ *     are rejected with CAST_ERR_UNSUPPORTED and a message; nothing is launched.
+ *   - The first call on a device looks up the array's device address with that device
+ *     current (no allocation); make that first call before any stream capture.
+ *   - All calls share the one array and the kernels fully overwrite what they read, so no
+ *     clearing is needed between calls; calls whose work overlaps on the GPU (concurrent
+ *     streams, or several host threads) race on it and must be serialised by the caller.
+ *   - Inputs, outputs and errors are those of cast_route_topk. */
+cast_status cast_route_topk_noalloc(const cast_route_args* args, void* stream);
+
 /* ------------------------------------------------------------------------ */
 /* Routed anchor attention: Eq. (block), App. B.4, App. B.5.                 */
 /* ------------------------------------------------------------------------ */

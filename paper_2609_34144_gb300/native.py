@@ -72,6 +72,7 @@ class BlockArgs(C.Structure):
 _lib.cast_route_topk.argtypes = [C.POINTER(RouteArgs), _vp, C.c_size_t, _vp]
 _lib.cast_route_workspace_size.argtypes = [C.POINTER(RouteArgs)]
 _lib.cast_route_workspace_size.restype = C.c_size_t
+_lib.cast_route_topk_noalloc.argtypes = [C.POINTER(RouteArgs), _vp]
 _lib.cast_anchor_attention.argtypes = [C.POINTER(AttnArgs), _vp]
 _lib.cast_par_reconstruct.argtypes = [C.POINTER(ParArgs), _vp, C.c_size_t, _vp]
 _lib.cast_par_workspace_size.argtypes = [C.POINTER(ParArgs)]
@@ -85,11 +86,11 @@ _lib.cast_status_string.restype = C.c_char_p
 _lib.cast_last_error_detail.restype = C.c_char_p
 _lib.cast_check_device.argtypes = [_vp]
 _lib.cast_version.restype = C.c_char_p
-for _f in ("cast_route_topk", "cast_anchor_attention", "cast_par_reconstruct", "cast_block_step",
+for _f in ("cast_route_topk", "cast_route_topk_noalloc", "cast_anchor_attention", "cast_par_reconstruct", "cast_block_step",
            "cast_check_device"):
     getattr(_lib, _f).restype = C.c_int
 
-EXPORTED = ["cast_route_topk", "cast_route_workspace_size", "cast_anchor_attention",
+EXPORTED = ["cast_route_topk", "cast_route_workspace_size", "cast_route_topk_noalloc", "cast_anchor_attention",
             "cast_par_reconstruct", "cast_par_workspace_size", "cast_par_params_default",
             "cast_block_step", "cast_block_workspace_size", "cast_status_string",
             "cast_last_error_detail", "cast_check_device", "cast_version"]
@@ -209,6 +210,19 @@ def cast_route_topk(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROU
     if want_pooled:
         out.append((qb, kb, vb))
     return out[0] if len(out) == 1 else tuple(out)
+
+
+def cast_route_topk_noalloc(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8,
+                            mode=ROUTE_OMISSION, want_u=False, stream=None):
+    """As cast_route_topk, with the library's fixed 16 MiB device scratch instead of a
+    caller workspace (for callers that cannot allocate); returns idx (and u)."""
+    a = _route_args(q, anchors, k_hist, v_hist, K, gram, eps, mode)
+    Kf, H, M = len(anchors), q.shape[2], k_hist.shape[0]
+    idx = torch.empty((Kf, H, min(K, M)), dtype=torch.int32, device=q.device)
+    u = torch.empty((Kf, H, M), dtype=torch.float32, device=q.device) if want_u else None
+    a.idx, a.u = _ptr(idx), _ptr(u)
+    _check(_lib.cast_route_topk_noalloc(C.byref(a), _stream(stream)))
+    return (idx, u) if want_u else idx
 
 
 # --------------------------------------------------------------------------- attention
