@@ -269,6 +269,46 @@ __host__ __device__ __forceinline__ void fwd2d(const float (&x)[8][8], int h, in
   }
 }
 
+template <int W, class Emit>
+__host__ __device__ __forceinline__ void rows_inv_emit(const float (&re)[8][5], const float (&im)[8][5],
+                                                       int h, Emit&& emit) {
+#pragma unroll
+  for (int y = 0; y < 8; ++y) {
+    if (y < h) {
+      float row[8];
+      rinv<W>(re[y], im[y], row);
+      emit(y, row);
+    }
+  }
+}
+
+// Unnormalised inverse of fwd2d, handing each output row (W values) to emit(y, row) as soon
+// as it is formed (destroys re/im).
+template <class Emit>
+__host__ __device__ __forceinline__ void inv2d_emit(float (&re)[8][5], float (&im)[8][5], int h,
+                                                    int w, Emit&& emit) {
+  switch (h) {
+    case 8: cols<8, 1>(w, re, im); break;
+    case 7: cols<7, 1>(w, re, im); break;
+    case 6: cols<6, 1>(w, re, im); break;
+    case 5: cols<5, 1>(w, re, im); break;
+    case 4: cols<4, 1>(w, re, im); break;
+    case 3: cols<3, 1>(w, re, im); break;
+    case 2: cols<2, 1>(w, re, im); break;
+    default: cols<1, 1>(w, re, im); break;
+  }
+  switch (w) {
+    case 8: rows_inv_emit<8>(re, im, h, emit); break;
+    case 7: rows_inv_emit<7>(re, im, h, emit); break;
+    case 6: rows_inv_emit<6>(re, im, h, emit); break;
+    case 5: rows_inv_emit<5>(re, im, h, emit); break;
+    case 4: rows_inv_emit<4>(re, im, h, emit); break;
+    case 3: rows_inv_emit<3>(re, im, h, emit); break;
+    case 2: rows_inv_emit<2>(re, im, h, emit); break;
+    default: rows_inv_emit<1>(re, im, h, emit); break;
+  }
+}
+
 // Unnormalised inverse of fwd2d for a Hermitian-consistent half spectrum (destroys re/im).
 __host__ __device__ __forceinline__ void inv2d(float (&re)[8][5], float (&im)[8][5], int h, int w,
                                                float (&x)[8][8]) {

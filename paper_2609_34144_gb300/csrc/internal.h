@@ -1,5 +1,6 @@
 // Internal declarations shared by the translation units of libcast.
 #pragma once
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cstddef>
@@ -13,6 +14,14 @@ namespace cast {
 cast_status fail(cast_status s, const char* fmt, ...);
 // Converts a pending launch error into CAST_ERR_CUDA.
 cast_status check_launch(const char* what);
+
+// cuTensorMapEncodeTiled fetched from the driver through the runtime (no libcuda link);
+// nullptr if unavailable.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
 
 constexpr size_t kWsAlign = 256;
 inline size_t align_up(size_t x, size_t a = kWsAlign) { return (x + a - 1) / a * a; }

@@ -2,7 +2,10 @@
 // fcpasm; App. A.2), one fused persistent kernel.
 //
 // Work is split into items (spectral tile p, channel chunk of 128 channels); one thread owns
-// one channel of the tile and keeps the 2-D spectrum of its h x w tokens in registers.
+// one channel of the tile.  Thread 0 streams the item's anchor tiles through a TMA 4-D map
+// ([frame][row][col][channel], out-of-range rows/cols/channels arrive as zeros) into a
+// shared-memory stage, issuing anchor j+1 while the CTA transforms anchor j; the current
+// spectrum stays in registers and the previous one in shared memory.
 //   stats item  : walks the anchors in order, forms each anchor's spectrum once, and for every
 //                 adjacent anchor pair with targets reduces Z = sum_c w_c F_b conj(F_a) and
 //                 W = sum_c w_c |F_b||F_a| over the chunk's channels into a partial record.
@@ -27,16 +30,17 @@ namespace {
 
 constexpr int kThreads = 128;      // channels per item
 constexpr int kNB = 40;            // stored bins of an 8-wide tile: 8 x 5
-constexpr int kNV = 3 * kNB;       // Re Z, Im Z, W per bin
+constexpr int kNV = 3 * kNB;       // (Re Z, Im Z, W) per bin, record index = 3 * bin + component
 constexpr int kMaxSeg = 128;
 constexpr int kCoefBatch = 8;
+constexpr int kSpecFloats = 2 * kNB * kThreads;   // one spectrum per thread, [value][thread]
 
-__device__ unsigned int g_par_error;   // nonzero: a recon item gave up waiting
+__device__ unsigned int g_par_error;   // 1: a wait gave up
 
 struct ParKArgs {
   char* r;
   const float* wch;
-  int dtype, F, Hg, Wg, C;
+  int F, Hg, Wg, C;
   int th, tw, tiles_x, n_tile, n_chunk;
   int n_anchor;
   int anchor_frame[CAST_MAX_ANCHORS];
@@ -53,20 +57,15 @@ struct ParKArgs {
   unsigned long long wait_ns;
 };
 
-__device__ __forceinline__ float ld_elem(const char* base, int64_t off, int dtype) {
-  if (dtype == CAST_BF16) {
-    const unsigned short b = __ldg(reinterpret_cast<const unsigned short*>(base) + off);
-    return __uint_as_float(((unsigned)b) << 16);
-  }
-  return __ldg(reinterpret_cast<const float*>(base) + off);
-}
-__device__ __forceinline__ void st_elem(char* base, int64_t off, int dtype, float v) {
-  if (dtype == CAST_BF16) {
-    __stcs(reinterpret_cast<__nv_bfloat16*>(base) + off, __float2bfloat16_rn(v));
-  } else {
-    __stcs(reinterpret_cast<float*>(base) + off, v);
-  }
-}
+template <typename T>
+__device__ __forceinline__ float to_f32(T v);
+template <>
+__device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+__device__ __forceinline__ void st_stream(float* p, float v) { __stcs(p, v); }
+__device__ __forceinline__ void st_stream(__nv_bfloat16* p, float v) { __stcs(p, __float2bfloat16_rn(v)); }
 
 __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
   unsigned v;
@@ -88,19 +87,6 @@ __device__ __forceinline__ TileGeom tile_geom(const ParKArgs& a, int tile) {
   return g;
 }
 
-// Loads one channel of an h x w tile of frame f (zeros outside the tile or channel range).
-__device__ __forceinline__ void load_tile(const ParKArgs& a, int f, const TileGeom& g, int c,
-                                          bool active, float (&x)[8][8]) {
-  const int64_t rowC = (int64_t)a.Wg * a.C;
-  const int64_t base = ((int64_t)f * a.Hg + g.y0) * rowC + (int64_t)g.x0 * a.C + c;
-#pragma unroll
-  for (int y = 0; y < 8; ++y)
-#pragma unroll
-    for (int xx = 0; xx < 8; ++xx)
-      x[y][xx] = (active && y < g.h && xx < g.w) ? ld_elem(a.r, base + y * rowC + xx * a.C, a.dtype)
-                                                 : 0.f;
-}
-
 // Warp transpose-reduction of 32 values: lane l returns the warp sum of v[l].
 __device__ __forceinline__ float warp_transpose_sum(float (&v)[32], int lane) {
 #pragma unroll
@@ -118,18 +104,7 @@ __device__ __forceinline__ float warp_transpose_sum(float (&v)[32], int lane) {
   return v[0];
 }
 
-// value index vi in [0, 120): component vi / 40 (0: Re Z, 1: Im Z, 2: W) of bin vi % 40
-__device__ __forceinline__ float stat_value(int vi, float wc, const float* fa, const float* fb,
-                                            int tid) {
-  const int comp = vi / kNB, b = vi % kNB;
-  const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
-  const float br = fb[(2 * b) * kThreads + tid], bi = fb[(2 * b + 1) * kThreads + tid];
-  if (comp == 0) return wc * (br * ar + bi * ai);
-  if (comp == 1) return wc * (bi * ar - br * ai);
-  return wc * sqrtf((ar * ar + ai * ai) * (br * br + bi * bi));
-}
-
-// Per-tile transport of one anchor pair (warp 0): theta and g per stored bin.
+// Per-tile transport of one anchor pair (warp 0): theta and g per stored bin (App. A.2).
 __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float* zw, float* th,
                                float* gate, float* own_th, int* own_rel, int lane) {
   const float inv_hw = 1.f / (float)(g.h * g.w);
@@ -142,9 +117,9 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float
     const int b = lane + 32 * s;
     const int ky = b / 5, kx = b % 5;
     valid[s] = b < kNB && ky < g.h && kx <= hw2;
-    Zr[s] = valid[s] ? zw[b] * inv_hw : 0.f;
-    Zi[s] = valid[s] ? zw[kNB + b] * inv_hw : 0.f;
-    Wv[s] = valid[s] ? zw[2 * kNB + b] * inv_hw : 0.f;
+    Zr[s] = valid[s] ? zw[3 * b] * inv_hw : 0.f;
+    Zi[s] = valid[s] ? zw[3 * b + 1] * inv_hw : 0.f;
+    Wv[s] = valid[s] ? zw[3 * b + 2] * inv_hw : 0.f;
     Za[s] = sqrtf(Zr[s] * Zr[s] + Zi[s] * Zi[s]);
     if (valid[s]) wmax = fmaxf(wmax, Wv[s]);
   }
@@ -215,20 +190,37 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float
   }
 }
 
-constexpr int kSpecFloats = 2 * kNB * kThreads;   // one spectrum per thread, [value][thread]
-constexpr size_t kParDynSmem = 2 * kSpecFloats * sizeof(float);
+template <typename T>
+constexpr size_t stage_bytes() { return (size_t)64 * kThreads * sizeof(T); }
+template <typename T>
+constexpr size_t par_dyn_smem() { return stage_bytes<T>() + kSpecFloats * sizeof(float) + 1024; }
 
+template <typename T>
 __global__ void __launch_bounds__(kThreads, 2)
-    k_par(const __grid_constant__ ParKArgs a, float* __restrict__ partial,
-          unsigned* __restrict__ counters) {
-  extern __shared__ float s_spec[];   // spectra of anchors j-1 and j: s_spec[(j & 1) * kSpecFloats + ...]
+    k_par(const __grid_constant__ CUtensorMap tm, const __grid_constant__ ParKArgs a,
+          float* __restrict__ partial, unsigned* __restrict__ counters) {
+  extern __shared__ uint8_t dsm_raw[];
+  const uint32_t raw = smem_u32(dsm_raw);
+  uint8_t* dsm = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+  const T* stage = reinterpret_cast<const T*>(dsm);          // [y][x][channel] of one anchor tile
+  float* s_fprev = reinterpret_cast<float*>(dsm + stage_bytes<T>());   // [value][thread]
   __shared__ float s_red[kThreads / 32][128];
   __shared__ float s_zw[kNV];
   __shared__ float s_th[kNB], s_g[kNB], s_own_th[kNB];
   __shared__ int s_own_rel[kNB];
   __shared__ float4 s_coef[kCoefBatch][kNB];
   __shared__ int s_ticket;
+  __shared__ __align__(8) uint64_t s_full;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // bytes one TMA box delivers: 128 channels x tile_w x tile_h (must match the tensor map)
+  const uint32_t kStageBytes = (uint32_t)(kThreads * a.tw * a.th * sizeof(T));
+  if (tid == 0) {
+    mbar_init(&s_full, 1);
+    fence_barrier_init();
+    tma_prefetch_desc(&tm);
+  }
+  __syncthreads();
+  uint32_t n_loaded = 0;   // tiles consumed so far (phase of s_full)
 
   for (;;) {
     if (tid == 0) s_ticket = (int)atomicAdd(&counters[0], 1u);
@@ -247,9 +239,9 @@ __global__ void __launch_bounds__(kThreads, 2)
     const bool active = c < a.C;
     const float wc = active ? (a.wch ? __ldg(a.wch + c) : 1.f) : 0.f;
 
-    if (recon) {
-      // wait (bounded) until every chunk of this tile has published its partials
-      if (tid == 0) {
+    if (tid == 0) {
+      if (recon) {
+        // every chunk of this tile must have published its partial records (bounded wait)
         const uint64_t t0 = global_ns();
         while (ld_acquire(&counters[1 + tile]) < (unsigned)a.n_chunk) {
           if (global_ns() - t0 > a.wait_ns) {
@@ -259,32 +251,56 @@ __global__ void __launch_bounds__(kThreads, 2)
           __nanosleep(128);
         }
       }
-      __syncthreads();
+      mbar_arrive_expect_tx(&s_full, kStageBytes);
+      tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * kThreads, g.x0, g.y0, a.anchor_frame[0]);
     }
+    if (recon) __syncthreads();
 
     for (int j = 0; j < a.n_anchor; ++j) {
-      float* fb = s_spec + (j & 1) * kSpecFloats;        // this anchor (thread-private column)
-      const float* fa = s_spec + ((j + 1) & 1) * kSpecFloats;   // previous anchor
+      float re[8][5], im[8][5];
       {
-        float x[8][8], re[8][5], im[8][5];
-        load_tile(a, a.anchor_frame[j], g, c, active, x);
-        dft::fwd2d(x, g.h, g.w, re, im);
+        const bool ok = mbar_wait(&s_full, n_loaded & 1u, a.wait_ns);
+        ++n_loaded;
+        float x[8][8];
 #pragma unroll
-        for (int b = 0; b < kNB; ++b) {
-          fb[(2 * b) * kThreads + tid] = re[b / 5][b % 5];
-          fb[(2 * b + 1) * kThreads + tid] = im[b / 5][b % 5];
+        for (int y = 0; y < 8; ++y)
+#pragma unroll
+          for (int xx = 0; xx < 8; ++xx)
+            x[y][xx] = (y < a.th && xx < a.tw) ? to_f32(stage[(y * a.tw + xx) * kThreads + tid]) : 0.f;
+        // the stage is free: prefetch the next anchor while transforming this one.  A tile
+        // that never arrived ends the kernel for every thread of the CTA (error word set);
+        // the barrier is never re-armed in an incomplete phase.
+        if (__syncthreads_or(!ok)) {
+          if (tid == 0) atomicExch(&g_par_error, 1u);
+          return;
         }
+        if (tid == 0 && j + 1 < a.n_anchor) {
+          mbar_arrive_expect_tx(&s_full, kStageBytes);
+          tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * kThreads, g.x0, g.y0,
+                      a.anchor_frame[j + 1]);
+        }
+        dft::fwd2d(x, g.h, g.w, re, im);
       }
       const bool has_targets = j > 0 && a.pair_tbeg[j + 1] > a.pair_tbeg[j];
+      const float* fa = s_fprev;   // spectrum of anchor j-1 (this thread's column)
       if (has_targets && !recon) {
-        // ---- partial Z, W of pair (j-1, j) over this chunk's channels
+        // ---- partial Z = sum w F_b conj(F_a), W = sum w |F_b||F_a| over the chunk (Eq. cross)
 #pragma unroll
         for (int grp = 0; grp < 4; ++grp) {
           float v[32];
 #pragma unroll
           for (int e = 0; e < 32; ++e) {
             const int vi = grp * 32 + e;
-            v[e] = vi < kNV ? stat_value(vi, wc, fa, fb, tid) : 0.f;
+            if (vi < kNV) {
+              const int b = vi / 3, comp = vi % 3;
+              const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
+              const float br = re[b / 5][b % 5], bi = im[b / 5][b % 5];
+              v[e] = comp == 0 ? wc * (br * ar + bi * ai)
+                   : comp == 1 ? wc * (bi * ar - br * ai)
+                               : wc * sqrtf((ar * ar + ai * ai) * (br * br + bi * bi));
+            } else {
+              v[e] = 0.f;
+            }
           }
           s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
         }
@@ -316,6 +332,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (warp == 0) tile_transport(a, g, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
         __syncthreads();
         const float inv_hw = 1.f / (float)(g.h * g.w);
+        const int64_t rowC = (int64_t)a.Wg * a.C;
         for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += kCoefBatch) {
           const int nt = min(kCoefBatch, a.pair_tbeg[j + 1] - t0);
           for (int e = tid; e < nt * kNB; e += kThreads) {
@@ -324,35 +341,44 @@ __global__ void __launch_bounds__(kThreads, 2)
             float sa, ca, sb, cb;
             sincosf(s_g[b] * al * s_th[b], &sa, &ca);
             sincosf(-s_g[b] * (1.f - al) * s_th[b], &sb, &cb);
-            const float fa = (1.f - al) * inv_hw, fb = al * inv_hw;
-            s_coef[k][b] = make_float4(fa * ca, fa * sa, fb * cb, fb * sb);
+            const float fa_ = (1.f - al) * inv_hw, fb_ = al * inv_hw;
+            s_coef[k][b] = make_float4(fa_ * ca, fa_ * sa, fb_ * cb, fb_ * sb);
           }
           __syncthreads();
           for (int k = 0; k < nt; ++k) {
+            // Eq. (fcpasm): (1-alpha) F_a U^{g alpha} + alpha F_b U^{-g (1-alpha)}, ortho scale folded
             float hr[8][5], hi[8][5];
 #pragma unroll
             for (int b = 0; b < kNB; ++b) {
               const int ky = b / 5, kx = b % 5;
               const float4 cf = s_coef[k][b];
               const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
-              const float br = fb[(2 * b) * kThreads + tid], bi = fb[(2 * b + 1) * kThreads + tid];
+              const float br = re[ky][kx], bi = im[ky][kx];
               hr[ky][kx] = cf.x * ar - cf.y * ai + cf.z * br - cf.w * bi;
               hi[ky][kx] = cf.x * ai + cf.y * ar + cf.z * bi + cf.w * br;
             }
-            float y[8][8];
-            dft::inv2d(hr, hi, g.h, g.w, y);
-            if (active) {
-              const int tf = a.target_frame[t0 + k];
-              const int64_t rowC = (int64_t)a.Wg * a.C;
-              const int64_t base = ((int64_t)tf * a.Hg + g.y0) * rowC + (int64_t)g.x0 * a.C + c;
-#pragma unroll
-              for (int yy = 0; yy < 8; ++yy)
+            T* out = reinterpret_cast<T*>(a.r) +
+                     (((int64_t)a.target_frame[t0 + k] * a.Hg + g.y0) * rowC + (int64_t)g.x0 * a.C + c);
+            const int Cs = a.C;
+            const int w = g.w;
+            dft::inv2d_emit(hr, hi, g.h, g.w, [&](int yy, const float* row) {
+              if (active) {
+                T* p = out + yy * rowC;
 #pragma unroll
                 for (int xx = 0; xx < 8; ++xx)
-                  if (yy < g.h && xx < g.w) st_elem(a.r, base + yy * rowC + xx * a.C, a.dtype, y[yy][xx]);
-            }
+                  if (xx < w) st_stream(p + xx * Cs, row[xx]);
+              }
+            });
           }
           __syncthreads();
+        }
+      }
+      // this anchor's spectrum becomes the previous one (thread-private column)
+      if (j + 1 < a.n_anchor) {
+#pragma unroll
+        for (int b = 0; b < kNB; ++b) {
+          s_fprev[(2 * b) * kThreads + tid] = re[b / 5][b % 5];
+          s_fprev[(2 * b + 1) * kThreads + tid] = im[b / 5][b % 5];
         }
       }
     }
@@ -364,6 +390,42 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
     }
   }
+}
+
+// 4-D map [F][Hg][Wg][C], box (128 channels, tw, th, 1), zero fill out of range
+bool make_r_map(CUtensorMap* m, const cast_par_args& a) {
+  EncodeTiledFn fn = tensor_map_encoder();
+  if (!fn) return false;
+  const cuuint64_t elt = a.dtype == CAST_BF16 ? 2 : 4;
+  cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.Wg, (cuuint64_t)a.Hg, (cuuint64_t)a.F};
+  cuuint64_t strides[3] = {a.C * elt, (cuuint64_t)a.Wg * a.C * elt, (cuuint64_t)a.Hg * a.Wg * a.C * elt};
+  cuuint32_t box[4] = {(cuuint32_t)kThreads, (cuuint32_t)a.params.tile_w, (cuuint32_t)a.params.tile_h, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, a.dtype == CAST_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+            4, a.r, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <typename T>
+cast_status launch_typed(const CUtensorMap& tm, const ParKArgs& k, int tickets, float* partial,
+                         unsigned* counters, cudaStream_t st) {
+  static bool attr_set = false;
+  constexpr size_t smem = par_dyn_smem<T>();
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(k_par<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+        cudaSuccess)
+      return check_launch("PAR smem attribute");
+    attr_set = true;
+  }
+  int dev = 0, nsm = 0, occ = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_par<T>, kThreads, smem);
+  if (occ < 1) occ = 1;
+  int grid = nsm * occ;
+  if (grid > tickets) grid = tickets;
+  k_par<T><<<grid, kThreads, smem, st>>>(tm, k, partial, counters);
+  return check_launch("PAR kernel");
 }
 
 }  // namespace
@@ -402,7 +464,6 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
   ParKArgs k{};
   k.r = static_cast<char*>(a.r);
   k.wch = a.channel_weight;
-  k.dtype = a.dtype;
   k.F = a.F;
   k.Hg = a.Hg;
   k.Wg = a.Wg;
@@ -436,7 +497,6 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
       for (int t = a1 + 1; t < a.F; ++t) add(t);
   }
   k.pair_tbeg[na] = nt;
-  k.pair_tbeg[0] = 0;
   // ticket schedule: S(0), S(1), R(0), S(2), R(1), ..., R(n-1)
   int nseg = 0, ticket = 0;
   auto seg = [&](int slab, bool recon) {
@@ -469,27 +529,15 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
   k.gate_mode = pp.gate_mode;
   k.wait_ns = 2000000000ull;
 
+  CUtensorMap tm;
+  if (!make_r_map(&tm, a)) return fail(CAST_ERR_CUDA, "PAR: cuTensorMapEncodeTiled failed");
   char* w = static_cast<char*>(ws);
   float* partial = reinterpret_cast<float*>(w);
   unsigned* counters = reinterpret_cast<unsigned*>(w + p.partial_bytes);
   if (cudaMemsetAsync(counters, 0, (size_t)(1 + p.n_tile) * sizeof(unsigned), st) != cudaSuccess)
     return check_launch("PAR counter reset");
-  int dev = 0, nsm = 0, occ = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(k_par, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kParDynSmem) !=
-        cudaSuccess)
-      return check_launch("PAR smem attribute");
-    attr_set = true;
-  }
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_par, kThreads, kParDynSmem);
-  if (occ < 1) occ = 1;
-  int grid = nsm * occ;
-  if (grid > ticket) grid = ticket;
-  k_par<<<grid, kThreads, kParDynSmem, st>>>(k, partial, counters);
-  return check_launch("PAR kernel");
+  if (a.dtype == CAST_BF16) return launch_typed<__nv_bfloat16>(tm, k, ticket, partial, counters, st);
+  return launch_typed<float>(tm, k, ticket, partial, counters, st);
 }
 
 unsigned int par_error_word(cudaStream_t st, bool clear) {
