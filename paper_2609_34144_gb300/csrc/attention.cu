@@ -3,20 +3,24 @@
 // One CTA computes a 128-row query tile of one (anchor i, head h):
 //   O = softmax(scale Q K^T) V over every token of the current chunk followed by the tokens
 //   of the routed history blocks idx[i, h, :].
+// Two CTAs share an SM (96 KB of shared memory and 256 TMEM columns each), so the tensor
+// core runs one CTA's UMMAs while the other CTA's warps do their softmax.
 // Warp roles (192 threads):
-//   warp 0       TMA producer: Q once, then K / V tiles of 128 tokens into a 2-stage ring
-//                (128-byte swizzle, 64-element boxes), current-chunk tiles from a 2-D map,
+//   warp 0       TMA producer: Q once, then K and V tiles of 128 tokens (one stage each,
+//                128-byte swizzle, 64-element boxes); current-chunk tiles from a 2-D map,
 //                history tiles from a 3-D map [block, token, channel] so a tile never reads
 //                past its block (out-of-range rows arrive as zeros and are masked).
-//   warp 1       TMEM owner and single-thread UMMA issuer: S_j = Q K_j^T (M=128, N=128,
-//                kind::f16, f32 accumulate) into one of two TMEM S buffers, then
-//                O += P_{j-1} V_{j-1} (V read MN-major) into a TMEM O accumulator.
+//   warp 1       TMEM owner and single-thread UMMA issuer: S = Q K_j^T (M=128, N=128,
+//                kind::f16, f32 accumulate) into TMEM, then O += P_j V_j with P read from
+//                TMEM (it overwrites the S columns it came from) and V read MN-major.
 //   warps 2..5   one query row per thread: tcgen05.ld of the S row, masking, online softmax
 //                in the exp2 domain with lazy rescaling (O and l are rescaled only when the
-//                running max grows by more than 8 = log2 256), P written to shared memory as
-//                bf16 in the 128-byte-swizzled K-major layout the UMMA reads, and the epilogue
-//                O / l (+ log-sum-exp).
-// Every wait is bounded; on a timeout the CTA records an error word and leaves.
+//                running max grows by more than 8 = log2 256), P packed to bf16 and stored to
+//                TMEM with tcgen05.st, and the epilogue O / l (+ log-sum-exp).
+// Ordering: the UMMAs of one thread execute in issue order, and the arrival on s_full for
+// tile j (a commit after S_j) therefore also means PV_{j-1} has completed, so O may be
+// rescaled in place as soon as S_j is visible.  Every wait is bounded; on a timeout the CTA
+// records an error word, drains its UMMAs and frees TMEM before leaving.
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -29,20 +33,20 @@ namespace {
 
 __device__ unsigned int g_attn_error;
 
-constexpr int BM = 128, BN = 128, KST = 2;
+constexpr int BM = 128, BN = 128;
 constexpr int kThreads = 192;
+constexpr int kTmemCols = 256;   // S / P at column 0, O at column 128
+constexpr uint32_t kColO = 128;
 constexpr float kRescaleThreshold = 8.f;
 
 template <int HD>
 struct Cfg {
   static constexpr int Q_BYTES = BM * HD * 2;
   static constexpr int KV_BYTES = BN * HD * 2;
-  static constexpr int P_BYTES = BM * BN * 2;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + Q_BYTES;
-  static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
-  static constexpr int OFF_P = OFF_V + KST * KV_BYTES;
-  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int OFF_V = OFF_K + KV_BYTES;
+  static constexpr int OFF_BAR = OFF_V + KV_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;   // + barriers + alignment slack
 };
 
@@ -59,10 +63,7 @@ struct AttnKArgs {
 };
 
 struct Bars {
-  uint64_t q_full;
-  uint64_t k_full[KST], k_empty[KST], v_full[KST], v_empty[KST];
-  uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
-  uint64_t fin;
+  uint64_t q_full, k_full, k_empty, v_full, v_empty, s_full, p_full, fin;
   uint32_t tmem_base;
   int abort;
 };
@@ -83,7 +84,7 @@ __device__ __forceinline__ void set_abort(Bars* b) {
 }
 
 template <int HD>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     k_attn(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
            const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kh,
            const __grid_constant__ CUtensorMap tm_vh, const __grid_constant__ AttnKArgs a) {
@@ -94,7 +95,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sQ = smem + C::OFF_Q;
   uint8_t* sK = smem + C::OFF_K;
   uint8_t* sV = smem + C::OFF_V;
-  uint8_t* sP = smem + C::OFF_P;
   Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -108,24 +108,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&bars->q_full, 1);
-    for (int s = 0; s < KST; ++s) {
-      mbar_init(&bars->k_full[s], 1);
-      mbar_init(&bars->k_empty[s], 1);
-      mbar_init(&bars->v_full[s], 1);
-      mbar_init(&bars->v_empty[s], 1);
-    }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&bars->s_full[s], 1);
-      mbar_init(&bars->s_empty[s], 128);
-      mbar_init(&bars->p_full[s], 128);
-      mbar_init(&bars->p_empty[s], 1);
-    }
+    mbar_init(&bars->k_full, 1);
+    mbar_init(&bars->k_empty, 1);
+    mbar_init(&bars->v_full, 1);
+    mbar_init(&bars->v_empty, 1);
+    mbar_init(&bars->s_full, 1);
+    mbar_init(&bars->p_full, 128);
     mbar_init(&bars->fin, 1);
     bars->abort = 0;
     fence_barrier_init();
   }
   if (warp == 1) {
-    tmem_alloc(&bars->tmem_base, 512);
+    tmem_alloc(&bars->tmem_base, kTmemCols);
     tmem_relinquish();
     tc_fence_before();
   }
@@ -162,23 +156,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             z = 0;
           }
         }
-        const int s = j % KST;
-        const uint32_t ph = (uint32_t)(j / KST) & 1u;
-        if (aborted(bars) || !mbar_wait(&bars->k_empty[s], ph ^ 1u, lim)) { set_abort(bars); break; }
-        mbar_arrive_expect_tx(&bars->k_full[s], C::KV_BYTES);
+        const uint32_t ph = (uint32_t)j & 1u;
+        if (aborted(bars) || !mbar_wait(&bars->k_empty, ph ^ 1u, lim)) { set_abort(bars); break; }
+        mbar_arrive_expect_tx(&bars->k_full, C::KV_BYTES);
 #pragma unroll
         for (int b = 0; b < HD / 64; ++b) {
-          uint8_t* dst = sK + s * C::KV_BYTES + b * BN * 128;
-          if (cur) tma_load_2d(dst, &tm_kc, &bars->k_full[s], h * HD + b * 64, y);
-          else tma_load_3d(dst, &tm_kh, &bars->k_full[s], h * HD + b * 64, y, z);
+          uint8_t* dst = sK + b * BN * 128;
+          if (cur) tma_load_2d(dst, &tm_kc, &bars->k_full, h * HD + b * 64, y);
+          else tma_load_3d(dst, &tm_kh, &bars->k_full, h * HD + b * 64, y, z);
         }
-        if (aborted(bars) || !mbar_wait(&bars->v_empty[s], ph ^ 1u, lim)) { set_abort(bars); break; }
-        mbar_arrive_expect_tx(&bars->v_full[s], C::KV_BYTES);
+        if (aborted(bars) || !mbar_wait(&bars->v_empty, ph ^ 1u, lim)) { set_abort(bars); break; }
+        mbar_arrive_expect_tx(&bars->v_full, C::KV_BYTES);
 #pragma unroll
         for (int b = 0; b < HD / 64; ++b) {
-          uint8_t* dst = sV + s * C::KV_BYTES + b * BN * 128;
-          if (cur) tma_load_2d(dst, &tm_vc, &bars->v_full[s], h * HD + b * 64, y);
-          else tma_load_3d(dst, &tm_vh, &bars->v_full[s], h * HD + b * 64, y, z);
+          uint8_t* dst = sV + b * BN * 128;
+          if (cur) tma_load_2d(dst, &tm_vc, &bars->v_full, h * HD + b * 64, y);
+          else tma_load_3d(dst, &tm_vh, &bars->v_full, h * HD + b * 64, y, z);
         }
       }
     }
@@ -187,51 +180,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, HD, false, true);
-      const uint32_t q_addr = smem_u32(sQ), k_addr = smem_u32(sK), v_addr = smem_u32(sV),
-                     p_addr = smem_u32(sP);
+      const uint32_t q_addr = smem_u32(sQ), k_addr = smem_u32(sK), v_addr = smem_u32(sV);
       bool ok = mbar_wait(&bars->q_full, 0, lim);
-      if (!ok) set_abort(bars);
       tc_fence_after();
-      auto issue_pv = [&](int jp) -> bool {
-        const int pb = jp & 1;
-        const int vs = jp % KST;
-        if (aborted(bars) || !mbar_wait(&bars->p_full[pb], (uint32_t)(jp >> 1) & 1u, lim)) return false;
-        if (!mbar_wait(&bars->v_full[vs], (uint32_t)(jp / KST) & 1u, lim)) return false;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t ad =
-              sdesc_sw128(p_addr + pb * C::P_BYTES + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd = sdesc_sw128(v_addr + vs * C::KV_BYTES + kk * 16 * 128, BN * 128, 1024);
-          umma_bf16_ss(tmem + 256, ad, bd, idesc_pv, (jp > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(&bars->v_empty[vs]);
-        umma_commit(&bars->p_empty[pb]);   // also signals "O includes P_jp V_jp"
-        return true;
-      };
       for (int j = 0; ok && j < n_tiles; ++j) {
-        const int sb = j & 1;
-        const int ks = j % KST;
-        if (aborted(bars) || !mbar_wait(&bars->s_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, lim) ||
-            !mbar_wait(&bars->k_full[ks], (uint32_t)(j / KST) & 1u, lim)) {
+        const uint32_t ph = (uint32_t)j & 1u;
+        if (aborted(bars) || !mbar_wait(&bars->k_full, ph, lim)) { ok = false; break; }
+        tc_fence_after();
+        // S = Q K_j^T; the S columns are free: PV_{j-1}, which read P_{j-1} from them, was
+        // issued earlier and UMMAs execute in order
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint64_t ad = sdesc_sw128(q_addr + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd = sdesc_sw128(k_addr + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024);
+          umma_bf16_ss(tmem, ad, bd, idesc_qk, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&bars->s_full);
+        umma_commit(&bars->k_empty);
+        // O += P_j V_j once the softmax warps have stored P_j
+        if (aborted(bars) || !mbar_wait(&bars->p_full, ph, lim) ||
+            !mbar_wait(&bars->v_full, ph, lim)) {
           ok = false;
           break;
         }
         tc_fence_after();
 #pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(q_addr + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd =
-              sdesc_sw128(k_addr + ks * C::KV_BYTES + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024);
-          umma_bf16_ss(tmem + sb * BN, ad, bd, idesc_qk, kk > 0 ? 1u : 0u);
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const uint64_t bd = sdesc_sw128(v_addr + kk * 16 * 128, BN * 128, 1024);
+          umma_bf16_ts(tmem + kColO, tmem + kk * 8, bd, idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
         }
-        umma_commit(&bars->s_full[sb]);
-        umma_commit(&bars->k_empty[ks]);
-        if (j > 0 && !issue_pv(j - 1)) { ok = false; break; }
+        umma_commit(&bars->v_empty);
       }
-      if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
       if (!ok) set_abort(bars);
-      // drain: every issued UMMA has completed before TMEM is released
+      // every issued UMMA has completed before the epilogue reads O and TMEM is released
       umma_commit(&bars->fin);
       mbar_wait(&bars->fin, 0, lim);
     }
@@ -243,15 +224,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
-      const int sb = j & 1;
-      bool w = !aborted(bars) && mbar_wait(&bars->s_full[sb], (uint32_t)(j >> 1) & 1u, lim);
+      bool w = !aborted(bars) && mbar_wait(&bars->s_full, (uint32_t)j & 1u, lim);
       if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
       tc_fence_after();
       uint32_t sr[BN];
-      tmem_ld_x64(tl + sb * BN, sr);
-      tmem_ld_x64(tl + sb * BN + 64, sr + 64);
-      tc_fence_before();
-      mbar_arrive(&bars->s_empty[sb]);
+      tmem_ld_x64(tl, sr);
+      tmem_ld_x64(tl + 64, sr + 64);
       int valid;
       if (j < a.n_cur_tiles) {
         valid = min(BN, a.cur_rows - j * BN);
@@ -259,13 +237,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int jj = j - a.n_cur_tiles;
         valid = min(BN, a.B_v - (jj % a.tiles_per_block) * BN);
       }
-      // raw-logit max over the valid columns (scale > 0 commutes with max)
-      float mxr = -INFINITY;
+      // columns past the chunk / block end (only in a ragged last tile) get -inf
+      if (valid < BN) {
 #pragma unroll
-      for (int c = 0; c < BN; ++c) {
-        if (c >= valid) sr[c] = __float_as_uint(-INFINITY);
-        mxr = fmaxf(mxr, __uint_as_float(sr[c]));
+        for (int c = 0; c < BN; ++c)
+          if (c >= valid) sr[c] = __float_as_uint(-INFINITY);
       }
+      // raw-logit max (scale > 0 commutes with max), 8 independent chains
+      float m8[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) m8[e] = __uint_as_float(sr[e]);
+#pragma unroll
+      for (int c = 8; c < BN; c += 8)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) m8[e] = fmaxf(m8[e], __uint_as_float(sr[c + e]));
+      const float mxr = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                              fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       const float mx = mxr * a.scale_log2;
       const bool need = mx > m_ref + kRescaleThreshold;
       float corr = 1.f;
@@ -274,52 +261,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         m_ref = mx;
         l *= corr;
       }
-      // P buffer sb is free once PV_{j-2} has completed
-      w = !aborted(bars) && mbar_wait(&bars->p_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, lim);
-      if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
-      float sum = 0.f;
-      uint8_t* prow = sP + sb * C::P_BYTES + row * 128;
+      float s8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
       const float nm = -m_ref;
+      // P_j packed to bf16 pairs, stored over the first 64 S columns of this lane
 #pragma unroll
-      for (int c16 = 0; c16 < BN / 8; ++c16) {
-        uint32_t pk[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c16 * 8 + 2 * e]), a.scale_log2, nm));
-          const float p1 = ex2_approx(fmaf(__uint_as_float(sr[c16 * 8 + 2 * e + 1]), a.scale_log2, nm));
-          sum += p0 + p1;
-          __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
-          pk[e] = *reinterpret_cast<uint32_t*>(&b2);
-        }
-        const int blk = c16 >> 3, c = c16 & 7;
-        *reinterpret_cast<uint4*>(prow + blk * (BM * 128) + ((c ^ (row & 7)) << 4)) =
-            make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      for (int c = 0; c < BN; c += 2) {
+        const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c]), a.scale_log2, nm));
+        const float p1 = ex2_approx(fmaf(__uint_as_float(sr[c + 1]), a.scale_log2, nm));
+        s8[(c >> 1) & 7] += p0 + p1;
+        __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
+        sr[c / 2] = *reinterpret_cast<uint32_t*>(&b2);
       }
-      l += sum;
+      l += ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
+      tmem_st_x64(tl, sr);
       if (j > 0 && __any_sync(0xffffffffu, need)) {
-        // O holds P_0..P_{j-1} V once PV_{j-1} has completed; its commit is the
-        // ((j-1)/2)-th completion of p_empty[(j-1)&1] (tracked phase by phase, never stale)
-        w = !aborted(bars) &&
-            mbar_wait(&bars->p_empty[(j - 1) & 1], (uint32_t)((j - 1) >> 1) & 1u, lim);
-        if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
-        tc_fence_after();
+        // O = P_0..P_{j-1} V is final here: s_full for tile j implies PV_{j-1} completed,
+        // and PV_j waits for p_full below
 #pragma unroll
         for (int half = 0; half < HD / 64; ++half) {
           uint32_t orr[64];
-          tmem_ld_x64(tl + 256 + half * 64, orr);
+          tmem_ld_x64(tl + kColO + half * 64, orr);
 #pragma unroll
           for (int c = 0; c < 64; ++c) orr[c] = __float_as_uint(__uint_as_float(orr[c]) * corr);
-          tmem_st_x64(tl + 256 + half * 64, orr);
+          tmem_st_x64(tl + kColO + half * 64, orr);
         }
       }
-      fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&bars->p_full[sb]);
+      mbar_arrive(&bars->p_full);
     }
-    if (ok && n_tiles > 0) {
-      const int jl = n_tiles - 1;
-      bool w = !aborted(bars) &&
-               mbar_wait(&bars->p_empty[jl & 1], (uint32_t)(jl >> 1) & 1u, lim);
+    if (ok) {
+      bool w = !aborted(bars) && mbar_wait(&bars->fin, 0, lim);
       ok = __all_sync(0xffffffffu, w);
     }
     if (!ok) {
@@ -333,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int half = 0; half < HD / 64; ++half) {
         uint32_t orr[64];
-        tmem_ld_x64(tl + 256 + half * 64, orr);   // warp-collective: every lane loads
+        tmem_ld_x64(tl + kColO + half * 64, orr);   // warp-collective: every lane loads
         if (s < a.S) {
           if (a.o_f32) {
             float* dst = static_cast<float*>(a.o) + off + half * 64;
@@ -358,17 +329,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      {
-        if (a.lse && s < a.S)
-          a.lse[((int64_t)i * a.H + h) * a.S + s] = (m_ref + log2f(l)) * 0.69314718055994531f;
-      }
+      if (a.lse && s < a.S)
+        a.lse[((int64_t)i * a.H + h) * a.S + s] = (m_ref + log2f(l)) * 0.69314718055994531f;
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 512);
+    tmem_dealloc(tmem, kTmemCols);
   }
 }
 
