@@ -264,6 +264,8 @@ def run_gpu(args):
             "gpu_launches": 5 * args.steps,
             "clocks": clk,
         }
+        if not args.no_scale_points:
+            line["scale_points"] = scale_points(lib, torch, dev, flush)
         if not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline(wl)
         print(json.dumps(line), flush=True)
@@ -271,14 +273,115 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
+# ------------------------------------------------------------------------------ scale points
+SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy")
+
+
+def _scale_setup(name, lib, torch, dev):
+    """Inputs (seeded, generated on the device) and the call for one full-size stage run.
+    Returns (fn, work, unit): work is algorithmic bytes or FLOP per call."""
+    g = torch.Generator(device=dev).manual_seed(0)
+
+    def rnd(*shape, dtype=torch.bfloat16):
+        return torch.randn(*shape, generator=g, device=dev, dtype=torch.float32).to(dtype)
+
+    if name.startswith("par_sweep"):
+        w = W.PAR_SWEEP
+        dt = torch.float32 if name.endswith("f32") else torch.bfloat16
+        r = rnd(w.F, w.grid[0], w.grid[1], w.C, dtype=dt)
+        wc = torch.rand(w.C, generator=g, device=dev)
+        mask = W.anchor_mask(w.F, w.anchors(2))
+        p = lib.par_params(band_radius=w.band_radius)
+        ws = torch.empty(lib.par_workspace_size(r, mask, p), dtype=torch.uint8, device=dev)
+        return (lambda: lib.cast_par_reconstruct(r, mask, wc, p, workspace=ws),
+                r.numel() * r.element_size(), "B")
+    if name == "route_stress":
+        s = W.STRESS
+        q = rnd(s.n_cur, s.S, s.H, s.d)
+        kh, vh = rnd(s.M, s.B_v, s.H, s.d), rnd(s.M, s.B_v, s.H, s.d)
+        an = list(range(s.n_cur))
+        ws = torch.empty(lib.route_workspace_size(q, an, kh, vh, 8), dtype=torch.uint8, device=dev)
+        return (lambda: lib.cast_route_topk(q, an, kh, vh, 8, workspace=ws),
+                (s.n_cur * s.S + 2 * s.M * s.B_v) * s.H * s.d * 2, "B")
+    if name == "attn_hy":
+        wl = W.HY
+        N, S = wl.n_cur, wl.S
+        q, kc, vc = rnd(N, S, wl.H, wl.d), rnd(N, S, wl.H, wl.d), rnd(N, S, wl.H, wl.d)
+        kh, vh = rnd(wl.M, wl.B_v, wl.H, wl.d), rnd(wl.M, wl.B_v, wl.H, wl.d)
+        Kf = len(wl.anchors)
+        perm = torch.stack([torch.randperm(wl.M, generator=torch.Generator().manual_seed(k))[:wl.K]
+                            for k in range(Kf * wl.H)]).view(Kf, wl.H, wl.K)
+        idx = perm.int().to(dev)
+        o = torch.empty((Kf, S, wl.H * wl.d), dtype=torch.bfloat16, device=dev)
+        flop = 4.0 * Kf * S * (N * S + wl.K * wl.B_v) * wl.d * wl.H
+        return (lambda: lib.cast_anchor_attention(q, kc, vc, list(wl.anchors), kh, vh, idx, out=o),
+                flop, "FLOP")
+    raise ValueError(name)
+
+
+def scale_points(lib, torch, dev, flush, reps=10):
+    """Each stage at the full size of its own workload (device-resident inputs, L2 flushed
+    between launches, CUDA events on the launching stream)."""
+    hbm, bf16, _ = _peaks()
+    out = {}
+    stream = torch.cuda.current_stream(dev)
+    for name in SCALE_POINTS:
+        fn, work, unit = _scale_setup(name, lib, torch, dev)
+        for _ in range(3):
+            fn()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for k in range(reps):
+            flush.fill_(k & 0xFF)
+            ev[k][0].record(stream)
+            fn()
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+        ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+        if unit == "B":
+            rate = work / ms / 1e6
+            out[name] = {"ms": round(ms, 4), "GB/s": round(rate, 1), "frac_hbm": round(rate / hbm, 4),
+                         "bytes": work}
+        else:
+            rate = work / ms / 1e9
+            out[name] = {"ms": round(ms, 4), "TFLOP/s": round(rate, 1),
+                         "frac_bf16": round(rate / bf16, 4), "flop": work}
+        del fn
+        torch.cuda.empty_cache()
+    return out
+
+
+def run_profile(name):
+    """A few launches of one stage at full size, for an ncu capture."""
+    import torch
+
+    from paper_2609_34144_gb300 import native as lib
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    fn, _, _ = _scale_setup(name, lib, torch, dev)
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    lib.cast_check_device()
+    print(f"profiled {name}")
+
+
 def _captured_traffic():
-    """DRAM bytes per attention launch from the committed ncu summary, if it is current."""
-    p = os.path.join(ROOT, "profiles", "attention_traffic.json")
-    if os.path.exists(p):
-        with open(p) as f:
-            d = json.load(f)
-        return d.get("dram_bytes_per_launch")
-    return None
+    """DRAM bytes per attention launch from the committed ncu summary, or None when the
+    kernel sources changed since that capture (hash of attention.cu + ptx.cuh)."""
+    import hashlib
+    import re
+    prof = os.path.join(ROOT, "profiles", "k_attn_mg_block_step.md")
+    if not os.path.exists(prof):
+        return None
+    m = re.search(r"dram_bytes_per_launch=(\d+) source_sha256_16=([0-9a-f]+)", open(prof).read())
+    if not m:
+        return None
+    csrc = os.path.join(ROOT, "paper_2609_34144_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in ("attention.cu", "ptx.cuh"):
+        h.update(open(os.path.join(csrc, f), "rb").read())
+    return int(m.group(1)) if h.hexdigest()[:16] == m.group(2) else None
 
 
 # ------------------------------------------------------------------------------ CPU oracle
@@ -360,10 +463,15 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-scale-points", action="store_true")
+    ap.add_argument("--profile", default=None, choices=SCALE_POINTS,
+                    help="run only a few launches of one full-size stage (for ncu) and exit")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.profile:
+        run_profile(args.profile)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)
