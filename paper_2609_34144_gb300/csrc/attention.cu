@@ -1,26 +1,28 @@
 // Routed anchor attention on sm_103a tensor cores (Eq. block, App. B.4, App. B.5).
 //
-// One CTA computes a 128-row query tile of one (anchor i, head h):
+// One CTA computes two 128-row query tiles (Q0, Q1: 256 consecutive rows) of one
+// (anchor i, head h):
 //   O = softmax(scale Q K^T) V over every token of the current chunk followed by the tokens
 //   of the routed history blocks idx[i, h, :].
-// Two CTAs share an SM (96 KB of shared memory and 256 TMEM columns each), so the tensor
-// core runs one CTA's UMMAs while the other CTA's warps do their softmax.
-// Warp roles (192 threads):
-//   warp 0       TMA producer: Q once, then K and V tiles of 128 tokens (one stage each,
-//                128-byte swizzle, 64-element boxes); current-chunk tiles from a 2-D map,
-//                history tiles from a 3-D map [block, token, channel] so a tile never reads
-//                past its block (out-of-range rows arrive as zeros and are masked).
-//   warp 1       TMEM owner and single-thread UMMA issuer: S = Q K_j^T (M=128, N=128,
-//                kind::f16, f32 accumulate) into TMEM, then O += P_j V_j with P read from
-//                TMEM (it overwrites the S columns it came from) and V read MN-major.
-//   warps 2..5   one query row per thread: tcgen05.ld of the S row, masking, online softmax
-//                in the exp2 domain with lazy rescaling (O and l are rescaled only when the
-//                running max grows by more than 8 = log2 256), P packed to bf16 and stored to
-//                TMEM with tcgen05.st, and the epilogue O / l (+ log-sum-exp).
-// Ordering: the UMMAs of one thread execute in issue order, and the arrival on s_full for
-// tile j (a commit after S_j) therefore also means PV_{j-1} has completed, so O may be
-// rescaled in place as soon as S_j is visible.  Every wait is bounded; on a timeout the CTA
-// records an error word, drains its UMMAs and frees TMEM before leaving.
+// Both query tiles consume every K/V tile, so each tile fetched from L2 feeds 256 rows.
+// Warp roles (320 threads, one CTA per SM, 193 KB shared memory, all 512 TMEM columns):
+//   warp 0       TMA producers: lane 0 loads Q0/Q1 and the K tiles, lane 1 the V tiles, each
+//                into a two-stage ring (128 tokens x d, 128-byte swizzle, 64-element boxes);
+//                current-chunk tiles come from a 2-D map, history tiles from a 3-D map
+//                [block, token, channel] so a tile never reads past its block.
+//   warp 1       TMEM owner and single-thread UMMA issuer, order
+//                S0_0 S1_0 | PV0_0 S0_1 PV1_0 S1_1 | PV0_1 S0_2 PV1_1 S1_2 | ...
+//                (S_t = Q_t K^T, kind::f16, M=N=128, f32 in TMEM; PV_t: O_t += P_t V with P_t
+//                read from TMEM over the S_t columns and V read MN-major).
+//   warps 2..5   softmax of Q0, warps 6..9 softmax of Q1: one query row per thread,
+//                tcgen05.ld of the S row, masking, exp2-domain online softmax with lazy
+//                rescaling (O_t and l rescaled only when the running max grows by more than
+//                8 = log2 256), P packed to bf16 and stored with tcgen05.st, epilogue O / l.
+// While one warpgroup runs its softmax the tensor core works on the other tile.  UMMAs of
+// one thread execute in issue order, so S_t for tile j+1 (issued after PV_t of tile j)
+// certifies that PV_t of tile j has completed: O_t may then be rescaled in place.
+// Every wait is bounded; on a timeout the CTA records an error word, drains its UMMAs and
+// frees TMEM before leaving.
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -33,25 +35,24 @@ namespace {
 
 __device__ unsigned int g_attn_error;
 
-constexpr int BM = 128, BN = 128;
-constexpr int kThreads = 192;
-constexpr int kTmemCols = 256;   // S / P at column 0, O at column 128
-constexpr uint32_t kColO = 128;
+constexpr int BM = 128, BN = 128, kStages = 2;
+constexpr int kThreads = 320;
+constexpr int kTmemCols = 512;   // S0/P0 at 0, S1/P1 at 128, O0 at 256, O1 at 384
 constexpr float kRescaleThreshold = 8.f;
 
 template <int HD>
 struct Cfg {
   static constexpr int Q_BYTES = BM * HD * 2;
   static constexpr int KV_BYTES = BN * HD * 2;
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = OFF_Q + Q_BYTES;
-  static constexpr int OFF_V = OFF_K + KV_BYTES;
-  static constexpr int OFF_BAR = OFF_V + KV_BYTES;
+  static constexpr int OFF_Q = 0;                                   // Q0, Q1
+  static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;                 // kStages K tiles
+  static constexpr int OFF_V = OFF_K + kStages * KV_BYTES;          // kStages V tiles
+  static constexpr int OFF_BAR = OFF_V + kStages * KV_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;   // + barriers + alignment slack
 };
 
 struct AttnKArgs {
-  int S, H, n_qt, n_anchors, n_cur_tiles, tiles_per_block, K_eff, M, cur_rows, B_v;
+  int S, H, n_qp, n_anchors, n_cur_tiles, tiles_per_block, K_eff, M, cur_rows, B_v;
   const int* idx;
   void* o;
   int o_f32;
@@ -63,7 +64,10 @@ struct AttnKArgs {
 };
 
 struct Bars {
-  uint64_t q_full, k_full, k_empty, v_full, v_empty, s_full, p_full, fin;
+  uint64_t q_full;
+  uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
+  uint64_t s_full[2], p_full[2];
+  uint64_t fin;
   uint32_t tmem_base;
   int abort;
 };
@@ -83,8 +87,32 @@ __device__ __forceinline__ void set_abort(Bars* b) {
   atomicExch(&g_attn_error, 1u);
 }
 
+// (tensor map, row, block) of K/V tile j: current-chunk tiles first, then the routed blocks
+struct TileCoord {
+  bool cur;
+  int y, z;
+};
+__device__ __forceinline__ TileCoord tile_coord(const AttnKArgs& a, int i, int h, int j) {
+  TileCoord c;
+  c.cur = j < a.n_cur_tiles;
+  if (c.cur) {
+    c.y = j * BN;
+    c.z = 0;
+  } else {
+    const int jj = j - a.n_cur_tiles;
+    const int blk = jj / a.tiles_per_block;
+    c.y = (jj - blk * a.tiles_per_block) * BN;
+    c.z = a.idx[((int64_t)i * a.H + h) * a.K_eff + blk];
+    if (c.z < 0 || c.z >= a.M) {
+      atomicExch(&g_attn_error, 2u);
+      c.z = 0;
+    }
+  }
+  return c;
+}
+
 template <int HD>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
     k_attn(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
            const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kh,
            const __grid_constant__ CUtensorMap tm_vh, const __grid_constant__ AttnKArgs a) {
@@ -100,20 +128,26 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // head slowest: CTAs resident together share the head's current-chunk K/V in L2
   const int lin = blockIdx.x;
-  const int qt = lin % a.n_qt;
-  const int rest = lin / a.n_qt;
+  const int qp = lin % a.n_qp;
+  const int rest = lin / a.n_qp;
   const int i = rest % a.n_anchors;
   const int h = rest / a.n_anchors;
   const int n_tiles = a.n_cur_tiles + a.K_eff * a.tiles_per_block;
+  const int row0 = qp * 2 * BM;
+  const bool has_q1 = row0 + BM < a.S;
 
   if (threadIdx.x == 0) {
     mbar_init(&bars->q_full, 1);
-    mbar_init(&bars->k_full, 1);
-    mbar_init(&bars->k_empty, 1);
-    mbar_init(&bars->v_full, 1);
-    mbar_init(&bars->v_empty, 1);
-    mbar_init(&bars->s_full, 1);
-    mbar_init(&bars->p_full, 128);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&bars->k_full[s], 1);
+      mbar_init(&bars->k_empty[s], 1);
+      mbar_init(&bars->v_full[s], 1);
+      mbar_init(&bars->v_empty[s], 1);
+    }
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(&bars->s_full[t], 1);
+      mbar_init(&bars->p_full[t], 128);
+    }
     mbar_init(&bars->fin, 1);
     bars->abort = 0;
     fence_barrier_init();
@@ -129,49 +163,48 @@ __global__ void __launch_bounds__(kThreads, 2)
   const uint64_t lim = a.wait_ns;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+    // ------------------------------------------------------------ TMA producers
     if (lane == 0) {
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_kc);
-      tma_prefetch_desc(&tm_vc);
       tma_prefetch_desc(&tm_kh);
-      tma_prefetch_desc(&tm_vh);
-      mbar_arrive_expect_tx(&bars->q_full, C::Q_BYTES);
+      mbar_arrive_expect_tx(&bars->q_full, (has_q1 ? 2 : 1) * C::Q_BYTES);
+      for (int t = 0; t < (has_q1 ? 2 : 1); ++t)
 #pragma unroll
-      for (int b = 0; b < HD / 64; ++b)
-        tma_load_3d(sQ + b * BM * 128, &tm_q, &bars->q_full, h * HD + b * 64, qt * BM,
-                    a.q_frame[i]);
+        for (int b = 0; b < HD / 64; ++b)
+          tma_load_3d(sQ + t * C::Q_BYTES + b * BM * 128, &tm_q, &bars->q_full, h * HD + b * 64,
+                      row0 + t * BM, a.q_frame[i]);
       for (int j = 0; j < n_tiles; ++j) {
-        const bool cur = j < a.n_cur_tiles;
-        int y = 0, z = 0;
-        if (cur) {
-          y = j * BN;
-        } else {
-          const int jj = j - a.n_cur_tiles;
-          const int blk = jj / a.tiles_per_block;
-          y = (jj - blk * a.tiles_per_block) * BN;
-          z = a.idx[((int64_t)i * a.H + h) * a.K_eff + blk];
-          if (z < 0 || z >= a.M) {
-            atomicExch(&g_attn_error, 2u);
-            z = 0;
-          }
+        const TileCoord c = tile_coord(a, i, h, j);
+        const int s = j % kStages;
+        if (aborted(bars) || !mbar_wait(&bars->k_empty[s], ((uint32_t)(j / kStages) & 1u) ^ 1u, lim)) {
+          set_abort(bars);
+          break;
         }
-        const uint32_t ph = (uint32_t)j & 1u;
-        if (aborted(bars) || !mbar_wait(&bars->k_empty, ph ^ 1u, lim)) { set_abort(bars); break; }
-        mbar_arrive_expect_tx(&bars->k_full, C::KV_BYTES);
+        mbar_arrive_expect_tx(&bars->k_full[s], C::KV_BYTES);
 #pragma unroll
         for (int b = 0; b < HD / 64; ++b) {
-          uint8_t* dst = sK + b * BN * 128;
-          if (cur) tma_load_2d(dst, &tm_kc, &bars->k_full, h * HD + b * 64, y);
-          else tma_load_3d(dst, &tm_kh, &bars->k_full, h * HD + b * 64, y, z);
+          uint8_t* dst = sK + s * C::KV_BYTES + b * BN * 128;
+          if (c.cur) tma_load_2d(dst, &tm_kc, &bars->k_full[s], h * HD + b * 64, c.y);
+          else tma_load_3d(dst, &tm_kh, &bars->k_full[s], h * HD + b * 64, c.y, c.z);
         }
-        if (aborted(bars) || !mbar_wait(&bars->v_empty, ph ^ 1u, lim)) { set_abort(bars); break; }
-        mbar_arrive_expect_tx(&bars->v_full, C::KV_BYTES);
+      }
+    } else if (lane == 1) {
+      tma_prefetch_desc(&tm_vc);
+      tma_prefetch_desc(&tm_vh);
+      for (int j = 0; j < n_tiles; ++j) {
+        const TileCoord c = tile_coord(a, i, h, j);
+        const int s = j % kStages;
+        if (aborted(bars) || !mbar_wait(&bars->v_empty[s], ((uint32_t)(j / kStages) & 1u) ^ 1u, lim)) {
+          set_abort(bars);
+          break;
+        }
+        mbar_arrive_expect_tx(&bars->v_full[s], C::KV_BYTES);
 #pragma unroll
         for (int b = 0; b < HD / 64; ++b) {
-          uint8_t* dst = sV + b * BN * 128;
-          if (cur) tma_load_2d(dst, &tm_vc, &bars->v_full, h * HD + b * 64, y);
-          else tma_load_3d(dst, &tm_vh, &bars->v_full, h * HD + b * 64, y, z);
+          uint8_t* dst = sV + s * C::KV_BYTES + b * BN * 128;
+          if (c.cur) tma_load_2d(dst, &tm_vc, &bars->v_full[s], h * HD + b * 64, c.y);
+          else tma_load_3d(dst, &tm_vh, &bars->v_full[s], h * HD + b * 64, c.y, c.z);
         }
       }
     }
@@ -181,55 +214,82 @@ __global__ void __launch_bounds__(kThreads, 2)
       constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, HD, false, true);
       const uint32_t q_addr = smem_u32(sQ), k_addr = smem_u32(sK), v_addr = smem_u32(sV);
-      bool ok = mbar_wait(&bars->q_full, 0, lim);
-      tc_fence_after();
-      for (int j = 0; ok && j < n_tiles; ++j) {
-        const uint32_t ph = (uint32_t)j & 1u;
-        if (aborted(bars) || !mbar_wait(&bars->k_full, ph, lim)) { ok = false; break; }
-        tc_fence_after();
-        // S = Q K_j^T; the S columns are free: PV_{j-1}, which read P_{j-1} from them, was
-        // issued earlier and UMMAs execute in order
+      const int nq = has_q1 ? 2 : 1;
+      // S_t = Q_t K_j^T into the S_t columns (t * 128)
+      auto qk = [&](int t, int j) {
+        const int s = j % kStages;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(q_addr + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd = sdesc_sw128(k_addr + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024);
-          umma_bf16_ss(tmem, ad, bd, idesc_qk, kk > 0 ? 1u : 0u);
+          const uint64_t ad = sdesc_sw128(q_addr + t * C::Q_BYTES + (kk >> 2) * (BM * 128) + (kk & 3) * 32,
+                                          16, 1024);
+          const uint64_t bd = sdesc_sw128(k_addr + s * C::KV_BYTES + (kk >> 2) * (BN * 128) + (kk & 3) * 32,
+                                          16, 1024);
+          umma_bf16_ss(tmem + t * BN, ad, bd, idesc_qk, kk > 0 ? 1u : 0u);
         }
-        umma_commit(&bars->s_full);
-        umma_commit(&bars->k_empty);
-        // O += P_j V_j once the softmax warps have stored P_j
-        if (aborted(bars) || !mbar_wait(&bars->p_full, ph, lim) ||
-            !mbar_wait(&bars->v_full, ph, lim)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
+        umma_commit(&bars->s_full[t]);
+      };
+      // O_t += P_t V_j, P_t read from TMEM over the S_t columns
+      auto pv = [&](int t, int j) {
+        const int s = j % kStages;
 #pragma unroll
         for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(v_addr + kk * 16 * 128, BN * 128, 1024);
-          umma_bf16_ts(tmem + kColO, tmem + kk * 8, bd, idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+          const uint64_t bd = sdesc_sw128(v_addr + s * C::KV_BYTES + kk * 16 * 128, BN * 128, 1024);
+          umma_bf16_ts(tmem + 256 + t * 128, tmem + t * BN + kk * 8, bd, idesc_pv,
+                       (j > 0 || kk > 0) ? 1u : 0u);
         }
-        umma_commit(&bars->v_empty);
+      };
+      bool ok = mbar_wait(&bars->q_full, 0, lim) && mbar_wait(&bars->k_full[0], 0, lim);
+      tc_fence_after();
+      if (ok && n_tiles > 0) {
+        for (int t = 0; t < nq; ++t) qk(t, 0);
+        umma_commit(&bars->k_empty[0]);
+      }
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int s = j % kStages;
+        const uint32_t ph = (uint32_t)j & 1u;
+        const bool more = j + 1 < n_tiles;
+        if (aborted(bars) || !mbar_wait(&bars->v_full[s], (uint32_t)(j / kStages) & 1u, lim) ||
+            !mbar_wait(&bars->p_full[0], ph, lim)) { ok = false; break; }
+        tc_fence_after();
+        pv(0, j);
+        if (more) {
+          const int s1 = (j + 1) % kStages;
+          if (!mbar_wait(&bars->k_full[s1], (uint32_t)((j + 1) / kStages) & 1u, lim)) { ok = false; break; }
+          tc_fence_after();
+          qk(0, j + 1);
+        }
+        if (nq == 2) {
+          if (aborted(bars) || !mbar_wait(&bars->p_full[1], ph, lim)) { ok = false; break; }
+          tc_fence_after();
+          pv(1, j);
+        }
+        umma_commit(&bars->v_empty[s]);
+        if (more) {
+          if (nq == 2) qk(1, j + 1);
+          umma_commit(&bars->k_empty[(j + 1) % kStages]);
+        }
       }
       if (!ok) set_abort(bars);
       // every issued UMMA has completed before the epilogue reads O and TMEM is released
       umma_commit(&bars->fin);
       mbar_wait(&bars->fin, 0, lim);
     }
-  } else {
+  } else if (warp < 6 || has_q1) {
     // ------------------------------------------------------------ softmax + epilogue
+    const int t = warp < 6 ? 0 : 1;
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
+    const uint32_t colS = t * BN, colO = 256 + t * 128;
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
-      bool w = !aborted(bars) && mbar_wait(&bars->s_full, (uint32_t)j & 1u, lim);
+      bool w = !aborted(bars) && mbar_wait(&bars->s_full[t], (uint32_t)j & 1u, lim);
       if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
       tc_fence_after();
       uint32_t sr[BN];
-      tmem_ld_x64(tl, sr);
-      tmem_ld_x64(tl + 64, sr + 64);
+      tmem_ld_x64(tl + colS, sr);
+      tmem_ld_x64(tl + colS + 64, sr + 64);
       int valid;
       if (j < a.n_cur_tiles) {
         valid = min(BN, a.cur_rows - j * BN);
@@ -263,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
       float s8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
       const float nm = -m_ref;
-      // P_j packed to bf16 pairs, stored over the first 64 S columns of this lane
+      // P packed to bf16 pairs, stored over the first 64 S columns of this lane
 #pragma unroll
       for (int c = 0; c < BN; c += 2) {
         const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c]), a.scale_log2, nm));
@@ -273,21 +333,21 @@ __global__ void __launch_bounds__(kThreads, 2)
         sr[c / 2] = *reinterpret_cast<uint32_t*>(&b2);
       }
       l += ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
-      tmem_st_x64(tl, sr);
+      tmem_st_x64(tl + colS, sr);
       if (j > 0 && __any_sync(0xffffffffu, need)) {
-        // O = P_0..P_{j-1} V is final here: s_full for tile j implies PV_{j-1} completed,
-        // and PV_j waits for p_full below
+        // O_t holds P_0..P_{j-1} V and is final: S_t of tile j was issued after PV_t of
+        // tile j-1, and PV_t of tile j waits for p_full below
 #pragma unroll
         for (int half = 0; half < HD / 64; ++half) {
           uint32_t orr[64];
-          tmem_ld_x64(tl + kColO + half * 64, orr);
+          tmem_ld_x64(tl + colO + half * 64, orr);
 #pragma unroll
           for (int c = 0; c < 64; ++c) orr[c] = __float_as_uint(__uint_as_float(orr[c]) * corr);
-          tmem_st_x64(tl + kColO + half * 64, orr);
+          tmem_st_x64(tl + colO + half * 64, orr);
         }
       }
       tc_fence_before();
-      mbar_arrive(&bars->p_full);
+      mbar_arrive(&bars->p_full[t]);
     }
     if (ok) {
       bool w = !aborted(bars) && mbar_wait(&bars->fin, 0, lim);
@@ -297,14 +357,14 @@ __global__ void __launch_bounds__(kThreads, 2)
       set_abort(bars);
     } else {
       tc_fence_after();
-      const int s = qt * BM + row;
+      const int s = row0 + t * BM + row;
       const float inv = l > 0.f ? 1.f / l : 0.f;
       const int64_t D = (int64_t)a.H * HD;
       const int64_t off = ((int64_t)a.o_frame[i] * a.S + s) * D + (int64_t)h * HD;
 #pragma unroll
       for (int half = 0; half < HD / 64; ++half) {
         uint32_t orr[64];
-        tmem_ld_x64(tl + kColO + half * 64, orr);   // warp-collective: every lane loads
+        tmem_ld_x64(tl + colO + half * 64, orr);   // warp-collective: every lane loads
         if (s < a.S) {
           if (a.o_f32) {
             float* dst = static_cast<float*>(a.o) + off + half * 64;
@@ -379,7 +439,7 @@ cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream
   AttnKArgs k{};
   k.S = a.S;
   k.H = a.H;
-  k.n_qt = (a.S + BM - 1) / BM;
+  k.n_qp = (a.S + 2 * BM - 1) / (2 * BM);
   k.n_anchors = a.n_anchors;
   k.n_cur_tiles = (int)((cur_rows + BN - 1) / BN);
   k.tiles_per_block = a.M > 0 ? (a.B_v + BN - 1) / BN : 0;
@@ -405,7 +465,7 @@ cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream
       return check_launch("attention smem attribute");
     attr_set = true;
   }
-  const int grid = k.n_qt * a.n_anchors * a.H;
+  const int grid = k.n_qp * a.n_anchors * a.H;
   k_attn<HD><<<grid, kThreads, C::SMEM, st>>>(mq, mkc, mvc, mkh, mvh, k);
   return check_launch("attention kernel");
 }
