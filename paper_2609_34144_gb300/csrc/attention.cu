@@ -52,7 +52,7 @@ struct Cfg {
 };
 
 struct AttnKArgs {
-  int S, H, n_qp, n_anchors, n_cur_tiles, tiles_per_block, K_eff, M, cur_rows, B_v;
+  int S, H, n_pairs, n_single, n_anchors, n_cur_tiles, tiles_per_block, K_eff, M, cur_rows, B_v;
   const int* idx;
   void* o;
   int o_f32;
@@ -77,6 +77,12 @@ __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
 __device__ __forceinline__ bool aborted(const Bars* b) {
@@ -126,10 +132,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // head slowest: CTAs resident together share the head's current-chunk K/V in L2
-  const int lin = blockIdx.x;
-  const int qp = lin % a.n_qp;
-  const int rest = lin / a.n_qp;
+  // Longest work first: every CTA holding two query tiles, then the CTAs holding a single
+  // remainder tile (S mod 256 <= 128), which fill the last round.  Head slowest within each
+  // group: CTAs resident together share the head's current-chunk K/V in L2.
+  int lin = blockIdx.x, qp, rest;
+  const int n_pair_ctas = a.n_pairs * a.n_anchors * a.H;
+  if (lin < n_pair_ctas) {
+    qp = lin % a.n_pairs;
+    rest = lin / a.n_pairs;
+  } else {
+    qp = a.n_pairs;
+    rest = lin - n_pair_ctas;
+  }
   const int i = rest % a.n_anchors;
   const int h = rest / a.n_anchors;
   const int n_tiles = a.n_cur_tiles + a.K_eff * a.tiles_per_block;
@@ -303,16 +317,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < BN; ++c)
           if (c >= valid) sr[c] = __float_as_uint(-INFINITY);
       }
-      // raw-logit max (scale > 0 commutes with max), 8 independent chains
+      // raw-logit max (scale > 0 commutes with max): 3-input max, 8 independent chains
       float m8[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) m8[e] = __uint_as_float(sr[e]);
+      for (int e = 0; e < 8; ++e) m8[e] = fmaxf(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1]));
 #pragma unroll
-      for (int c = 8; c < BN; c += 8)
+      for (int c = 16; c < BN; c += 16)
 #pragma unroll
-        for (int e = 0; e < 8; ++e) m8[e] = fmaxf(m8[e], __uint_as_float(sr[c + e]));
-      const float mxr = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
-                              fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+        for (int e = 0; e < 8; ++e)
+          m8[e] = max3(m8[e], __uint_as_float(sr[c + 2 * e]), __uint_as_float(sr[c + 2 * e + 1]));
+      const float mxr = max3(max3(m8[0], m8[1], m8[2]), max3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
       const float mx = mxr * a.scale_log2;
       const bool need = mx > m_ref + kRescaleThreshold;
       float corr = 1.f;
@@ -321,18 +335,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         m_ref = mx;
         l *= corr;
       }
-      float s8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      const float nm = -m_ref;
-      // P packed to bf16 pairs, stored over the first 64 S columns of this lane
+      // P = 2^(s * scale_log2 - m_ref): packed f32x2 FMA and sums, one MUFU op per element,
+      // packed to bf16 pairs over the first 64 S columns of this lane
+      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+      const float2 nm2 = make_float2(-m_ref, -m_ref);
+      float2 s4[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                      make_float2(0.f, 0.f)};
 #pragma unroll
       for (int c = 0; c < BN; c += 2) {
-        const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c]), a.scale_log2, nm));
-        const float p1 = ex2_approx(fmaf(__uint_as_float(sr[c + 1]), a.scale_log2, nm));
-        s8[(c >> 1) & 7] += p0 + p1;
-        __nv_bfloat162 b2 = __floats2bfloat162_rn(p0, p1);
+        const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])),
+                                    sc2, nm2);
+        const float2 p = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+        s4[(c >> 1) & 3] = __fadd2_rn(s4[(c >> 1) & 3], p);
+        __nv_bfloat162 b2 = __floats2bfloat162_rn(p.x, p.y);
         sr[c / 2] = *reinterpret_cast<uint32_t*>(&b2);
       }
-      l += ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
+      const float2 s2 = __fadd2_rn(__fadd2_rn(s4[0], s4[1]), __fadd2_rn(s4[2], s4[3]));
+      l += s2.x + s2.y;
       tmem_st_x64(tl + colS, sr);
       if (j > 0 && __any_sync(0xffffffffu, need)) {
         // O_t holds P_0..P_{j-1} V and is final: S_t of tile j was issued after PV_t of
@@ -439,7 +458,10 @@ cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream
   AttnKArgs k{};
   k.S = a.S;
   k.H = a.H;
-  k.n_qp = (a.S + 2 * BM - 1) / (2 * BM);
+  // query rows per (anchor, head): pairs of 128-row tiles, plus one single tile when the
+  // remainder is at most 128 rows
+  k.n_pairs = a.S / (2 * BM) + (a.S % (2 * BM) > BM ? 1 : 0);
+  k.n_single = (a.S % (2 * BM) > 0 && a.S % (2 * BM) <= BM) ? 1 : 0;
   k.n_anchors = a.n_anchors;
   k.n_cur_tiles = (int)((cur_rows + BN - 1) / BN);
   k.tiles_per_block = a.M > 0 ? (a.B_v + BN - 1) / BN : 0;
@@ -465,7 +487,7 @@ cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream
       return check_launch("attention smem attribute");
     attr_set = true;
   }
-  const int grid = k.n_qp * a.n_anchors * a.H;
+  const int grid = (k.n_pairs + k.n_single) * a.n_anchors * a.H;
   k_attn<HD><<<grid, kThreads, C::SMEM, st>>>(mq, mkc, mvc, mkh, mvh, k);
   return check_launch("attention kernel");
 }
