@@ -185,6 +185,9 @@ def run_gpu(args):
                       dtype=torch.uint8, device=dev)
     pws = torch.empty(max(lib.par_workspace_size(r_par.view(N, wl.grid[0], wl.grid[1], H * dh), mask,
                                                  params), 256), dtype=torch.uint8, device=dev)
+    aws = torch.empty(max(lib.attention_workspace_size(d["q"], d["k_cur"], d["v_cur"], anchors,
+                                                      d["k_hist"], d["v_hist"], idx), 256),
+                      dtype=torch.uint8, device=dev)
     nb = max(20, args.steps // 4)
     st_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(nb)]
     rp = r_par.view(N, wl.grid[0], wl.grid[1], H * dh)
@@ -197,7 +200,7 @@ def run_gpu(args):
         if e:
             e[1].record(stream)
         lib.cast_anchor_attention(d["q"], d["k_cur"], d["v_cur"], anchors, d["k_hist"], d["v_hist"],
-                                  idx, out=o_att)
+                                  idx, out=o_att, workspace=aws)
         if e:
             e[2].record(stream)
         lib.cast_par_reconstruct(rp, mask, None, params, workspace=pws)
@@ -314,7 +317,10 @@ def _scale_setup(name, lib, torch, dev):
         idx = perm.int().to(dev)
         o = torch.empty((Kf, S, wl.H * wl.d), dtype=torch.bfloat16, device=dev)
         flop = 4.0 * Kf * S * (N * S + wl.K * wl.B_v) * wl.d * wl.H
-        return (lambda: lib.cast_anchor_attention(q, kc, vc, list(wl.anchors), kh, vh, idx, out=o),
+        aws = torch.empty(max(lib.attention_workspace_size(q, kc, vc, list(wl.anchors), kh, vh, idx), 256),
+                          dtype=torch.uint8, device=dev)
+        return (lambda: lib.cast_anchor_attention(q, kc, vc, list(wl.anchors), kh, vh, idx, out=o,
+                                                  workspace=aws),
                 flop, "FLOP")
     raise ValueError(name)
 

@@ -29,9 +29,8 @@
  *     returned; cast_last_error_detail() gives a message for the calling thread.
  *     CAST_ERR_CUDA reports a launch or runtime error seen after enqueuing.
  *   - Kernels never wait without bound.  A wait that exceeds its limit makes the
- *     kernel record an error word and return; the next call on this device that
- *     finds the word set returns CAST_ERR_DEVICE_TIMEOUT (cast_check_device()
- *     polls it explicitly; it synchronises `stream`).
+ *     kernel record an error word and return; cast_check_device() reads (and
+ *     clears) that word and returns CAST_ERR_DEVICE_TIMEOUT.
  *   - Layouts are row-major.  Token tensors are [frames, S, H, d] with d
  *     contiguous and S = Hg * Wg tokens of a frame's latent grid in row-major
  *     (y, x) order; the token row stride (elements between consecutive tokens)
@@ -156,10 +155,16 @@ typedef struct {
 /* O[i, s, h, :] = sum_j softmax_j(scale * q_i,s,h . k_j) v_j, where j runs over every
  * token of the current chunk (no causal mask inside the chunk) and every token of the
  * history blocks idx[i, h, :].  bf16 operands, f32 softmax and accumulation (Tab. config).
+ * The workspace (cast_attention_workspace_size() bytes; 0 and NULL allowed when that is 0)
+ * holds the partial results of query tiles whose keys are split over several SMs to fill the
+ * last round of work.
  * Errors: INVALID_ARG for NULL pointers, bad shapes or strides, anchors not ascending,
- * K_eff > 0 with M == 0; UNSUPPORTED for d not 64/128 or S*n_frames >= 2^31.
- * Block indices outside [0, M) make the kernel record an error and skip that block. */
-cast_status cast_anchor_attention(const cast_attn_args* args, void* stream);
+ * K_eff > 0 with M == 0, a short workspace; UNSUPPORTED for d not 64/128 or
+ * S*n_frames >= 2^31.  Block indices outside [0, M) make the kernel record an error and
+ * read block 0 instead. */
+cast_status cast_anchor_attention(const cast_attn_args* args, void* workspace,
+                                  size_t workspace_bytes, void* stream);
+size_t cast_attention_workspace_size(const cast_attn_args* args);
 
 /* ------------------------------------------------------------------------ */
 /* Phase-Aware Reconstruction: Section 4.3, Eqs. (cross), (confidence),      */

@@ -21,6 +21,10 @@
 // While one warpgroup runs its softmax the tensor core works on the other tile.  UMMAs of
 // one thread execute in issue order, so S_t for tile j+1 (issued after PV_t of tile j)
 // certifies that PV_t of tile j has completed: O_t may then be rescaled in place.
+// Load balance: a unit is one CTA's pair of query tiles with all its K/V tiles.  Units fill
+// whole rounds of one CTA per SM; the units of a last, partial round are split along the K/V
+// axis over all SMs, each part writes its unnormalised O with its row max and sum, and the
+// part that arrives last merges them (exp2-weighted by the row maxima).
 // Every wait is bounded; on a timeout the CTA records an error word, drains its UMMAs and
 // frees TMEM before leaving.
 #include <cuda_bf16.h>
@@ -53,6 +57,12 @@ struct Cfg {
 
 struct AttnKArgs {
   int S, H, n_pairs, n_single, n_anchors, n_cur_tiles, tiles_per_block, K_eff, M, cur_rows, B_v;
+  int n_full;        // units run whole (CTAs 0 .. n_full-1)
+  int n_split;       // parts of every remaining unit
+  int chunk;         // K/V tiles per part
+  float* part_o;     // [tail unit][part][2][128][HD] unnormalised O of the parts
+  float* part_ml;    // [tail unit][part][2][128][2] row max (log2 domain) and row sum
+  unsigned* counters;   // [tail unit] parts finished
   const int* idx;
   void* o;
   int o_f32;
@@ -67,9 +77,10 @@ struct Bars {
   uint64_t q_full;
   uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
   uint64_t s_full[2], p_full[2];
-  uint64_t fin;
+  uint64_t fin, part_done, merge_go;
   uint32_t tmem_base;
   int abort;
+  int last;
 };
 
 // 2^x in one MUFU op (flush-to-zero; 2^-inf = 0)
@@ -132,21 +143,35 @@ __global__ void __launch_bounds__(kThreads, 1)
   Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // Longest work first: every CTA holding two query tiles, then the CTAs holding a single
-  // remainder tile (S mod 256 <= 128), which fill the last round.  Head slowest within each
-  // group: CTAs resident together share the head's current-chunk K/V in L2.
-  int lin = blockIdx.x, qp, rest;
-  const int n_pair_ctas = a.n_pairs * a.n_anchors * a.H;
-  if (lin < n_pair_ctas) {
-    qp = lin % a.n_pairs;
-    rest = lin / a.n_pairs;
+  // Unit of this CTA (whole, or one K/V part of a tail unit).  Units are ordered longest
+  // first: every pair of query tiles, then the single remainder tiles (S mod 256 <= 128).
+  // Head slowest within each group: CTAs resident together share the head's current-chunk
+  // K/V in L2.
+  const int n_tiles_all = a.n_cur_tiles + a.K_eff * a.tiles_per_block;
+  int u, part = 0, k0 = 0, k1 = n_tiles_all;
+  const bool split = (int)blockIdx.x >= a.n_full;
+  if (!split) {
+    u = blockIdx.x;
+  } else {
+    const int t = blockIdx.x - a.n_full;
+    u = a.n_full + t / a.n_split;
+    part = t % a.n_split;
+    k0 = part * a.chunk;
+    k1 = min(n_tiles_all, k0 + a.chunk);
+  }
+  const int tail_unit = u - a.n_full;
+  int qp, rest;
+  const int n_pair_units = a.n_pairs * a.n_anchors * a.H;
+  if (u < n_pair_units) {
+    qp = u % a.n_pairs;
+    rest = u / a.n_pairs;
   } else {
     qp = a.n_pairs;
-    rest = lin - n_pair_ctas;
+    rest = u - n_pair_units;
   }
   const int i = rest % a.n_anchors;
   const int h = rest / a.n_anchors;
-  const int n_tiles = a.n_cur_tiles + a.K_eff * a.tiles_per_block;
+  const int n_tiles = k1 - k0;   // K/V tiles of this CTA: global tiles k0 .. k1-1
   const int row0 = qp * 2 * BM;
   const bool has_q1 = row0 + BM < a.S;
 
@@ -163,7 +188,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->p_full[t], 128);
     }
     mbar_init(&bars->fin, 1);
+    mbar_init(&bars->part_done, (has_q1 ? 2 : 1) * 128);
+    mbar_init(&bars->merge_go, 1);
     bars->abort = 0;
+    bars->last = 0;
     fence_barrier_init();
   }
   if (warp == 1) {
@@ -189,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_3d(sQ + t * C::Q_BYTES + b * BM * 128, &tm_q, &bars->q_full, h * HD + b * 64,
                       row0 + t * BM, a.q_frame[i]);
       for (int j = 0; j < n_tiles; ++j) {
-        const TileCoord c = tile_coord(a, i, h, j);
+        const TileCoord c = tile_coord(a, i, h, k0 + j);
         const int s = j % kStages;
         if (aborted(bars) || !mbar_wait(&bars->k_empty[s], ((uint32_t)(j / kStages) & 1u) ^ 1u, lim)) {
           set_abort(bars);
@@ -207,7 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tm_vc);
       tma_prefetch_desc(&tm_vh);
       for (int j = 0; j < n_tiles; ++j) {
-        const TileCoord c = tile_coord(a, i, h, j);
+        const TileCoord c = tile_coord(a, i, h, k0 + j);
         const int s = j % kStages;
         if (aborted(bars) || !mbar_wait(&bars->v_empty[s], ((uint32_t)(j / kStages) & 1u) ^ 1u, lim)) {
           set_abort(bars);
@@ -305,10 +333,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld_x64(tl + colS, sr);
       tmem_ld_x64(tl + colS + 64, sr + 64);
       int valid;
-      if (j < a.n_cur_tiles) {
-        valid = min(BN, a.cur_rows - j * BN);
+      const int jg = k0 + j;   // global K/V tile
+      if (jg < a.n_cur_tiles) {
+        valid = min(BN, a.cur_rows - jg * BN);
       } else {
-        const int jj = j - a.n_cur_tiles;
+        const int jj = jg - a.n_cur_tiles;
         valid = min(BN, a.B_v - (jj % a.tiles_per_block) * BN);
       }
       // columns past the chunk / block end (only in a ragged last tile) get -inf
@@ -372,44 +401,111 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool w = !aborted(bars) && mbar_wait(&bars->fin, 0, lim);
       ok = __all_sync(0xffffffffu, w);
     }
-    if (!ok) {
-      set_abort(bars);
-    } else {
-      tc_fence_after();
-      const int s = row0 + t * BM + row;
-      const float inv = l > 0.f ? 1.f / l : 0.f;
-      const int64_t D = (int64_t)a.H * HD;
-      const int64_t off = ((int64_t)a.o_frame[i] * a.S + s) * D + (int64_t)h * HD;
+    if (!ok) set_abort(bars);
+    tc_fence_after();
+    const int s = row0 + t * BM + row;
+    const int64_t D = (int64_t)a.H * HD;
+    const int64_t off = ((int64_t)a.o_frame[i] * a.S + s) * D + (int64_t)h * HD;
+    // final row: O scaled by inv, written as bf16 or f32
+    auto store_half = [&](int half, const float* v, float inv) {
+      if (a.o_f32) {
+        float* dst = static_cast<float*>(a.o) + off + half * 64;
 #pragma unroll
-      for (int half = 0; half < HD / 64; ++half) {
-        uint32_t orr[64];
-        tmem_ld_x64(tl + colO + half * 64, orr);   // warp-collective: every lane loads
-        if (s < a.S) {
-          if (a.o_f32) {
-            float* dst = static_cast<float*>(a.o) + off + half * 64;
+        for (int c = 0; c < 64; c += 4)
+          *reinterpret_cast<float4*>(dst + c) =
+              make_float4(v[c] * inv, v[c + 1] * inv, v[c + 2] * inv, v[c + 3] * inv);
+      } else {
+        __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(a.o) + off + half * 64;
 #pragma unroll
-            for (int c = 0; c < 64; c += 4)
-              *reinterpret_cast<float4*>(dst + c) =
-                  make_float4(__uint_as_float(orr[c]) * inv, __uint_as_float(orr[c + 1]) * inv,
-                              __uint_as_float(orr[c + 2]) * inv, __uint_as_float(orr[c + 3]) * inv);
-          } else {
-            __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(a.o) + off + half * 64;
+        for (int c = 0; c < 64; c += 8) {
+          uint32_t pk4[4];
 #pragma unroll
-            for (int c = 0; c < 64; c += 8) {
-              uint32_t pk4[4];
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(orr[c + 2 * e]) * inv,
-                                                          __uint_as_float(orr[c + 2 * e + 1]) * inv);
-                pk4[e] = *reinterpret_cast<uint32_t*>(&b2);
-              }
-              *reinterpret_cast<uint4*>(dst + c) = make_uint4(pk4[0], pk4[1], pk4[2], pk4[3]);
-            }
+          for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 b2 = __floats2bfloat162_rn(v[c + 2 * e] * inv, v[c + 2 * e + 1] * inv);
+            pk4[e] = *reinterpret_cast<uint32_t*>(&b2);
           }
+          *reinterpret_cast<uint4*>(dst + c) = make_uint4(pk4[0], pk4[1], pk4[2], pk4[3]);
         }
       }
-      if (a.lse && s < a.S)
-        a.lse[((int64_t)i * a.H + h) * a.S + s] = (m_ref + log2f(l)) * 0.69314718055994531f;
+    };
+    if (!split) {
+      if (ok) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+        for (int half = 0; half < HD / 64; ++half) {
+          uint32_t orr[64];
+          tmem_ld_x64(tl + colO + half * 64, orr);   // warp-collective: every lane loads
+          if (s < a.S) store_half(half, reinterpret_cast<const float*>(orr), inv);
+        }
+        if (a.lse && s < a.S)
+          a.lse[((int64_t)i * a.H + h) * a.S + s] = (m_ref + log2f(l)) * 0.69314718055994531f;
+      }
+    } else {
+      // this part's unnormalised O with its row max (log2 domain) and row sum
+      const int64_t slot0 = ((int64_t)tail_unit * a.n_split) * 2 * BM + t * BM + row;
+      if (ok) {
+        const int64_t slot = slot0 + (int64_t)part * 2 * BM;
+#pragma unroll
+        for (int half = 0; half < HD / 64; ++half) {
+          uint32_t orr[64];
+          tmem_ld_x64(tl + colO + half * 64, orr);
+          float4* dst = reinterpret_cast<float4*>(a.part_o + slot * HD + half * 64);
+#pragma unroll
+          for (int c = 0; c < 64; c += 4)
+            __stcg(dst + c / 4, make_float4(__uint_as_float(orr[c]), __uint_as_float(orr[c + 1]),
+                                            __uint_as_float(orr[c + 2]), __uint_as_float(orr[c + 3])));
+        }
+        __stcg(reinterpret_cast<float2*>(a.part_ml) + slot, make_float2(m_ref, l));
+      }
+      // every softmax thread arrives (also after a failure, so nobody waits forever); one
+      // thread then counts this part in, and the part that completes the count merges
+      mbar_arrive(&bars->part_done);
+      if (warp == 2 && lane == 0) {
+        const bool w = mbar_wait(&bars->part_done, 0, lim);
+        int last = 0;
+        if (w && !aborted(bars)) {
+          __threadfence();
+          last = atomicAdd(&a.counters[tail_unit], 1u) == (unsigned)(a.n_split - 1);
+          __threadfence();
+        } else {
+          set_abort(bars);
+        }
+        bars->last = last;
+        mbar_arrive(&bars->merge_go);
+      }
+      const bool go = mbar_wait(&bars->merge_go, 0, lim);
+      if (go && ok && *reinterpret_cast<volatile int*>(&bars->last) && s < a.S) {
+        const float2* ml = reinterpret_cast<const float2*>(a.part_ml);
+        float mm = -INFINITY, lsum = 0.f;
+        for (int p = 0; p < a.n_split; ++p) mm = fmaxf(mm, __ldcg(ml + slot0 + (int64_t)p * 2 * BM).x);
+        for (int p = 0; p < a.n_split; ++p) {
+          const float2 v = __ldcg(ml + slot0 + (int64_t)p * 2 * BM);
+          lsum += ex2_approx(v.x - mm) * v.y;
+        }
+        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+#pragma unroll
+        for (int half = 0; half < HD / 64; ++half) {
+          float acc[64];
+#pragma unroll
+          for (int c = 0; c < 64; ++c) acc[c] = 0.f;
+          for (int p = 0; p < a.n_split; ++p) {
+            const int64_t sp = slot0 + (int64_t)p * 2 * BM;
+            const float wgt = ex2_approx(__ldcg(ml + sp).x - mm);
+            const float4* src = reinterpret_cast<const float4*>(a.part_o + sp * HD + half * 64);
+#pragma unroll
+            for (int c = 0; c < 64; c += 4) {
+              const float4 v = __ldcg(src + c / 4);
+              acc[c] = fmaf(wgt, v.x, acc[c]);
+              acc[c + 1] = fmaf(wgt, v.y, acc[c + 1]);
+              acc[c + 2] = fmaf(wgt, v.z, acc[c + 2]);
+              acc[c + 3] = fmaf(wgt, v.w, acc[c + 3]);
+            }
+          }
+          store_half(half, acc, inv);
+        }
+        if (a.lse)
+          a.lse[((int64_t)i * a.H + h) * a.S + s] = (mm + log2f(lsum)) * 0.69314718055994531f;
+      }
     }
   }
   tc_fence_before();
@@ -437,7 +533,8 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows,
 }
 
 template <int HD>
-cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream_t st) {
+cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_of_anchor, void* ws,
+                      cudaStream_t st) {
   using C = Cfg<HD>;
   const int D = a.H * HD;
   CUtensorMap mq, mkc, mvc, mkh, mvh;
@@ -458,13 +555,11 @@ cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream
   AttnKArgs k{};
   k.S = a.S;
   k.H = a.H;
-  // query rows per (anchor, head): pairs of 128-row tiles, plus one single tile when the
-  // remainder is at most 128 rows
-  k.n_pairs = a.S / (2 * BM) + (a.S % (2 * BM) > BM ? 1 : 0);
-  k.n_single = (a.S % (2 * BM) > 0 && a.S % (2 * BM) <= BM) ? 1 : 0;
+  k.n_pairs = pl.n_pairs;
+  k.n_single = pl.n_single;
   k.n_anchors = a.n_anchors;
-  k.n_cur_tiles = (int)((cur_rows + BN - 1) / BN);
-  k.tiles_per_block = a.M > 0 ? (a.B_v + BN - 1) / BN : 0;
+  k.n_cur_tiles = pl.n_cur_tiles;
+  k.tiles_per_block = pl.tiles_per_block;
   k.K_eff = a.M > 0 ? a.K_eff : 0;
   k.M = a.M;
   k.cur_rows = (int)cur_rows;
@@ -473,6 +568,13 @@ cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream
   k.o = a.o;
   k.o_f32 = a.o_dtype == CAST_F32;
   k.lse = a.lse;
+  k.n_full = pl.n_full;
+  k.n_split = pl.n_split;
+  k.chunk = pl.chunk;
+  char* w = static_cast<char*>(ws);
+  k.part_o = reinterpret_cast<float*>(w);
+  k.part_ml = reinterpret_cast<float*>(w + pl.part_o_bytes);
+  k.counters = reinterpret_cast<unsigned*>(w + pl.part_o_bytes + pl.part_ml_bytes);
   const float scale = a.scale > 0.f ? a.scale : 1.f / sqrtf((float)HD);
   k.scale_log2 = scale * 1.4426950408889634f;
   k.wait_ns = 2000000000ull;
@@ -487,16 +589,58 @@ cast_status launch_hd(const cast_attn_args& a, int o_frame_of_anchor, cudaStream
       return check_launch("attention smem attribute");
     attr_set = true;
   }
-  const int grid = (k.n_pairs + k.n_single) * a.n_anchors * a.H;
-  k_attn<HD><<<grid, kThreads, C::SMEM, st>>>(mq, mkc, mvc, mkh, mvh, k);
+  if (pl.n_tail > 0 &&
+      cudaMemsetAsync(k.counters, 0, (size_t)pl.n_tail * sizeof(unsigned), st) != cudaSuccess)
+    return check_launch("attention counter reset");
+  k_attn<HD><<<pl.grid, kThreads, C::SMEM, st>>>(mq, mkc, mvc, mkh, mvh, k);
   return check_launch("attention kernel");
 }
 
 }  // namespace
 
-cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, cudaStream_t st) {
-  if (a.d == 128) return launch_hd<128>(a, o_frame_of_anchor, st);
-  return launch_hd<64>(a, o_frame_of_anchor, st);
+AttnPlan attention_plan(const cast_attn_args& a) {
+  AttnPlan p{};
+  p.n_pairs = a.S / (2 * BM) + (a.S % (2 * BM) > BM ? 1 : 0);
+  p.n_single = (a.S % (2 * BM) > 0 && a.S % (2 * BM) <= BM) ? 1 : 0;
+  p.n_cur_tiles = (int)(((int64_t)a.n_frames * a.S + BN - 1) / BN);
+  p.tiles_per_block = a.M > 0 ? (a.B_v + BN - 1) / BN : 0;
+  const int n_tiles = p.n_cur_tiles + (a.M > 0 ? a.K_eff : 0) * p.tiles_per_block;
+  const int units = (p.n_pairs + p.n_single) * a.n_anchors * a.H;
+  int dev = 0, nsm = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  if (nsm < 1) nsm = 1;
+  // whole rounds of one unit per SM run unsplit; the units of the last, partial round are
+  // split along K/V over the SMs (never into parts of fewer than 4 tiles)
+  const int rounds = units / nsm;
+  const int tail = units - rounds * nsm;
+  int n_split = tail > 0 ? nsm / tail : 1;
+  if (n_split > n_tiles / 4) n_split = n_tiles / 4;
+  if (n_split < 2) {
+    p.n_full = units;
+    p.n_tail = 0;
+    p.n_split = 1;
+    p.chunk = n_tiles;
+  } else {
+    p.chunk = (n_tiles + n_split - 1) / n_split;
+    n_split = (n_tiles + p.chunk - 1) / p.chunk;   // no empty part
+    p.n_full = rounds * nsm;
+    p.n_tail = tail;
+    p.n_split = n_split;
+  }
+  p.grid = p.n_full + p.n_tail * p.n_split;
+  const size_t rows = (size_t)p.n_tail * p.n_split * 2 * BM;
+  p.part_o_bytes = align_up(rows * a.d * sizeof(float));
+  p.part_ml_bytes = align_up(rows * 2 * sizeof(float));
+  p.counter_bytes = align_up((size_t)(p.n_tail > 0 ? p.n_tail : 1) * sizeof(unsigned));
+  p.total_bytes = p.n_tail > 0 ? p.part_o_bytes + p.part_ml_bytes + p.counter_bytes : 0;
+  return p;
+}
+
+cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, void* ws,
+                             cudaStream_t st) {
+  const AttnPlan pl = attention_plan(a);
+  if (a.d == 128) return launch_hd<128>(a, pl, o_frame_of_anchor, ws, st);
+  return launch_hd<64>(a, pl, o_frame_of_anchor, ws, st);
 }
 
 unsigned int attention_error_word(cudaStream_t st, bool clear) {

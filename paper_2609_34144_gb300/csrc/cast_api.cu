@@ -248,9 +248,9 @@ cast_attn_args attn_of_block(const cast_block_args* a, const int32_t* idx) {
   return t;
 }
 
-// block-step workspace: [route ws][idx (when idx_out is NULL)][par ws]
+// block-step workspace: [route ws][idx (when idx_out is NULL)][attention ws][par ws]
 struct BlockPlan {
-  size_t route_bytes, idx_bytes, par_bytes, total;
+  size_t route_bytes, idx_bytes, attn_bytes, par_bytes, total;
 };
 BlockPlan block_plan(const cast_block_args* a) {
   BlockPlan b{};
@@ -259,10 +259,12 @@ BlockPlan block_plan(const cast_block_args* a) {
   b.route_bytes = (a->M > 0 && a->K > 0) ? route_plan(r).total_bytes : 0;
   const int keff = a->K < a->M ? a->K : a->M;
   b.idx_bytes = a->idx_out ? 0 : align_up((size_t)a->n_anchors * a->H * (keff > 0 ? keff : 1) * 4);
+  cast_attn_args t = attn_of_block(a, nullptr);
+  b.attn_bytes = align_up(attention_plan(t).total_bytes);
   uint8_t mask[CAST_MAX_FRAMES];
   cast_par_args p = par_of_block(a, mask);
   b.par_bytes = par_plan(p).total_bytes;
-  b.total = b.route_bytes + b.idx_bytes + b.par_bytes;
+  b.total = b.route_bytes + b.idx_bytes + b.attn_bytes + b.par_bytes;
   return b;
 }
 
@@ -323,11 +325,22 @@ cast_status cast_route_topk(const cast_route_args* a, void* ws, size_t ws_bytes,
   return launch_route(*a, ws, static_cast<cudaStream_t>(stream));
 }
 
-cast_status cast_anchor_attention(const cast_attn_args* a, void* stream) {
+size_t cast_attention_workspace_size(const cast_attn_args* a) {
+  if (!a || a->n_anchors < 1 || a->H < 1 || a->S < 1 || a->n_frames < 1 || (a->d != 64 && a->d != 128))
+    return 0;
+  return attention_plan(*a).total_bytes;
+}
+
+cast_status cast_anchor_attention(const cast_attn_args* a, void* ws, size_t ws_bytes, void* stream) {
   g_detail[0] = 0;
   cast_status s = validate_attn(a);
   if (s) return s;
-  return launch_attention(*a, 0, static_cast<cudaStream_t>(stream));
+  const size_t need = attention_plan(*a).total_bytes;
+  if (need > 0 && (ws_bytes < need || !ws))
+    return fail(CAST_ERR_INVALID_ARG, "cast_anchor_attention: workspace %zu B < %zu B", ws_bytes, need);
+  if (need > 0 && reinterpret_cast<uintptr_t>(ws) % kWsAlign)
+    return fail(CAST_ERR_INVALID_ARG, "cast_anchor_attention: workspace not 256-byte aligned");
+  return launch_attention(*a, 0, ws, static_cast<cudaStream_t>(stream));
 }
 
 size_t cast_par_workspace_size(const cast_par_args* a) {
@@ -388,9 +401,9 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
   if (a->M > 0 && a->K > 0) {
     if ((s = launch_route(r, w, st))) return s;
   }
-  if ((s = launch_attention(t, 1, st))) return s;
+  if ((s = launch_attention(t, 1, w + bp.route_bytes + bp.idx_bytes, st))) return s;
   if (par_plan(p).n_target > 0) {
-    if ((s = launch_par(p, w + bp.route_bytes + bp.idx_bytes, st))) return s;
+    if ((s = launch_par(p, w + bp.route_bytes + bp.idx_bytes + bp.attn_bytes, st))) return s;
   }
   if (a->x) {
     const size_t n = (size_t)a->n_frames * a->Hg * a->Wg * a->H * a->d;

@@ -37,9 +37,17 @@ RoutePlan route_plan(const cast_route_args& a);
 cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st);
 
 // ------------------------------------------------------------------ attention
+struct AttnPlan {
+  int n_pairs, n_single, n_cur_tiles, tiles_per_block;
+  int n_full, n_tail, n_split, chunk, grid;
+  size_t part_o_bytes, part_ml_bytes, counter_bytes, total_bytes;
+};
+AttnPlan attention_plan(const cast_attn_args& a);
 // o_frame_of_anchor: 0 -> output frame i for anchor i (o is [n_anchors, S, H*d]);
 //                    1 -> output frame anchors[i] (o is [n_frames, S, H*d], block step).
-cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, cudaStream_t st);
+// ws holds attention_plan(a).total_bytes (may be null when that is 0).
+cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, void* ws,
+                             cudaStream_t st);
 unsigned int attention_error_word(cudaStream_t st, bool clear);
 
 // ------------------------------------------------------------------ PAR

@@ -73,7 +73,9 @@ _lib.cast_route_topk.argtypes = [C.POINTER(RouteArgs), _vp, C.c_size_t, _vp]
 _lib.cast_route_workspace_size.argtypes = [C.POINTER(RouteArgs)]
 _lib.cast_route_workspace_size.restype = C.c_size_t
 _lib.cast_route_topk_noalloc.argtypes = [C.POINTER(RouteArgs), _vp]
-_lib.cast_anchor_attention.argtypes = [C.POINTER(AttnArgs), _vp]
+_lib.cast_anchor_attention.argtypes = [C.POINTER(AttnArgs), _vp, C.c_size_t, _vp]
+_lib.cast_attention_workspace_size.argtypes = [C.POINTER(AttnArgs)]
+_lib.cast_attention_workspace_size.restype = C.c_size_t
 _lib.cast_par_reconstruct.argtypes = [C.POINTER(ParArgs), _vp, C.c_size_t, _vp]
 _lib.cast_par_workspace_size.argtypes = [C.POINTER(ParArgs)]
 _lib.cast_par_workspace_size.restype = C.c_size_t
@@ -90,7 +92,8 @@ for _f in ("cast_route_topk", "cast_route_topk_noalloc", "cast_anchor_attention"
            "cast_check_device"):
     getattr(_lib, _f).restype = C.c_int
 
-EXPORTED = ["cast_route_topk", "cast_route_workspace_size", "cast_route_topk_noalloc", "cast_anchor_attention",
+EXPORTED = ["cast_route_topk", "cast_route_workspace_size", "cast_route_topk_noalloc",
+            "cast_anchor_attention", "cast_attention_workspace_size",
             "cast_par_reconstruct", "cast_par_workspace_size", "cast_par_params_default",
             "cast_block_step", "cast_block_workspace_size", "cast_status_string",
             "cast_last_error_detail", "cast_check_device", "cast_version"]
@@ -226,11 +229,8 @@ def cast_route_topk_noalloc(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8,
 
 
 # --------------------------------------------------------------------------- attention
-def cast_anchor_attention(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale=0.0,
-                          out_dtype=torch.bfloat16, want_lse=False, out=None, stream=None):
-    """Returns O [K_f, S, H*d] (and lse [K_f, H, S])."""
+def _attn_args(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale=0.0):
     N, S, H, d = q.shape
-    Kf = len(anchors)
     M = k_hist.shape[0] if k_hist is not None else 0
     a = AttnArgs()
     a.q, a.k_cur, a.v_cur = _ptr(q), _ptr(k_cur), _ptr(v_cur)
@@ -238,7 +238,7 @@ def cast_anchor_attention(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale=0
     a.n_frames, a.S, a.H, a.d = N, S, H, d
     a._anchors = _host_i32(anchors)
     a.anchors = C.cast(a._anchors, C.POINTER(_i32))
-    a.n_anchors = Kf
+    a.n_anchors = len(anchors)
     a.k_hist, a.v_hist = _ptr(k_hist), _ptr(v_hist)
     a.hist_row_stride = _row_stride(k_hist) if M > 0 else H * d
     a.M = M
@@ -246,11 +246,28 @@ def cast_anchor_attention(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale=0
     a.idx = _ptr(idx)
     a.K_eff = idx.shape[-1] if idx is not None else 0
     a.scale = scale
+    return a
+
+
+def attention_workspace_size(q, k_cur, v_cur, anchors, k_hist, v_hist, idx):
+    a = _attn_args(q, k_cur, v_cur, anchors, k_hist, v_hist, idx)
+    return _lib.cast_attention_workspace_size(C.byref(a))
+
+
+def cast_anchor_attention(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale=0.0,
+                          out_dtype=torch.bfloat16, want_lse=False, out=None, workspace=None,
+                          stream=None):
+    """Returns O [K_f, S, H*d] (and lse [K_f, H, S])."""
+    N, S, H, d = q.shape
+    Kf = len(anchors)
+    a = _attn_args(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale)
     o = out if out is not None else torch.empty((Kf, S, H * d), dtype=out_dtype, device=q.device)
     a.o, a.o_dtype = _ptr(o), _dtype_code(o)
     lse = torch.empty((Kf, H, S), dtype=torch.float32, device=q.device) if want_lse else None
     a.lse = _ptr(lse)
-    _check(_lib.cast_anchor_attention(C.byref(a), _stream(stream)))
+    need = _lib.cast_attention_workspace_size(C.byref(a))
+    ws = workspace if workspace is not None else _workspace(need, q.device)
+    _check(_lib.cast_anchor_attention(C.byref(a), _ptr(ws), ws.numel(), _stream(stream)))
     return (o, lse) if want_lse else o
 
 

@@ -147,6 +147,6 @@ def test_attention_validation(lib):
     a.n_anchors = 1
     a.M, a.B_v, a.K_eff = 0, 1, 1          # routed blocks without history
     a.o, a.o_dtype = _fake(), lib.BF16
-    assert lib.library().cast_anchor_attention(C.byref(a), None) == 1
+    assert lib.library().cast_anchor_attention(C.byref(a), None, 0, None) == 1
     a.K_eff, a.d = 0, 80
-    assert lib.library().cast_anchor_attention(C.byref(a), None) == 2
+    assert lib.library().cast_anchor_attention(C.byref(a), None, 0, None) == 2
