@@ -32,10 +32,115 @@ constexpr int kThreads = 128;      // channels per item
 constexpr int kNB = 40;            // stored bins of an 8-wide tile: 8 x 5
 constexpr int kNV = 3 * kNB;       // (Re Z, Im Z, W) per bin, record index = 3 * bin + component
 constexpr int kMaxSeg = 128;
-constexpr int kCoefBatch = 8;
+constexpr int kCoefBatch = 4;
 constexpr int kSpecFloats = 2 * kNB * kThreads;   // one spectrum per thread, [value][thread]
 
 __device__ unsigned int g_par_error;   // 1: a wait gave up
+
+// Non-redundant (bin, component) values of an 8x8 tile's Z / W record, encoded bin * 4 +
+// component (0: Re Z, 1: Im Z, 2: W): mirrors (ky > 4 in the kx = 0 and kx = 4 columns) are
+// conjugates of their representatives, the self-conjugate bins have Im Z = 0, and DC needs
+// only W (reduced separately).  96 values = three 32-value transpose groups.
+__host__ __device__ __forceinline__ constexpr int fast_value(int n) {
+  return
+      n == 0 ? 4 :
+      n == 1 ? 5 :
+      n == 2 ? 6 :
+      n == 3 ? 8 :
+      n == 4 ? 9 :
+      n == 5 ? 10 :
+      n == 6 ? 12 :
+      n == 7 ? 13 :
+      n == 8 ? 14 :
+      n == 9 ? 16 :
+      n == 10 ? 18 :
+      n == 11 ? 20 :
+      n == 12 ? 21 :
+      n == 13 ? 22 :
+      n == 14 ? 24 :
+      n == 15 ? 25 :
+      n == 16 ? 26 :
+      n == 17 ? 28 :
+      n == 18 ? 29 :
+      n == 19 ? 30 :
+      n == 20 ? 32 :
+      n == 21 ? 33 :
+      n == 22 ? 34 :
+      n == 23 ? 36 :
+      n == 24 ? 37 :
+      n == 25 ? 38 :
+      n == 26 ? 40 :
+      n == 27 ? 41 :
+      n == 28 ? 42 :
+      n == 29 ? 44 :
+      n == 30 ? 45 :
+      n == 31 ? 46 :
+      n == 32 ? 48 :
+      n == 33 ? 49 :
+      n == 34 ? 50 :
+      n == 35 ? 52 :
+      n == 36 ? 53 :
+      n == 37 ? 54 :
+      n == 38 ? 56 :
+      n == 39 ? 57 :
+      n == 40 ? 58 :
+      n == 41 ? 60 :
+      n == 42 ? 61 :
+      n == 43 ? 62 :
+      n == 44 ? 64 :
+      n == 45 ? 65 :
+      n == 46 ? 66 :
+      n == 47 ? 68 :
+      n == 48 ? 69 :
+      n == 49 ? 70 :
+      n == 50 ? 72 :
+      n == 51 ? 73 :
+      n == 52 ? 74 :
+      n == 53 ? 76 :
+      n == 54 ? 77 :
+      n == 55 ? 78 :
+      n == 56 ? 80 :
+      n == 57 ? 82 :
+      n == 58 ? 84 :
+      n == 59 ? 85 :
+      n == 60 ? 86 :
+      n == 61 ? 88 :
+      n == 62 ? 89 :
+      n == 63 ? 90 :
+      n == 64 ? 92 :
+      n == 65 ? 93 :
+      n == 66 ? 94 :
+      n == 67 ? 96 :
+      n == 68 ? 98 :
+      n == 69 ? 104 :
+      n == 70 ? 105 :
+      n == 71 ? 106 :
+      n == 72 ? 108 :
+      n == 73 ? 109 :
+      n == 74 ? 110 :
+      n == 75 ? 112 :
+      n == 76 ? 113 :
+      n == 77 ? 114 :
+      n == 78 ? 124 :
+      n == 79 ? 125 :
+      n == 80 ? 126 :
+      n == 81 ? 128 :
+      n == 82 ? 129 :
+      n == 83 ? 130 :
+      n == 84 ? 132 :
+      n == 85 ? 133 :
+      n == 86 ? 134 :
+      n == 87 ? 144 :
+      n == 88 ? 145 :
+      n == 89 ? 146 :
+      n == 90 ? 148 :
+      n == 91 ? 149 :
+      n == 92 ? 150 :
+      n == 93 ? 152 :
+      n == 94 ? 153 :
+      n == 95 ? 154 :
+      0;
+}
 
 struct ParKArgs {
   char* r;
@@ -55,6 +160,9 @@ struct ParKArgs {
   float tau_low, tau_high, q, T, eps, eta_rel, eta_abs, band;
   int gate_mode;
   unsigned long long wait_ns;
+  // 8x8 tiles: record entry t (3 * bin + component) = sign * reduced value |fast_src[t]| - 1,
+  // 0 = not needed (Z at DC) or identically zero (Im Z at self-conjugate bins)
+  signed char fast_src[kNV];
 };
 
 template <typename T>
@@ -64,8 +172,6 @@ __device__ __forceinline__ float to_f32<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
 
-__device__ __forceinline__ void st_stream(float* p, float v) { __stcs(p, v); }
-__device__ __forceinline__ void st_stream(__nv_bfloat16* p, float v) { __stcs(p, __float2bfloat16_rn(v)); }
 
 __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
   unsigned v;
@@ -193,7 +299,9 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float
 template <typename T>
 constexpr size_t stage_bytes() { return (size_t)64 * kThreads * sizeof(T); }
 template <typename T>
-constexpr size_t par_dyn_smem() { return stage_bytes<T>() + kSpecFloats * sizeof(float) + 1024; }
+constexpr size_t par_dyn_smem() {
+  return 2 * stage_bytes<T>() + kSpecFloats * sizeof(float) + 128;   // in, out, previous spectrum
+}
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 2)
@@ -201,9 +309,10 @@ __global__ void __launch_bounds__(kThreads, 2)
           float* __restrict__ partial, unsigned* __restrict__ counters) {
   extern __shared__ uint8_t dsm_raw[];
   const uint32_t raw = smem_u32(dsm_raw);
-  uint8_t* dsm = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+  uint8_t* dsm = dsm_raw + (((raw + 127u) & ~127u) - raw);   // TMA boxes without swizzle: 128 B
   const T* stage = reinterpret_cast<const T*>(dsm);          // [y][x][channel] of one anchor tile
   float* s_fprev = reinterpret_cast<float*>(dsm + stage_bytes<T>());   // [value][thread]
+  T* ostage = reinterpret_cast<T*>(dsm + stage_bytes<T>() + kSpecFloats * sizeof(float));
   __shared__ float s_red[kThreads / 32][128];
   __shared__ float s_zw[kNV];
   __shared__ float s_th[kNB], s_g[kNB], s_own_th[kNB];
@@ -262,11 +371,18 @@ __global__ void __launch_bounds__(kThreads, 2)
         const bool ok = mbar_wait(&s_full, n_loaded & 1u, a.wait_ns);
         ++n_loaded;
         float x[8][8];
+        if (a.tw == 8 && a.th == 8) {
 #pragma unroll
-        for (int y = 0; y < 8; ++y)
+          for (int y = 0; y < 8; ++y)
 #pragma unroll
-          for (int xx = 0; xx < 8; ++xx)
-            x[y][xx] = (y < a.th && xx < a.tw) ? to_f32(stage[(y * a.tw + xx) * kThreads + tid]) : 0.f;
+            for (int xx = 0; xx < 8; ++xx) x[y][xx] = to_f32(stage[(y * 8 + xx) * kThreads + tid]);
+        } else {
+#pragma unroll
+          for (int y = 0; y < 8; ++y)
+#pragma unroll
+            for (int xx = 0; xx < 8; ++xx)
+              x[y][xx] = (y < a.th && xx < a.tw) ? to_f32(stage[(y * a.tw + xx) * kThreads + tid]) : 0.f;
+        }
         // the stage is free: prefetch the next anchor while transforming this one.  A tile
         // that never arrived ends the kernel for every thread of the CTA (error word set);
         // the barrier is never re-armed in an incomplete phase.
@@ -285,33 +401,69 @@ __global__ void __launch_bounds__(kThreads, 2)
       const float* fa = s_fprev;   // spectrum of anchor j-1 (this thread's column)
       if (has_targets && !recon) {
         // ---- partial Z = sum w F_b conj(F_a), W = sum w |F_b||F_a| over the chunk (Eq. cross)
+        if (g.h == 8 && g.w == 8) {
+          // the 96 non-redundant values in three transpose groups, W at DC by a warp sum
 #pragma unroll
-        for (int grp = 0; grp < 4; ++grp) {
-          float v[32];
+          for (int grp = 0; grp < 3; ++grp) {
+            float v[32];
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int vi = grp * 32 + e;
-            if (vi < kNV) {
-              const int b = vi / 3, comp = vi % 3;
+            for (int e = 0; e < 32; ++e) {
+              const int code = fast_value(grp * 32 + e);
+              const int b = code >> 2, comp = code & 3;
               const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
               const float br = re[b / 5][b % 5], bi = im[b / 5][b % 5];
               v[e] = comp == 0 ? wc * (br * ar + bi * ai)
                    : comp == 1 ? wc * (bi * ar - br * ai)
                                : wc * sqrtf((ar * ar + ai * ai) * (br * br + bi * bi));
-            } else {
-              v[e] = 0.f;
             }
+            s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
           }
-          s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
-        }
-        __syncthreads();
-        if (tid < kNV) {
-          float s = 0.f;
+          float wdc = wc * fabsf(re[0][0]) * fabsf(fa[tid]);
 #pragma unroll
-          for (int w = 0; w < kThreads / 32; ++w) s += s_red[w][tid];
-          partial[(((int64_t)j * a.n_tile + tile) * a.n_chunk + chunk) * kNV + tid] = s;
+          for (int o = 16; o > 0; o >>= 1) wdc += __shfl_xor_sync(0xffffffffu, wdc, o);
+          if (lane == 0) s_red[warp][96] = wdc;
+          __syncthreads();
+          if (tid < kNV) {
+            const int src = a.fast_src[tid];
+            float sum = 0.f;
+            if (src != 0) {
+              const int k = (src > 0 ? src : -src) - 1;
+#pragma unroll
+              for (int w = 0; w < kThreads / 32; ++w) sum += s_red[w][k];
+              if (src < 0) sum = -sum;
+            }
+            partial[(((int64_t)j * a.n_tile + tile) * a.n_chunk + chunk) * kNV + tid] = sum;
+          }
+          __syncthreads();
+        } else {
+#pragma unroll
+          for (int grp = 0; grp < 4; ++grp) {
+            float v[32];
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const int vi = grp * 32 + e;
+              if (vi < kNV) {
+                const int b = vi / 3, comp = vi % 3;
+                const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
+                const float br = re[b / 5][b % 5], bi = im[b / 5][b % 5];
+                v[e] = comp == 0 ? wc * (br * ar + bi * ai)
+                     : comp == 1 ? wc * (bi * ar - br * ai)
+                                 : wc * sqrtf((ar * ar + ai * ai) * (br * br + bi * bi));
+              } else {
+                v[e] = 0.f;
+              }
+            }
+            s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
+          }
+          __syncthreads();
+          if (tid < kNV) {
+            float sum = 0.f;
+#pragma unroll
+            for (int w = 0; w < kThreads / 32; ++w) sum += s_red[w][tid];
+            partial[(((int64_t)j * a.n_tile + tile) * a.n_chunk + chunk) * kNV + tid] = sum;
+          }
+          __syncthreads();
         }
-        __syncthreads();
       } else if (has_targets && recon) {
         // ---- transport of pair (j-1, j) on this tile
         if (tid < kNV) {
@@ -357,18 +509,26 @@ __global__ void __launch_bounds__(kThreads, 2)
               hr[ky][kx] = cf.x * ar - cf.y * ai + cf.z * br - cf.w * bi;
               hi[ky][kx] = cf.x * ai + cf.y * ar + cf.z * bi + cf.w * br;
             }
-            T* out = reinterpret_cast<T*>(a.r) +
-                     (((int64_t)a.target_frame[t0 + k] * a.Hg + g.y0) * rowC + (int64_t)g.x0 * a.C + c);
-            const int Cs = a.C;
-            const int w = g.w;
+            // the previous tile store must have finished reading the out stage
+            if (tid == 0) bulk_wait_read_all();
+            __syncthreads();
+            const int tw = a.tw;
             dft::inv2d_emit(hr, hi, g.h, g.w, [&](int yy, const float* row) {
-              if (active) {
-                T* p = out + yy * rowC;
+              if (tw == 8) {
+#pragma unroll
+                for (int xx = 0; xx < 8; ++xx) ostage[(yy * 8 + xx) * kThreads + tid] = T(row[xx]);
+              } else {
 #pragma unroll
                 for (int xx = 0; xx < 8; ++xx)
-                  if (xx < w) st_stream(p + xx * Cs, row[xx]);
+                  if (xx < tw) ostage[(yy * tw + xx) * kThreads + tid] = T(row[xx]);
               }
             });
+            fence_proxy_async_smem();
+            __syncthreads();
+            if (tid == 0) {
+              tma_store_4d(&tm, ostage, chunk * kThreads, g.x0, g.y0, a.target_frame[t0 + k]);
+              bulk_commit();
+            }
           }
           __syncthreads();
         }
@@ -390,6 +550,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
     }
   }
+  if (tid == 0) bulk_wait_all();   // tile stores complete before the CTA's shared memory goes
 }
 
 // 4-D map [F][Hg][Wg][C], box (128 channels, tw, th, 1), zero fill out of range
@@ -528,6 +689,24 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
   k.band = pp.band_radius;
   k.gate_mode = pp.gate_mode;
   k.wait_ns = 2000000000ull;
+  {
+    // record entry t = 3 * bin + comp of an 8x8 tile from the 96 reduced values (+ W at DC = 96)
+    int pos[40 * 4];
+    for (int q = 0; q < 160; ++q) pos[q] = -1;
+    for (int n = 0; n < 96; ++n) pos[fast_value(n)] = n;
+    for (int t = 0; t < kNV; ++t) {
+      const int b = t / 3, comp = t % 3, ky = b / 5, kx = b % 5;
+      const bool edge = kx == 0 || kx == 4;
+      const bool selfc = edge && (ky == 0 || ky == 4);
+      const bool mirror = edge && !selfc && ky > 4;
+      const int r = mirror ? (8 - ky) * 5 + kx : b;
+      int src = 0;
+      if (r == 0) src = comp == 2 ? 96 + 1 : 0;                 // DC: only W
+      else if (comp == 1 && selfc) src = 0;                     // Im Z of a real bin
+      else src = (pos[r * 4 + comp] + 1) * ((mirror && comp == 1) ? -1 : 1);
+      k.fast_src[t] = (signed char)src;
+    }
+  }
 
   CUtensorMap tm;
   if (!make_r_map(&tm, a)) return fail(CAST_ERR_CUDA, "PAR: cuTensorMapEncodeTiled failed");
