@@ -391,3 +391,136 @@ def block_step(inp, K, grid, p: ParParams = ParParams(), eps=1e-8, idx=None, O=N
     mask[anchors] = 1
     r = par_reconstruct(r.reshape(N, grid[0], grid[1], H * d), mask, None, p)
     return idx, O, r.reshape(N, S, H * d)
+
+
+# ===========================================================================
+# Reconstruction-coupled routing refinement (Section 4.4, Eqs. abc, risk,
+# objective, topk; App. B.2 Eqs. abcclosed, boundarycoeff, boundaryrisk;
+# App. B.3 Eqs. gain, boundarygain, Alg. routing; Tab. config_cast)
+# ===========================================================================
+
+
+@dataclass
+class RoutingCoefficients:
+    """Interval coefficients of the adjacent anchor pairs (index j: anchors j-1, j) and of the
+    two boundary sets (L: frames before anchor 0, pair (0, 1); R: frames after the last anchor,
+    pair (J-1, J)).  Anchor positions are indices into the ordered anchor list."""
+    A: np.ndarray   # [n_anchors] (entry 0 unused)
+    B: np.ndarray
+    C: np.ndarray
+    AL: float
+    BL: float
+    CL: float
+    AR: float
+    BR: float
+    CR: float
+
+
+def routing_coefficients(anchors, n_frames) -> RoutingCoefficients:
+    """Eq. (abc) over each interval's skipped frames and Eq. (boundarycoeff) over the boundary
+    sets, with the alpha of Eq. (block)."""
+    an = [int(a) for a in anchors]
+    J = len(an)
+    A = np.zeros(J)
+    B = np.zeros(J)
+    C = np.zeros(J)
+    for j in range(1, J):
+        a, b = an[j - 1], an[j]
+        al = np.array([(t - a) / (b - a) for t in range(a + 1, b)])
+        A[j] = np.sum((1 - al) ** 2)
+        B[j] = np.sum(al ** 2)
+        C[j] = np.sum(al * (1 - al))
+    AL = BL = CL = AR = BR = CR = 0.0
+    if J >= 2:
+        a, b = an[0], an[1]
+        al = np.array([(t - a) / (b - a) for t in range(0, a)])
+        AL, BL, CL = np.sum((1 - al) ** 2), np.sum(al ** 2), np.sum(np.abs(al * (1 - al)))
+        a, b = an[-2], an[-1]
+        al = np.array([(t - a) / (b - a) for t in range(b + 1, n_frames)])
+        AR, BR, CR = np.sum((1 - al) ** 2), np.sum(al ** 2), np.sum(np.abs(al * (1 - al)))
+    return RoutingCoefficients(A, B, C, float(AL), float(BL), float(CL), float(AR), float(BR),
+                               float(CR))
+
+
+def _pair_risk(A, B, C, xa, xb, ua, ub):
+    """Eq. (risk) summed over blocks: A (1-x_a) u_a + B (1-x_b) u_b + 2C (1-x_a)(1-x_b) sqrt(u_a u_b)."""
+    return np.sum(A * (1 - xa) * ua + B * (1 - xb) * ub + 2 * C * (1 - xa) * (1 - xb) * np.sqrt(ua * ub))
+
+
+def routing_objective(u, x, co: RoutingCoefficients, lam_anc=1.0, lam_rec=1.0):
+    """Eq. (objective) for one head: u, x [n_anchors, M] (x binary)."""
+    J = u.shape[0]
+    val = lam_anc * np.sum((1 - x) * u)
+    rec = 0.0
+    for j in range(1, J):
+        rec += _pair_risk(co.A[j], co.B[j], co.C[j], x[j - 1], x[j], u[j - 1], u[j])
+    if J >= 2:   # Eq. (boundaryrisk): both sets, also when they share the pair (K_f = 2)
+        rec += _pair_risk(co.AL, co.BL, co.CL, x[0], x[1], u[0], u[1])
+        rec += _pair_risk(co.AR, co.BR, co.CR, x[J - 2], x[J - 1], u[J - 2], u[J - 1])
+    return float(val + lam_rec * rec)
+
+
+def retain_gains(i, u, x, co: RoutingCoefficients, lam_anc=1.0, lam_rec=1.0):
+    """Eq. (gain) with Eq. (boundarygain): G_{i,m}, the decrease of J when anchor i keeps m."""
+    J = u.shape[0]
+    G = lam_anc * u[i].copy()
+    if i >= 1:      # left neighbour, interval (i-1, i)
+        l = i - 1
+        G += lam_rec * (co.B[i] * u[i] + 2 * co.C[i] * (1 - x[l]) * np.sqrt(u[l] * u[i]))
+    if i + 1 < J:   # right neighbour, interval (i, i+1)
+        r = i + 1
+        G += lam_rec * (co.A[r] * u[i] + 2 * co.C[r] * (1 - x[r]) * np.sqrt(u[i] * u[r]))
+    if J >= 2:
+        for (aq, bq, Aq, Bq, Cq) in ((0, 1, co.AL, co.BL, co.CL),
+                                     (J - 2, J - 1, co.AR, co.BR, co.CR)):
+            if i == aq:
+                G += lam_rec * (Aq * u[i] + 2 * Cq * (1 - x[bq]) * np.sqrt(u[i] * u[bq]))
+            if i == bq:
+                G += lam_rec * (Bq * u[i] + 2 * Cq * (1 - x[aq]) * np.sqrt(u[i] * u[aq]))
+    return G
+
+
+def _mask_from_topk(score, K):
+    x = np.zeros_like(score)
+    if score.size:
+        x[topk_blocks(score[None], K)[0]] = 1.0
+    return x
+
+
+def coupled_routing(u, anchors, n_frames, K, passes=2, lam_anc=1.0, lam_rec=1.0, tol=1e-6,
+                    with_info=False):
+    """Alg. (routing) for one head: u [n_anchors, M] omission scores.  Initialise every mask
+    with TopK(u_i), then `passes` directional passes (forward, backward, ...) replacing M_i by
+    TopK(G_i) when J drops by more than tol * max(J, 1e-8); stop after a pass with no change.
+    Returns idx [n_anchors, K_eff] ascending (and the objective trace with with_info)."""
+    u = np.asarray(u, dtype=np.float64)
+    J_, M = u.shape
+    keff = min(K, M)
+    co = routing_coefficients(anchors, n_frames)
+    x = np.stack([_mask_from_topk(u[i], keff) for i in range(J_)]) if M else np.zeros((J_, 0))
+    trace = [routing_objective(u, x, co, lam_anc, lam_rec)]
+    ambiguous = False
+    if 0 < keff < M:
+        for s in range(1, passes + 1):
+            changed = False
+            order = range(J_) if s % 2 == 1 else range(J_ - 1, -1, -1)
+            for i in order:
+                G = retain_gains(i, u, x, co, lam_anc, lam_rec)
+                new = _mask_from_topk(G, keff)
+                gain = float(np.sum(G * new) - np.sum(G * x[i]))
+                Jcur = routing_objective(u, x, co, lam_anc, lam_rec)
+                thr = tol * max(Jcur, 1e-8)
+                srt = -np.sort(-G)
+                if abs(gain - thr) <= 1e-4 * max(thr, 1e-12) or (
+                        srt[keff - 1] - srt[keff] <= 1e-4 * max(abs(srt[keff - 1]), 1e-12)):
+                    ambiguous = True
+                if gain > thr:
+                    x[i] = new
+                    changed = True
+                    trace.append(routing_objective(u, x, co, lam_anc, lam_rec))
+            if not changed:
+                break
+    idx = np.stack([np.flatnonzero(x[i]) for i in range(J_)]) if keff else np.zeros((J_, 0), int)
+    if with_info:
+        return idx, {"trace": trace, "ambiguous": ambiguous, "x": x, "coefficients": co}
+    return idx

@@ -450,4 +450,94 @@ def check_attention_dense_limit():
     assert np.allclose(O.routed_attention(q, kc, vc, kh, vh, anchors, perm), out, atol=1e-12)
 
 
+# ---------------------------------------------------------------------------
+# Coupled routing refinement (Section 4.4 Eqs. abc, risk, objective, topk; App. B.2, B.3)
+# ---------------------------------------------------------------------------
+
+
+def check_routing_coefficients():
+    """Interior coefficients equal the closed forms of Eq. (abcclosed); boundary coefficients make
+    the frozen-transport extrapolation bound (App. B.2) hold and be attained: with U and g frozen,
+    sum over the boundary frames of ||(1-a) T_a v_a + a T_b v_b||^2 is at most
+    A_q |v_a|^2 + B_q |v_b|^2 + 2 C_q |v_a| |v_b|, with equality for g = 0 and v_b = -v_a."""
+    for n, A_ref, C_ref in read_golden("abc_closed_form.txt"):
+        co = O.routing_coefficients([2, 2 + int(n)], 4 + int(n))
+        assert abs(co.A[1] - float(A_ref)) < 1e-12 and abs(co.B[1] - float(A_ref)) < 1e-12
+        assert abs(co.C[1] - float(C_ref)) < 1e-12
+    r = _rng(20)
+    h = w = 8
+    b = O.tile_bins(h, w)
+    Ra, Rb = r.standard_normal((2, 3, h, w))
+    tt = O.tile_transport(O.rfft2_ortho(Ra), O.rfft2_ortho(Rb), None, O.ParParams(), b)
+    anchors, F = [3, 5, 6], 10          # left set {0,1,2} with pair (3,5); right set {7,8,9} with (5,6)
+    co = O.routing_coefficients(anchors, F)
+    for (a, bb, Aq, Bq, Cq, frames) in ((3, 5, co.AL, co.BL, co.CL, range(0, 3)),
+                                        (5, 6, co.AR, co.BR, co.CR, range(7, 10))):
+        va = r.standard_normal((3, h, w))
+        vb = r.standard_normal((3, h, w))
+        Fa, Fb = O.rfft2_ortho(va), O.rfft2_ortho(vb)
+        lhs = sum(np.sum(O.irfft2_ortho(O.blend(Fa, Fb, tt.theta, tt.g, (t - a) / (bb - a)), w) ** 2)
+                  for t in frames)
+        na, nb = np.linalg.norm(va), np.linalg.norm(vb)
+        assert lhs <= Aq * na ** 2 + Bq * nb ** 2 + 2 * Cq * na * nb + 1e-9
+        z = np.zeros_like(tt.g)
+        eq = sum(np.sum(O.irfft2_ortho(O.blend(Fa, -Fa, tt.theta, z, (t - a) / (bb - a)), w) ** 2)
+                 for t in frames)
+        assert abs(eq - (Aq + Bq + 2 * Cq) * na ** 2) < 1e-9 * max(1.0, eq)
+
+
+def check_retain_gain_linearity():
+    """Holding the other masks fixed, J = constant - sum_m x_{i,m} G_{i,m} (App. B.3): flipping
+    x_{i,m} changes Eq. (objective) by exactly -G_{i,m}, for interior and boundary anchors,
+    including K_f = 2 where both boundary sets share the pair."""
+    r = _rng(21)
+    for anchors, F, M in (([1, 3, 4, 8], 11, 5), ([2, 5], 9, 4), ([0, 2, 4, 6], 8, 3)):
+        J = len(anchors)
+        u = r.exponential(size=(J, M))
+        x = (r.uniform(size=(J, M)) < 0.5).astype(float)
+        co = O.routing_coefficients(anchors, F)
+        lam = (0.7, 1.3)
+        for i in range(J):
+            G = O.retain_gains(i, u, x, co, *lam)
+            for m in range(M):
+                x1, x0 = x.copy(), x.copy()
+                x1[i, m], x0[i, m] = 1.0, 0.0
+                d = O.routing_objective(u, x1, co, *lam) - O.routing_objective(u, x0, co, *lam)
+                assert abs(d + G[m]) < 1e-9 * max(1.0, abs(G[m])), (anchors, i, m)
+
+
+def check_coupled_routing():
+    """Alg. (routing): every anchor keeps exactly K blocks, J never increases, the result is no
+    worse than independent TopK, lambda_rec = 0 gives independent TopK, and once passes stop
+    changing, no single anchor can lower J with any K-subset (brute force)."""
+    r = _rng(22)
+    for trial in range(12):
+        anchors = sorted(r.choice(9, size=int(r.integers(2, 5)), replace=False).tolist())
+        M, K = 6, 2
+        u = r.exponential(size=(len(anchors), M)) * r.uniform(0.2, 3.0, size=(1, M))
+        idx, info = O.coupled_routing(u, anchors, 9, K, passes=2, with_info=True)
+        assert idx.shape == (len(anchors), K)
+        assert all(len(set(row)) == K for row in idx)
+        tr = info["trace"]
+        assert all(b <= a + 1e-12 for a, b in zip(tr, tr[1:]))
+        co = O.routing_coefficients(anchors, 9)
+        xi = np.zeros_like(u)
+        ind = O.topk_blocks(u, K)
+        for i in range(len(anchors)):
+            xi[i, ind[i]] = 1
+        assert O.routing_objective(u, info["x"], co) <= O.routing_objective(u, xi, co) + 1e-12
+        assert np.array_equal(O.coupled_routing(u, anchors, 9, K, lam_rec=0.0), ind)
+        idx50, info50 = O.coupled_routing(u, anchors, 9, K, passes=60, with_info=True)
+        x = info50["x"]
+        J0 = O.routing_objective(u, x, co)
+        for i in range(len(anchors)):
+            for sub in itertools.combinations(range(M), K):
+                y = x.copy()
+                y[i] = 0
+                y[i, list(sub)] = 1
+                assert O.routing_objective(u, y, co) >= J0 - 1e-6 * max(J0, 1e-8) - 1e-12
+    u = r.exponential(size=(3, 4))
+    assert np.array_equal(O.coupled_routing(u, [0, 2, 4], 5, 7), np.tile(np.arange(4), (3, 1)))
+
+
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

@@ -84,7 +84,33 @@ def _attn_no_scale(q, kc, vc, kh, vh, anchors, idx, scale=None, **kw):
     return _orig_attn(q, kc, vc, kh, vh, anchors, idx, scale=1.0, **kw)
 
 
+_orig_gains = O.retain_gains
+_orig_coeffs = O.routing_coefficients
+
+
+def _gains_no_neighbour_mask(i, u, x, co, lam_anc=1.0, lam_rec=1.0):
+    return _orig_gains(i, u, np.zeros_like(x), co, lam_anc, lam_rec)   # drops the (1 - x) factor
+
+
+def _gains_swapped_ab(i, u, x, co, lam_anc=1.0, lam_rec=1.0):
+    sw = O.RoutingCoefficients(co.B, co.A, co.C, co.BL, co.AL, co.CL, co.BR, co.AR, co.CR)
+    return _orig_gains(i, u, x, sw, lam_anc, lam_rec)
+
+
+def _coeffs_signed_boundary_cross(anchors, n_frames):
+    co = _orig_coeffs(anchors, n_frames)
+    an = [int(a) for a in anchors]
+    if len(an) >= 2:
+        a, b = an[0], an[1]
+        al = np.array([(t - a) / (b - a) for t in range(0, a)])
+        co.CL = float(np.sum(al * (1 - al)))      # forgets |.| outside [0, 1]
+    return co
+
+
 MUTATIONS = {
+    "gain_neighbour_mask_dropped": ("retain_gains", _gains_no_neighbour_mask),
+    "gain_interval_coefficients_swapped": ("retain_gains", _gains_swapped_ab),
+    "boundary_cross_without_abs": ("routing_coefficients", _coeffs_signed_boundary_cross),
     "blend_phase_sign": ("blend", _blend_sign),
     "blend_weights_swapped": ("blend", _blend_swapped),
     "blend_gate_dropped": ("blend", _blend_no_gate),
