@@ -4,7 +4,9 @@
 
 Workload: the Matrix-Game-3.0-shaped bf16 block step (8 current latent frames of 30x52 tokens,
 12 heads x 128, 16 history blocks of 1560 tokens, K = 4, anchors every second frame).
-A step is cast_block_step: routing -> routed anchor attention -> PAR.
+A step is cast_block_step: routing (pooled scores, TopK, then the reconstruction-coupled
+refinement with the paper's L_s = 2 passes and (lambda_anc, lambda_rec) = (1, 1)) -> routed
+anchor attention -> PAR.
   value   frames/s with inputs resident in HBM (CUDA events around each step, L2 flushed
           between steps outside the timed events)
   e2e     frames/s through the same C call with the inputs copied from pinned host memory
@@ -136,7 +138,8 @@ def run_gpu(args):
     idx = torch.empty((len(anchors), H, keff), dtype=torch.int32, device=dev)
     params = lib.par_params(band_radius=wl.band_radius)
     bargs = lib.block_args(d["q"], d["k_cur"], d["v_cur"], anchors, d["k_hist"], d["v_hist"],
-                           wl.K, wl.grid, r_out, idx_out=idx, params=params)
+                           wl.K, wl.grid, r_out, idx_out=idx, params=params,
+                           refine=lib.REFINE_PAPER)
     ws = torch.empty(max(lib.block_workspace_size(bargs), 256), dtype=torch.uint8, device=dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -181,7 +184,8 @@ def run_gpu(args):
     r_par = torch.empty_like(r_out)
     r_par.copy_(r_out)
     mask = W.anchor_mask(N, anchors)
-    rws = torch.empty(max(lib.route_workspace_size(d["q"], anchors, d["k_hist"], d["v_hist"], wl.K), 256),
+    rws = torch.empty(max(lib.route_workspace_size(d["q"], anchors, d["k_hist"], d["v_hist"], wl.K,
+                                                   refine=lib.REFINE_PAPER), 256),
                       dtype=torch.uint8, device=dev)
     pws = torch.empty(max(lib.par_workspace_size(r_par.view(N, wl.grid[0], wl.grid[1], H * dh), mask,
                                                  params), 256), dtype=torch.uint8, device=dev)
@@ -196,7 +200,8 @@ def run_gpu(args):
         e = st_ev[k - 3] if k >= 3 else None
         if e:
             e[0].record(stream)
-        lib.cast_route_topk(d["q"], anchors, d["k_hist"], d["v_hist"], wl.K, workspace=rws)
+        lib.cast_route_topk(d["q"], anchors, d["k_hist"], d["v_hist"], wl.K, workspace=rws,
+                            refine=lib.REFINE_PAPER)
         if e:
             e[1].record(stream)
         lib.cast_anchor_attention(d["q"], d["k_cur"], d["v_cur"], anchors, d["k_hist"], d["v_hist"],
@@ -245,6 +250,7 @@ def run_gpu(args):
             "config": {"workload": wl.name, "frames_per_step": N, "grid": list(wl.grid),
                        "heads": H, "head_dim": dh, "history_blocks": wl.M, "block_tokens": wl.B_v,
                        "K": wl.K, "anchors": anchors, "global_batch": world,
+                       "routing": "coupled refinement, 2 passes, lambda (1, 1), tol 1e-6",
                        "l2": "flushed (256 MiB write) between timed steps, outside the events",
                        "parallelism": f"replicas x{world} (independent chunks, no collective)"},
             "roofline": {"bound": "tensor", "kernel": "k_attn<128> (routed anchor attention)",
@@ -255,7 +261,7 @@ def run_gpu(args):
             "breakdown": {
                 "route": {"ms": round(t_route, 5), "GB/s": round(route_bytes / t_route / 1e6, 1),
                           "frac_hbm": round(route_bytes / t_route / 1e6 / hbm, 4),
-                          "bytes": route_bytes, "kernels": 3},
+                          "bytes": route_bytes, "kernels": 4},
                 "attention": {"ms": round(t_attn, 5), "TFLOP/s": round(achieved, 2),
                               "frac_bf16": round(achieved / bf16, 4)},
                 "par": {"ms": round(t_par, 5), "GB/s": round(par_bytes / t_par / 1e6, 1),
@@ -264,7 +270,7 @@ def run_gpu(args):
             "e2e": {"value": round(N / (e2e_ms / 1e3) * world, 3), "unit": "frames/s",
                     "ms_per_step": round(e2e_ms, 4), "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h)},
-            "gpu_launches": 5 * args.steps,
+            "gpu_launches": 6 * args.steps,
             "clocks": clk,
         }
         if not args.no_scale_points:
@@ -402,7 +408,8 @@ def _oracle_sample(wl, inp, R, heads, row_stride, tiles):
     t0 = time.perf_counter()
     rt = O.pooled_routing(inp["q"][:, :, hs], anchors, inp["k_hist"][:, :, hs],
                           inp["v_hist"][:, :, hs])
-    idx = O.topk_blocks(rt.u, wl.K)
+    idx = np.stack([O.coupled_routing(rt.u[:, h], anchors, wl.n_cur, wl.K)
+                    for h in range(rt.u.shape[1])], axis=1)
     t1 = time.perf_counter()
     rows = np.arange(0, wl.S, row_stride)
     O.routed_attention(inp["q"][:, :, hs], inp["k_cur"][:, :, hs], inp["v_cur"][:, :, hs],
@@ -414,7 +421,8 @@ def _oracle_sample(wl, inp, R, heads, row_stride, tiles):
     t3 = time.perf_counter()
     hf = wl.H / heads
     est = (t1 - t0) * hf + (t2 - t1) * hf * (wl.S / len(rows)) + (t3 - t2) * (n_tiles / tiles)
-    desc = (f"routing on {heads}/{wl.H} heads (all tokens, all blocks), attention on those heads "
+    desc = (f"routing with 2-pass refinement on {heads}/{wl.H} heads (all tokens, all blocks), "
+            f"attention on those heads "
             f"for {len(rows)}/{wl.S} query rows of every anchor, PAR on {tiles}/{n_tiles} tiles; "
             f"each stage scaled to the full workload by its share of the work")
     return est, desc

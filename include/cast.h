@@ -97,6 +97,13 @@ typedef struct {
   float* kbar;                    /* optional [M, H, d] pooled keys */
   float* vbar;                    /* optional [M, H, d] pooled values */
   int32_t* k_eff;                 /* optional HOST: receives K_eff */
+  /* Reconstruction-coupled refinement (Alg. routing, App. B.3): refine_passes > 0 runs that many
+     directional best-response passes (forward, backward, ...) after the TopK initialisation,
+     minimising Eq. (objective) with weights lambda_anc, lambda_rec under the fixed budget K_eff,
+     accepting a change only when J drops by more than refine_tol * max(J, 1e-8).  The paper:
+     2 passes, (1, 1), 1e-6.  0 passes = independent TopK.  Needs CAST_ROUTE_OMISSION. */
+  int32_t refine_passes;
+  float lambda_anc, lambda_rec, refine_tol;
 } cast_route_args;
 
 /* Pooled mean statistics q_bar, k_bar, v_bar (mean over a frame's S tokens and over a
@@ -227,6 +234,8 @@ typedef struct {
   int32_t K;
   float route_eps;
   int32_t route_mode;
+  int32_t route_refine_passes;    /* as cast_route_args.refine_passes (0 = independent TopK) */
+  float route_lambda_anc, route_lambda_rec, route_refine_tol;
   float scale;                    /* <= 0: 1/sqrt(d) */
   void* r_out;                    /* device [n_frames, S, H*d]: anchor rows = attention
                                      output, skipped rows = PAR reconstruction */

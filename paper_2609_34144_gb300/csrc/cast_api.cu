@@ -120,6 +120,16 @@ cast_status validate_route(const cast_route_args* a) {
   if (a->mode != CAST_ROUTE_OMISSION && a->mode != CAST_ROUTE_SIMILARITY)
     return fail(CAST_ERR_INVALID_ARG, "%s: mode %d", who, a->mode);
   if (!(a->eps >= 0.f)) return fail(CAST_ERR_INVALID_ARG, "%s: eps must be >= 0", who);
+  if (a->refine_passes < 0) return fail(CAST_ERR_INVALID_ARG, "%s: refine_passes < 0", who);
+  if (a->refine_passes > 0) {
+    if (a->mode != CAST_ROUTE_OMISSION)
+      return fail(CAST_ERR_INVALID_ARG, "%s: refinement needs CAST_ROUTE_OMISSION", who);
+    if (!(a->lambda_anc >= 0.f) || !(a->lambda_rec >= 0.f) || !(a->refine_tol >= 0.f))
+      return fail(CAST_ERR_INVALID_ARG, "%s: refinement weights and tolerance must be >= 0", who);
+    if (refine_smem_bytes(*a) > 200 * 1024)
+      return fail(CAST_ERR_UNSUPPORTED, "%s: refinement of %d anchors x %d blocks exceeds shared memory",
+                  who, a->n_anchors, a->M);
+  }
   return CAST_OK;
 }
 
@@ -217,6 +227,10 @@ cast_route_args route_of_block(const cast_block_args* a, int32_t* idx) {
   r.K = a->K;
   r.eps = a->route_eps;
   r.mode = a->route_mode;
+  r.refine_passes = a->route_refine_passes;
+  r.lambda_anc = a->route_lambda_anc;
+  r.lambda_rec = a->route_lambda_rec;
+  r.refine_tol = a->route_refine_tol;
   r.idx = idx;
   return r;
 }

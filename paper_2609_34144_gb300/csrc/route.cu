@@ -8,6 +8,8 @@
 //   K_score    : one CTA per (anchor, head): s, pi, o_bar, delta, u (Eq. omission, with an
 //                optional Gram matrix G = P^T P of the output projection) and a warp-level
 //                TopK with ties to the lower block index, written in ascending order.
+//   K_refine   : optional, one CTA per head: the reconstruction-coupled fixed-budget best
+//                responses of Alg. (routing) (App. B.3) starting from the TopK masks.
 #include <cuda_bf16.h>
 
 #include <cfloat>
@@ -292,7 +294,169 @@ __global__ void __launch_bounds__(kScoreThreads)
   }
 }
 
+// ---------------------------------------------------------------------- refinement
+struct RefineArgs {
+  int n_anchors, M, K_eff, H, passes;
+  float lam_anc, lam_rec, tol;
+  float A[CAST_MAX_ANCHORS], B[CAST_MAX_ANCHORS], C[CAST_MAX_ANCHORS];   // interval (j-1, j)
+  float AL, BL, CL, AR, BR, CR;                                          // boundary sets
+};
+
+constexpr int kRefineThreads = 256;
+
+// Warp 0: mask[m] = 1 for the K largest key[m] (ties to the lower index), 0 elsewhere.
+__device__ void warp_topk_mask(const float* key, float* mask, int M, int K, int lane) {
+  for (int m = lane; m < M; m += 32) mask[m] = 0.f;
+  __syncwarp();
+  for (int k = 0; k < K; ++k) {
+    float best = -INFINITY;
+    int bi = 0x7fffffff;
+    for (int m = lane; m < M; m += 32) {
+      if (mask[m] != 0.f) continue;
+      const float v = key[m];
+      if (bi == 0x7fffffff || v > best) { best = v; bi = m; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (oi != 0x7fffffff && (bi == 0x7fffffff || ov > best || (ov == best && oi < bi))) {
+        best = ov;
+        bi = oi;
+      }
+    }
+    if (lane == 0 && bi != 0x7fffffff) mask[bi] = 1.f;
+    __syncwarp();
+  }
+}
+
+// Eq. (risk) term of one block for the anchor pair (p, q) with coefficients (A, B, C)
+__device__ __forceinline__ float pair_risk(float A, float B, float C, float xp, float xq, float up,
+                                           float uq) {
+  return A * (1.f - xp) * up + B * (1.f - xq) * uq + 2.f * C * (1.f - xp) * (1.f - xq) * sqrtf(up * uq);
+}
+
+__device__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = 0.f;
+  if (threadIdx.x < 32) {
+    t = threadIdx.x < kRefineThreads / 32 ? red[threadIdx.x] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (threadIdx.x == 0) red[31] = t;
+  }
+  __syncthreads();
+  return red[31];
+}
+
+// Eq. (objective) of the current masks (block-wide)
+__device__ float objective(const RefineArgs& r, const float* u, const float* x, float* red) {
+  const int na = r.n_anchors, M = r.M;
+  float v = 0.f;
+  for (int m = threadIdx.x; m < M; m += kRefineThreads) {
+    for (int i = 0; i < na; ++i) v += r.lam_anc * (1.f - x[i * M + m]) * u[i * M + m];
+    float rec = 0.f;
+    for (int j = 1; j < na; ++j)
+      rec += pair_risk(r.A[j], r.B[j], r.C[j], x[(j - 1) * M + m], x[j * M + m], u[(j - 1) * M + m],
+                       u[j * M + m]);
+    if (na >= 2) {
+      rec += pair_risk(r.AL, r.BL, r.CL, x[m], x[M + m], u[m], u[M + m]);
+      rec += pair_risk(r.AR, r.BR, r.CR, x[(na - 2) * M + m], x[(na - 1) * M + m], u[(na - 2) * M + m],
+                       u[(na - 1) * M + m]);
+    }
+    v += r.lam_rec * rec;
+  }
+  return block_sum(v, red);
+}
+
+// grid (H).  Dynamic smem: u [na][M], x [na][M], G [M], xn [M] (floats).
+__global__ void __launch_bounds__(kRefineThreads)
+    k_refine(const float* __restrict__ u_all, const __grid_constant__ RefineArgs r,
+             int32_t* __restrict__ idx) {
+  extern __shared__ float sm[];
+  __shared__ float red[32];
+  __shared__ int s_accept;
+  const int h = blockIdx.x, na = r.n_anchors, M = r.M, K = r.K_eff;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  float* u = sm;
+  float* x = u + na * M;
+  float* G = x + na * M;
+  float* xn = G + M;
+  for (int e = tid; e < na * M; e += kRefineThreads) {
+    const int i = e / M, m = e - i * M;
+    u[e] = u_all[((int64_t)i * r.H + h) * M + m];
+  }
+  __syncthreads();
+  // initial masks: TopK of u per anchor (one warp per anchor)
+  for (int i = warp; i < na; i += kRefineThreads / 32) warp_topk_mask(u + i * M, x + i * M, M, K, lane);
+  __syncthreads();
+  float J = objective(r, u, x, red);
+  for (int pass = 1; pass <= r.passes; ++pass) {
+    bool changed = false;
+    for (int step = 0; step < na; ++step) {
+      const int i = (pass & 1) ? step : na - 1 - step;
+      // retain gains, Eqs. (gain) and (boundarygain)
+      for (int m = tid; m < M; m += kRefineThreads) {
+        const float ui = u[i * M + m];
+        float g = r.lam_anc * ui, rec = 0.f;
+        if (i >= 1) {
+          const float ul = u[(i - 1) * M + m];
+          rec += r.B[i] * ui + 2.f * r.C[i] * (1.f - x[(i - 1) * M + m]) * sqrtf(ul * ui);
+        }
+        if (i + 1 < na) {
+          const float ur = u[(i + 1) * M + m];
+          rec += r.A[i + 1] * ui + 2.f * r.C[i + 1] * (1.f - x[(i + 1) * M + m]) * sqrtf(ui * ur);
+        }
+        if (na >= 2) {
+          if (i == 0) rec += r.AL * ui + 2.f * r.CL * (1.f - x[M + m]) * sqrtf(ui * u[M + m]);
+          if (i == 1) rec += r.BL * ui + 2.f * r.CL * (1.f - x[m]) * sqrtf(ui * u[m]);
+          if (i == na - 2) rec += r.AR * ui + 2.f * r.CR * (1.f - x[(na - 1) * M + m]) * sqrtf(ui * u[(na - 1) * M + m]);
+          if (i == na - 1) rec += r.BR * ui + 2.f * r.CR * (1.f - x[(na - 2) * M + m]) * sqrtf(ui * u[(na - 2) * M + m]);
+        }
+        G[m] = g + r.lam_rec * rec;
+      }
+      __syncthreads();
+      if (warp == 0) warp_topk_mask(G, xn, M, K, lane);
+      __syncthreads();
+      float d = 0.f;
+      for (int m = tid; m < M; m += kRefineThreads) d += G[m] * (xn[m] - x[i * M + m]);
+      const float gain = block_sum(d, red);
+      if (tid == 0) s_accept = gain > r.tol * fmaxf(J, 1e-8f);
+      __syncthreads();
+      if (s_accept) {
+        for (int m = tid; m < M; m += kRefineThreads) x[i * M + m] = xn[m];
+        __syncthreads();
+        J = objective(r, u, x, red);
+        changed = true;
+      }
+    }
+    if (!changed) break;
+  }
+  __syncthreads();
+  // ascending block indices of every anchor's mask
+  for (int i = warp; i < na; i += kRefineThreads / 32) {
+    int base = 0;
+    int32_t* out = idx + ((int64_t)i * r.H + h) * K;
+    for (int m0 = 0; m0 < M; m0 += 32) {
+      const int m = m0 + lane;
+      const bool on = m < M && x[i * M + m] != 0.f;
+      const unsigned bal = __ballot_sync(0xffffffffu, on);
+      if (on) out[base + __popc(bal & ((1u << lane) - 1u))] = m;
+      base += __popc(bal);
+    }
+  }
+}
+
 }  // namespace
+
+size_t refine_smem_bytes(const cast_route_args& a) {
+  return (size_t)(2 * a.n_anchors + 2) * (size_t)a.M * sizeof(float);
+}
 
 RoutePlan route_plan(const cast_route_args& a) {
   RoutePlan p{};
@@ -309,7 +473,8 @@ RoutePlan route_plan(const cast_route_args& a) {
   p.nsplit = nsplit;
   p.partial_bytes = align_up((size_t)p.n_seg * nsplit * D * sizeof(float));
   p.pooled_bytes = align_up((size_t)p.n_seg * D * sizeof(float));
-  p.total_bytes = p.partial_bytes + p.pooled_bytes;
+  p.u_bytes = (a.refine_passes > 0 && !a.u) ? align_up((size_t)a.n_anchors * a.H * a.M * sizeof(float)) : 0;
+  p.total_bytes = p.partial_bytes + p.pooled_bytes + p.u_bytes;
   return p;
 }
 
@@ -357,9 +522,59 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
                              (int)smem) != cudaSuccess)
       return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory", smem);
   }
+  const bool refine = a.refine_passes > 0 && K_eff > 0 && K_eff < a.M;
+  float* u_buf = a.u ? a.u : (p.u_bytes ? reinterpret_cast<float*>(w + p.partial_bytes + p.pooled_bytes) : nullptr);
   k_score_topk<<<dim3(a.H, a.n_anchors), kScoreThreads, smem, st>>>(
-      qbar, kbar, vbar, a.gram, a.H, a.d, a.M, K_eff, a.eps, a.mode, a.idx, a.u);
-  return check_launch("routing score/TopK kernel");
+      qbar, kbar, vbar, a.gram, a.H, a.d, a.M, K_eff, a.eps, a.mode, a.idx, u_buf);
+  s = check_launch("routing score/TopK kernel");
+  if (s != CAST_OK || !refine) return s;
+  // Alg. (routing): interval and boundary coefficients of the anchor layout (Eqs. abc,
+  // boundarycoeff), then the directional best-response passes on the GPU
+  RefineArgs r{};
+  r.n_anchors = a.n_anchors;
+  r.M = a.M;
+  r.K_eff = K_eff;
+  r.H = a.H;
+  r.passes = a.refine_passes;
+  r.lam_anc = a.lambda_anc;
+  r.lam_rec = a.lambda_rec;
+  r.tol = a.refine_tol;
+  for (int j = 1; j < a.n_anchors; ++j) {
+    const int x0 = a.anchors[j - 1], x1 = a.anchors[j];
+    double A = 0, B = 0, C = 0;
+    for (int t = x0 + 1; t < x1; ++t) {
+      const double al = (double)(t - x0) / (double)(x1 - x0);
+      A += (1 - al) * (1 - al);
+      B += al * al;
+      C += al * (1 - al);
+    }
+    r.A[j] = (float)A;
+    r.B[j] = (float)B;
+    r.C[j] = (float)C;
+  }
+  if (a.n_anchors >= 2) {
+    auto bset = [&](int x0, int x1, int t0, int t1, float& A, float& B, float& C) {
+      double sa = 0, sb = 0, sc = 0;
+      for (int t = t0; t < t1; ++t) {
+        const double al = (double)(t - x0) / (double)(x1 - x0);
+        sa += (1 - al) * (1 - al);
+        sb += al * al;
+        sc += std::fabs(al * (1 - al));
+      }
+      A = (float)sa;
+      B = (float)sb;
+      C = (float)sc;
+    };
+    bset(a.anchors[0], a.anchors[1], 0, a.anchors[0], r.AL, r.BL, r.CL);
+    bset(a.anchors[a.n_anchors - 2], a.anchors[a.n_anchors - 1], a.anchors[a.n_anchors - 1] + 1,
+         a.n_frames, r.AR, r.BR, r.CR);
+  }
+  const size_t rsm = refine_smem_bytes(a);
+  if (rsm > 48 * 1024 &&
+      cudaFuncSetAttribute(k_refine, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsm) != cudaSuccess)
+    return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory for refinement", rsm);
+  k_refine<<<a.H, kRefineThreads, rsm, st>>>(u_buf, r, a.idx);
+  return check_launch("routing refinement kernel");
 }
 
 }  // namespace cast

@@ -35,7 +35,8 @@ class RouteArgs(C.Structure):
                 ("k_hist", _vp), ("v_hist", _vp), ("hist_row_stride", _i64), ("M", _i32),
                 ("B_v", _i32), ("gram", _vp), ("K", _i32), ("eps", _f32), ("mode", _i32),
                 ("idx", _vp), ("u", _vp), ("qbar", _vp), ("kbar", _vp), ("vbar", _vp),
-                ("k_eff", C.POINTER(_i32))]
+                ("k_eff", C.POINTER(_i32)), ("refine_passes", _i32), ("lambda_anc", _f32),
+                ("lambda_rec", _f32), ("refine_tol", _f32)]
 
 
 class AttnArgs(C.Structure):
@@ -65,7 +66,9 @@ class BlockArgs(C.Structure):
                 ("H", _i32), ("d", _i32), ("anchors", C.POINTER(_i32)), ("n_anchors", _i32),
                 ("k_hist", _vp), ("v_hist", _vp), ("hist_row_stride", _i64), ("M", _i32),
                 ("B_v", _i32), ("gram", _vp), ("K", _i32), ("route_eps", _f32),
-                ("route_mode", _i32), ("scale", _f32), ("r_out", _vp), ("r_dtype", _i32),
+                ("route_mode", _i32), ("route_refine_passes", _i32), ("route_lambda_anc", _f32),
+                ("route_lambda_rec", _f32), ("route_refine_tol", _f32), ("scale", _f32),
+                ("r_out", _vp), ("r_dtype", _i32),
                 ("x", _vp), ("idx_out", _vp), ("channel_weight", _vp), ("par", ParParams)]
 
 
@@ -164,7 +167,11 @@ def default_par_params():
 
 
 # --------------------------------------------------------------------------- routing
-def _route_args(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_OMISSION):
+REFINE_PAPER = dict(passes=2, lambda_anc=1.0, lambda_rec=1.0, tol=1e-6)   # Tab. config_cast
+
+
+def _route_args(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_OMISSION,
+                refine=None):
     N, S, H, d = q.shape
     M = k_hist.shape[0]
     a = RouteArgs()
@@ -179,18 +186,22 @@ def _route_args(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_O
     a.M, a.B_v = M, k_hist.shape[1]
     a.gram = _ptr(gram)
     a.K, a.eps, a.mode = K, eps, mode
+    if refine:
+        a.refine_passes, a.lambda_anc = refine["passes"], refine["lambda_anc"]
+        a.lambda_rec, a.refine_tol = refine["lambda_rec"], refine["tol"]
     return a
 
 
-def route_workspace_size(q, anchors, k_hist, v_hist, K):
-    a = _route_args(q, anchors, k_hist, v_hist, K)
+def route_workspace_size(q, anchors, k_hist, v_hist, K, refine=None):
+    a = _route_args(q, anchors, k_hist, v_hist, K, refine=refine)
     return _lib.cast_route_topk and _lib.cast_route_workspace_size(C.byref(a))
 
 
 def cast_route_topk(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_OMISSION,
-                    want_u=False, want_pooled=False, workspace=None, stream=None):
-    """Returns idx [K_f, H, K_eff] int32 (and u, (qbar, kbar, vbar) when asked)."""
-    a = _route_args(q, anchors, k_hist, v_hist, K, gram, eps, mode)
+                    want_u=False, want_pooled=False, workspace=None, stream=None, refine=None):
+    """Returns idx [K_f, H, K_eff] int32 (and u, (qbar, kbar, vbar) when asked).  refine: None
+    (independent TopK) or a dict like REFINE_PAPER (coupled refinement, Alg. routing)."""
+    a = _route_args(q, anchors, k_hist, v_hist, K, gram, eps, mode, refine)
     Kf, H, d, M = len(anchors), q.shape[2], q.shape[3], k_hist.shape[0]
     keff = min(K, M)
     dev = q.device
@@ -304,7 +315,7 @@ def cast_par_reconstruct(r, anchor_mask, channel_weight=None, params=None, works
 # --------------------------------------------------------------------------- block step
 def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None, idx_out=None,
                gram=None, route_eps=1e-8, route_mode=ROUTE_OMISSION, scale=0.0,
-               channel_weight=None, params=None):
+               channel_weight=None, params=None, refine=None):
     N, S, H, d = q.shape
     M = k_hist.shape[0]
     a = BlockArgs()
@@ -318,6 +329,9 @@ def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None,
     a.hist_row_stride = _row_stride(k_hist) if M > 0 else H * d
     a.M, a.B_v = M, k_hist.shape[1]
     a.gram, a.K, a.route_eps, a.route_mode, a.scale = _ptr(gram), K, route_eps, route_mode, scale
+    if refine:
+        a.route_refine_passes, a.route_lambda_anc = refine["passes"], refine["lambda_anc"]
+        a.route_lambda_rec, a.route_refine_tol = refine["lambda_rec"], refine["tol"]
     a.r_out, a.r_dtype = _ptr(r_out), _dtype_code(r_out)
     a.x = _ptr(x)
     a.idx_out = _ptr(idx_out)

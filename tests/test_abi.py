@@ -81,6 +81,10 @@ def _route(lib, **kw):
     ({"q": _fake(0x10008)}, 1),
     ({"K": -1}, 1),
     ({"mode": 7}, 1),
+    ({"refine_passes": -1}, 1),
+    ({"refine_passes": 2, "mode": 1}, 1),            # refinement needs the omission score
+    ({"refine_passes": 2, "lambda_rec": -1.0}, 1),
+    ({"refine_passes": 2, "M": 10000}, 2),           # u and masks exceed shared memory
 ])
 def test_route_validation(lib, bad, status):
     a = _route(lib, **bad)
