@@ -5,7 +5,8 @@
 //   O = softmax(scale Q K^T) V over every token of the current chunk followed by the tokens
 //   of the routed history blocks idx[i, h, :].
 // Both query tiles consume every K/V tile, so each tile fetched from L2 feeds 256 rows.
-// Warp roles (320 threads, one CTA per SM, 193 KB shared memory, all 512 TMEM columns):
+// Warp roles (384 threads = three warpgroups, one CTA per SM, 193 KB shared memory, all 512
+// TMEM columns; warpgroup 0 gives registers to the two softmax warpgroups with setmaxnreg):
 //   warp 0       TMA producers: lane 0 loads Q0/Q1 and the K tiles, lane 1 the V tiles, each
 //                into a two-stage ring (128 tokens x d, 128-byte swizzle, 64-element boxes);
 //                current-chunk tiles come from a 2-D map, history tiles from a 3-D map
@@ -14,7 +15,8 @@
 //                S0_0 S1_0 | PV0_0 S0_1 PV1_0 S1_1 | PV0_1 S0_2 PV1_1 S1_2 | ...
 //                (S_t = Q_t K^T, kind::f16, M=N=128, f32 in TMEM; PV_t: O_t += P_t V with P_t
 //                read from TMEM over the S_t columns and V read MN-major).
-//   warps 2..5   softmax of Q0, warps 6..9 softmax of Q1: one query row per thread,
+//   warps 2, 3   idle (they complete warpgroup 0 for the register hand-over)
+//   warps 4..7   softmax of Q0, warps 8..11 softmax of Q1: one query row per thread,
 //                tcgen05.ld of the S row, masking, exp2-domain online softmax with lazy
 //                rescaling (O_t and l rescaled only when the running max grows by more than
 //                8 = log2 256), P packed to bf16 and stored with tcgen05.st, epilogue O / l.
@@ -40,7 +42,13 @@ namespace {
 __device__ unsigned int g_attn_error;
 
 constexpr int BM = 128, BN = 128, kStages = 2;
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;
+// Registers: every thread starts with kLaunchRegs; warpgroup 0 (producer, MMA issuer, two
+// idle warps) drops to kRegsCtl and the softmax warpgroups rise to kRegsSoftmax.
+constexpr int kLaunchRegs = 168, kRegsCtl = 96, kRegsSoftmax = 200;
+static_assert(128 * kRegsCtl + 256 * kRegsSoftmax <= kThreads * kLaunchRegs,
+              "register split exceeds the launch allocation");
+static_assert(kThreads * kLaunchRegs <= 65536, "launch allocation exceeds the register file");
 constexpr int kTmemCols = 512;   // S0/P0 at 0, S1/P1 at 128, O0 at 256, O1 at 384
 constexpr float kRescaleThreshold = 8.f;
 
@@ -94,6 +102,11 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   float d;
   asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
   return d;
+}
+
+// Whole-CTA barrier reached from the code of different roles (non-aligned form, barrier 1).
+__device__ __forceinline__ void end_barrier() {
+  asm volatile("barrier.sync 1, %0;" ::"n"(kThreads) : "memory");
 }
 
 __device__ __forceinline__ bool aborted(const Bars* b) {
@@ -204,6 +217,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bars->tmem_base;
   const uint64_t lim = a.wait_ns;
 
+  if (warp < 4) {
+  setmaxnreg_dec<kRegsCtl>();
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producers
     if (lane == 0) {
@@ -316,9 +331,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       umma_commit(&bars->fin);
       mbar_wait(&bars->fin, 0, lim);
     }
-  } else if (warp < 6 || has_q1) {
+  }
+  // the last UMMA has completed (fin) and every softmax thread has read TMEM
+  tc_fence_before();
+  end_barrier();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+  } else {
+  setmaxnreg_inc<kRegsSoftmax>();
+  if (warp < 8 || has_q1) {
     // ------------------------------------------------------------ softmax + epilogue
-    const int t = warp < 6 ? 0 : 1;
+    const int t = warp < 8 ? 0 : 1;
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
@@ -460,7 +485,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // every softmax thread arrives (also after a failure, so nobody waits forever); one
       // thread then counts this part in, and the part that completes the count merges
       mbar_arrive(&bars->part_done);
-      if (warp == 2 && lane == 0) {
+      if (warp == 4 && lane == 0) {
         const bool w = mbar_wait(&bars->part_done, 0, lim);
         int last = 0;
         if (w && !aborted(bars)) {
@@ -509,10 +534,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+  end_barrier();
   }
 }
 
@@ -584,6 +606,13 @@ cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_o
   }
   static bool attr_set = false;
   if (!attr_set) {
+    // the register hand-over in the kernel assumes exactly kLaunchRegs per thread at launch
+    cudaFuncAttributes fa{};
+    if (cudaFuncGetAttributes(&fa, k_attn<HD>) != cudaSuccess)
+      return check_launch("attention kernel attributes");
+    if (fa.numRegs != kLaunchRegs)
+      return fail(CAST_ERR_UNSUPPORTED, "attention kernel built with %d registers per thread, expected %d",
+                  fa.numRegs, kLaunchRegs);
     if (cudaFuncSetAttribute(k_attn<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
         cudaSuccess)
       return check_launch("attention smem attribute");
