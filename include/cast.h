@@ -93,9 +93,9 @@ typedef struct {
   /* outputs (device unless noted) */
   int32_t* idx;                   /* [n_anchors, H, K_eff] ascending block indices */
   float* u;                       /* optional [n_anchors, H, M] routing scores used for TopK */
-  float* qbar;                    /* optional [n_anchors, H, d] pooled queries */
-  float* kbar;                    /* optional [M, H, d] pooled keys */
-  float* vbar;                    /* optional [M, H, d] pooled values */
+  float* qbar;                    /* optional [n_anchors, H, d] pooled queries (16-B aligned) */
+  float* kbar;                    /* optional [M, H, d] pooled keys (16-B aligned) */
+  float* vbar;                    /* optional [M, H, d] pooled values (16-B aligned) */
   int32_t* k_eff;                 /* optional HOST: receives K_eff */
   /* Reconstruction-coupled refinement (Alg. routing, App. B.3): refine_passes > 0 runs that many
      directional best-response passes (forward, backward, ...) after the TopK initialisation,
@@ -114,7 +114,10 @@ typedef struct {
  * M == 0 writes nothing (routing bypass, App. B.3).
  * Errors: INVALID_ARG for NULL required pointers, n_anchors < 1 or > CAST_MAX_ANCHORS,
  * anchors not ascending / out of range, K < 0, M < 0, B_v < 1 with M > 0, bad strides,
- * a workspace smaller than cast_route_workspace_size(); UNSUPPORTED for d not 64/128. */
+ * a workspace smaller than cast_route_workspace_size(), refinement with a negative weight or
+ * tolerance or outside CAST_ROUTE_OMISSION; UNSUPPORTED for d not 64/128, M > 16384,
+ * H*d > 51200 channels (pooling shared memory) or 4*(2*K_f*d + 3*K_f*M + M + 8*d) bytes of
+ * per-head state above 200 KB. */
 cast_status cast_route_topk(const cast_route_args* args, void* workspace,
                             size_t workspace_bytes, void* stream);
 size_t cast_route_workspace_size(const cast_route_args* args);

@@ -107,7 +107,7 @@ cast_status validate_route(const cast_route_args* a) {
     return fail(CAST_ERR_INVALID_ARG, "%s: n_frames, S, H must be positive", who);
   if (a->M < 0 || a->K < 0) return fail(CAST_ERR_INVALID_ARG, "%s: M and K must be >= 0", who);
   if (a->M > 0 && a->B_v < 1) return fail(CAST_ERR_INVALID_ARG, "%s: B_v must be >= 1", who);
-  if (a->M > 65536) return fail(CAST_ERR_UNSUPPORTED, "%s: M=%d above 65536", who, a->M);
+  if (a->M > 16384) return fail(CAST_ERR_UNSUPPORTED, "%s: M=%d above 16384", who, a->M);
   cast_status s = validate_anchors(a->anchors, a->n_anchors, a->n_frames, who);
   if (s) return s;
   s = validate_tokens(a->q, a->q_row_stride, a->H, a->d, "q", who);
@@ -119,6 +119,9 @@ cast_status validate_route(const cast_route_args* a) {
   }
   if (a->mode != CAST_ROUTE_OMISSION && a->mode != CAST_ROUTE_SIMILARITY)
     return fail(CAST_ERR_INVALID_ARG, "%s: mode %d", who, a->mode);
+  for (const float* p : {a->qbar, a->kbar, a->vbar})
+    if (reinterpret_cast<uintptr_t>(p) % 16)
+      return fail(CAST_ERR_INVALID_ARG, "%s: qbar/kbar/vbar must be 16-byte aligned", who);
   if (!(a->eps >= 0.f)) return fail(CAST_ERR_INVALID_ARG, "%s: eps must be >= 0", who);
   if (a->refine_passes < 0) return fail(CAST_ERR_INVALID_ARG, "%s: refine_passes < 0", who);
   if (a->refine_passes > 0) {
@@ -126,10 +129,13 @@ cast_status validate_route(const cast_route_args* a) {
       return fail(CAST_ERR_INVALID_ARG, "%s: refinement needs CAST_ROUTE_OMISSION", who);
     if (!(a->lambda_anc >= 0.f) || !(a->lambda_rec >= 0.f) || !(a->refine_tol >= 0.f))
       return fail(CAST_ERR_INVALID_ARG, "%s: refinement weights and tolerance must be >= 0", who);
-    if (refine_smem_bytes(*a) > 200 * 1024)
-      return fail(CAST_ERR_UNSUPPORTED, "%s: refinement of %d anchors x %d blocks exceeds shared memory",
-                  who, a->n_anchors, a->M);
   }
+  if (route_pool_smem_bytes(*a) > 200 * 1024)
+    return fail(CAST_ERR_UNSUPPORTED, "%s: H*d = %d channels exceed the pooling kernel's shared memory",
+                who, a->H * a->d);
+  if (a->M > 0 && route_head_smem_bytes(*a) > 200 * 1024)
+    return fail(CAST_ERR_UNSUPPORTED, "%s: %d anchors x %d blocks exceed the per-head shared memory",
+                who, a->n_anchors, a->M);
   return CAST_OK;
 }
 

@@ -29,12 +29,14 @@ inline size_t align_up(size_t x, size_t a = kWsAlign) { return (x + a - 1) / a *
 // ------------------------------------------------------------------ routing
 struct RoutePlan {
   int n_seg;        // n_anchors + 2 M pooled segments
-  int nsplit;       // row splits per segment
-  size_t partial_bytes, pooled_bytes, u_bytes, total_bytes;
+  int nsplit;       // row splits per segment (CTAs of one cluster)
+  size_t pooled_bytes, total_bytes;
 };
 RoutePlan route_plan(const cast_route_args& a);
-// shared memory of the refinement kernel (u and masks of every anchor for one head)
-size_t refine_smem_bytes(const cast_route_args& a);
+// shared memory of the pooling kernel (column sums of one CTA) and of the per-head kernel
+// (pooled query, o_bar, pi, keys and masks of every anchor of one head)
+size_t route_pool_smem_bytes(const cast_route_args& a);
+size_t route_head_smem_bytes(const cast_route_args& a);
 // Arguments must have been validated; ws holds at least route_plan(a).total_bytes.
 cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st);
 

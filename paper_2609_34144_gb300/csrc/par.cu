@@ -484,7 +484,6 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (warp == 0) tile_transport(a, g, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
         __syncthreads();
         const float inv_hw = 1.f / (float)(g.h * g.w);
-        const int64_t rowC = (int64_t)a.Wg * a.C;
         for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += kCoefBatch) {
           const int nt = min(kCoefBatch, a.pair_tbeg[j + 1] - t0);
           for (int e = tid; e < nt * kNB; e += kThreads) {

@@ -1,15 +1,19 @@
-// Routing of historical KV blocks (Section 4.4, Eqs. pooled, omission, topk).
+// Routing of historical KV blocks (Section 4.4, Eqs. pooled, omission, topk; App. B.3).
 //
-//   K_pool     : column sums of every pooled segment (anchor query frames, history key
-//                blocks, history value blocks), split over rows; HBM-bound streaming of
-//                (K_f S + 2 M B_v) H d elements with 16-byte loads.
-//   K_finalize : sums the row splits in a fixed order and divides by the row count
-//                (deterministic means q_bar, k_bar, v_bar in f32).
-//   K_score    : one CTA per (anchor, head): s, pi, o_bar, delta, u (Eq. omission, with an
-//                optional Gram matrix G = P^T P of the output projection) and a warp-level
-//                TopK with ties to the lower block index, written in ascending order.
-//   K_refine   : optional, one CTA per head: the reconstruction-coupled fixed-budget best
-//                responses of Alg. (routing) (App. B.3) starting from the TopK masks.
+//   K_pool  : mean of every pooled segment (anchor query frames, history key blocks, history
+//             value blocks): HBM-bound streaming of (K_f S + 2 M B_v) H d elements with 16-byte
+//             loads.  A segment's rows are split over the CTAs of one thread-block cluster;
+//             the CTAs reduce their column sums through distributed shared memory in rank order
+//             (deterministic) and write q_bar, k_bar, v_bar in f32.  No partial sums leave the
+//             chip.
+//   K_head  : one CTA per head, every anchor at once: s, pi, o_bar, delta, u (Eq. omission,
+//             with an optional Gram matrix G = P^T P of the output projection), the TopK mask of
+//             each anchor (ties to the lower block index) and, when asked, the reconstruction-
+//             coupled best-response passes of Alg. (routing); block indices are written in
+//             ascending order.
+// The head kernel is launched as a programmatic dependent of the pooling kernel: its CTAs
+// become resident while the pooling drains and wait on the grid dependency before reading the
+// means.
 #include <cuda_bf16.h>
 
 #include <cfloat>
@@ -20,12 +24,29 @@
 namespace cast {
 namespace {
 
-constexpr int kPoolThreads = 256;
+constexpr int kPoolMaxThreads = 512;
+constexpr int kPoolUnroll = 8;     // 16-byte loads in flight per thread
+constexpr int kMaxClusterSplit = 8;
+
+// Thread layout of the pooling CTA: cgs 16-byte column groups side by side, lanes_r row lanes.
+struct PoolShape {
+  int cgs, lanes_r;
+};
+inline PoolShape pool_shape(int D, int elt) {
+  const int ncg = D / (16 / elt);
+  PoolShape p;
+  p.cgs = ncg >= kPoolMaxThreads ? kPoolMaxThreads : ncg;
+  p.lanes_r = kPoolMaxThreads / p.cgs;
+  return p;
+}
 
 struct PoolArgs {
   const char* q;          // anchor frame base = q + anchors[i] * S * q_row_stride * elt
   const char* k;
   const char* v;
+  float* qbar;            // [n_anchors, D]
+  float* kbar;            // [M, D]
+  float* vbar;            // [M, D]
   int64_t q_row_stride, hist_row_stride;   // elements
   int n_anchors, M, S, B_v, D, nsplit, elt;
   int anchors[CAST_MAX_ANCHORS];
@@ -50,36 +71,63 @@ __device__ __forceinline__ void load_vec<__nv_bfloat16>(const char* p, float (&x
   }
 }
 
-// grid (nsplit, n_seg); partial[(seg * nsplit + split) * D + col]
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ float ld_dsmem(const float* local, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+               : "=r"(remote)
+               : "r"((uint32_t)__cvta_generic_to_shared(local)), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+  return v;
+}
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// grid (nsplit, n_seg), cluster (nsplit, 1, 1), cgs * lanes_r threads.  Dynamic smem:
+// colsum[D] and (lanes_r - 1) rows of per-lane sums.
 template <typename T>
-__global__ void __launch_bounds__(kPoolThreads) k_pool(PoolArgs a, float* __restrict__ partial) {
+__global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant__ PoolArgs a) {
   constexpr int VEC = 16 / sizeof(T);
+  extern __shared__ float colsum[];
+  launch_dependents();
   const int seg = blockIdx.y, split = blockIdx.x;
   const char* base;
   int64_t rs;
   int nrows;
+  float* out;
   if (seg < a.n_anchors) {
     base = a.q + (int64_t)a.anchors[seg] * a.S * a.q_row_stride * a.elt;
     rs = a.q_row_stride;
     nrows = a.S;
+    out = a.qbar + (int64_t)seg * a.D;
   } else if (seg < a.n_anchors + a.M) {
     base = a.k + (int64_t)(seg - a.n_anchors) * a.B_v * a.hist_row_stride * a.elt;
     rs = a.hist_row_stride;
     nrows = a.B_v;
+    out = a.kbar + (int64_t)(seg - a.n_anchors) * a.D;
   } else {
     base = a.v + (int64_t)(seg - a.n_anchors - a.M) * a.B_v * a.hist_row_stride * a.elt;
     rs = a.hist_row_stride;
     nrows = a.B_v;
+    out = a.vbar + (int64_t)(seg - a.n_anchors - a.M) * a.D;
   }
   const int per = (nrows + a.nsplit - 1) / a.nsplit;
   const int r0 = split * per, r1 = min(nrows, r0 + per);
-  const int ncg = a.D / VEC;                          // 16-byte column groups
-  const int lanes_r = ncg >= kPoolThreads ? 1 : kPoolThreads / ncg;   // row lanes
-  const int tcg = threadIdx.x % (ncg >= kPoolThreads ? kPoolThreads : ncg);
-  const int trl = threadIdx.x / (ncg >= kPoolThreads ? kPoolThreads : ncg);
-  __shared__ float red[kPoolThreads * 8];
-  float* out = partial + ((int64_t)seg * a.nsplit + split) * a.D;
-  for (int cg = tcg; cg < ncg; cg += (ncg >= kPoolThreads ? kPoolThreads : ncg)) {
+  const int ncg = a.D / VEC;                                    // 16-byte column groups
+  const int nthreads = blockDim.x;
+  const int cgs = ncg >= kPoolMaxThreads ? kPoolMaxThreads : ncg;   // column groups per pass
+  const int lanes_r = nthreads / cgs;                               // row lanes (>= 1)
+  const int tcg = threadIdx.x % cgs, trl = threadIdx.x / cgs;
+  float* lane_sum = colsum + a.D;                               // [lanes_r - 1][D] when lanes_r > 1
+  for (int cg = tcg; cg < ncg; cg += cgs) {
     float acc[VEC];
 #pragma unroll
     for (int k = 0; k < VEC; ++k) acc[k] = 0.f;
@@ -87,15 +135,21 @@ __global__ void __launch_bounds__(kPoolThreads) k_pool(PoolArgs a, float* __rest
       const char* p = base + ((int64_t)(r0 + trl) * rs + (int64_t)cg * VEC) * a.elt;
       const int64_t step = (int64_t)lanes_r * rs * a.elt;
       int r = r0 + trl;
-      for (; r + 3 * lanes_r < r1; r += 4 * lanes_r) {
-        float x0[VEC], x1[VEC], x2[VEC], x3[VEC];
-        load_vec<T>(p, x0);
-        load_vec<T>(p + step, x1);
-        load_vec<T>(p + 2 * step, x2);
-        load_vec<T>(p + 3 * step, x3);
-        p += 4 * step;
+      for (; r + (kPoolUnroll - 1) * lanes_r < r1; r += kPoolUnroll * lanes_r) {
+        float x[kPoolUnroll][VEC];
 #pragma unroll
-        for (int k = 0; k < VEC; ++k) acc[k] += (x0[k] + x1[k]) + (x2[k] + x3[k]);
+        for (int u = 0; u < kPoolUnroll; ++u) load_vec<T>(p + u * step, x[u]);
+        p += kPoolUnroll * step;
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+          float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+          for (int u = 0; u < kPoolUnroll; u += 2) {
+            s0 += x[u][k];
+            s1 += x[u + 1][k];
+          }
+          acc[k] += s0 + s1;
+        }
       }
       for (; r < r1; r += lanes_r) {
         float x0[VEC];
@@ -105,47 +159,50 @@ __global__ void __launch_bounds__(kPoolThreads) k_pool(PoolArgs a, float* __rest
         for (int k = 0; k < VEC; ++k) acc[k] += x0[k];
       }
     }
-    if (lanes_r == 1) {
+    if (trl == 0) {
 #pragma unroll
-      for (int k = 0; k < VEC; ++k) out[cg * VEC + k] = acc[k];
-    } else {
-      // reduce the row lanes of this column group through shared memory (fixed order)
-      __syncthreads();
-      if (trl < lanes_r) {
+      for (int k = 0; k < VEC; ++k) colsum[cg * VEC + k] = acc[k];
+    } else if (trl < lanes_r) {
 #pragma unroll
-        for (int k = 0; k < VEC; ++k) red[(trl * ncg + cg) * VEC + k] = acc[k];
-      }
-      __syncthreads();
-      if (trl == 0) {
-        for (int l = 1; l < lanes_r; ++l)
-#pragma unroll
-          for (int k = 0; k < VEC; ++k) acc[k] += red[(l * ncg + cg) * VEC + k];
-#pragma unroll
-        for (int k = 0; k < VEC; ++k) out[cg * VEC + k] = acc[k];
-      }
+      for (int k = 0; k < VEC; ++k) lane_sum[(int64_t)(trl - 1) * a.D + cg * VEC + k] = acc[k];
     }
   }
-}
-
-// pooled[seg * D + col] = (sum over splits in order) / rows(seg)
-__global__ void k_finalize(const float* __restrict__ partial, float* __restrict__ qbar,
-                           float* __restrict__ kbar, float* __restrict__ vbar, int n_anchors,
-                           int M, int S, int B_v, int D, int nsplit) {
-  const int seg = blockIdx.y;
-  const int col = blockIdx.x * blockDim.x + threadIdx.x;
-  if (col >= D) return;
-  float s = 0.f;
-  for (int k = 0; k < nsplit; ++k) s += partial[((int64_t)seg * nsplit + k) * D + col];
-  if (seg < n_anchors) {
-    qbar[(int64_t)seg * D + col] = s / (float)S;
-  } else if (seg < n_anchors + M) {
-    kbar[(int64_t)(seg - n_anchors) * D + col] = s / (float)B_v;
-  } else {
-    vbar[(int64_t)(seg - n_anchors - M) * D + col] = s / (float)B_v;
+  if (lanes_r > 1) {   // row lanes of each column, fixed order
+    __syncthreads();
+    for (int c = threadIdx.x; c < a.D; c += nthreads) {
+      float s = colsum[c];
+      for (int l = 1; l < lanes_r; ++l) s += lane_sum[(int64_t)(l - 1) * a.D + c];
+      colsum[c] = s;
+    }
   }
+  // the cluster's column sums, reduced over its CTAs in rank order; this CTA owns one slice
+  cluster_sync_all();
+  const int cpr = (a.D + a.nsplit - 1) / a.nsplit;
+  const int c0 = split * cpr, c1 = min(a.D, c0 + cpr);
+  const float inv = 1.f / (float)nrows;
+  for (int c = c0 + threadIdx.x; c < c1; c += nthreads) {
+    float s = 0.f;
+    for (int r = 0; r < a.nsplit; ++r) s += ld_dsmem(colsum + c, (uint32_t)r);
+    out[c] = s * inv;
+  }
+  cluster_sync_all();   // no CTA leaves while a peer still reads its shared memory
 }
 
-constexpr int kScoreThreads = 256;
+// ---------------------------------------------------------------------- per-head kernel
+constexpr int kHeadThreads = 256, kHeadWarps = kHeadThreads / 32;
+
+struct HeadArgs {
+  const float* qbar;
+  const float* kbar;
+  const float* vbar;
+  const float* gram;
+  int32_t* idx;
+  float* u_out;
+  int H, d, M, n_anchors, K_eff, mode, passes, stage_kv;
+  float eps, lam_anc, lam_rec, tol;
+  float A[CAST_MAX_ANCHORS], B[CAST_MAX_ANCHORS], C[CAST_MAX_ANCHORS];   // interval (j-1, j)
+  float AL, BL, CL, AR, BR, CR;                                          // boundary sets
+};
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -157,291 +214,282 @@ __device__ __forceinline__ float warp_max(float v) {
   for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
 }
+// TopK membership of key[m] among key[0..M): rank = #(larger, or equal with a lower index).
+// Eight independent loads per round; the scan stops after a round that ranks K above m.
+__device__ __forceinline__ bool in_topk(const float* key, int M, int K, int m) {
+  const float v = key[m];
+  int rank = 0, j = 0;
+  for (; j + 8 <= M && rank < K; j += 8) {
+    float w[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) w[t] = key[j + t];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) rank += (w[t] > v) || (w[t] == v && j + t < m);
+  }
+  for (; j < M && rank < K; ++j) {
+    const float w = key[j];
+    rank += (w > v) || (w == v && j < m);
+  }
+  return rank < K;
+}
 
-// grid (H, n_anchors).  Dynamic smem: s[M], pi[M], key[M], sel[M] (int), obar[d], qb[d],
-// e[8 warps][d] scratch.
-__global__ void __launch_bounds__(kScoreThreads)
-    k_score_topk(const float* __restrict__ qbar, const float* __restrict__ kbar,
-                 const float* __restrict__ vbar, const float* __restrict__ gram, int H, int d,
-                 int M, int K_eff, float eps, int mode, int32_t* __restrict__ idx,
-                 float* __restrict__ u_out) {
+// Warp-wide sum of one value per lane (every lane gets the total).
+__device__ __forceinline__ float warp_total(float v) { return warp_sum(v); }
+
+// grid (H).  Dynamic smem (floats): qb[na*d], ob[na*d], pi[na*M], key[na*M], x[na*M], G[M],
+// e[kHeadWarps*d] (Gram scratch) and, when stage_kv, kb[M*d], vb[M*d] (this head's means).
+__global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ HeadArgs a) {
   extern __shared__ float sm[];
-  const int h = blockIdx.x, i = blockIdx.y;
-  const int D = H * d;
-  float* s = sm;
-  float* pi = s + M;
-  float* key = pi + M;
-  int* sel = reinterpret_cast<int*>(key + M);
-  float* ob = reinterpret_cast<float*>(sel + M);
-  float* qb = ob + d;
-  float* ew = qb + d;   // [kScoreThreads/32][d]
-  __shared__ float red[32];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = kScoreThreads / 32;
-  const float scale = rsqrtf((float)d);
-
-  for (int c = tid; c < d; c += kScoreThreads) qb[c] = qbar[(int64_t)i * D + h * d + c];
-  for (int m = tid; m < M; m += kScoreThreads) sel[m] = 0;
-  __syncthreads();
-  // s_m = q_bar . k_bar_m / sqrt(d)   (Eq. pooled)
-  for (int m = warp; m < M; m += nwarp) {
-    const float* kb = kbar + (int64_t)m * D + h * d;
-    float acc = 0.f;
-    for (int c = lane; c < d; c += 32) acc = fmaf(qb[c], kb[c], acc);
-    acc = warp_sum(acc);
-    if (lane == 0) s[m] = acc * scale;
-  }
-  __syncthreads();
-  // softmax over blocks
-  float mx = -FLT_MAX;
-  for (int m = tid; m < M; m += kScoreThreads) mx = fmaxf(mx, s[m]);
-  mx = warp_max(mx);
-  if (lane == 0) red[warp] = mx;
-  __syncthreads();
-  if (warp == 0) {
-    float v = lane < nwarp ? red[lane] : -FLT_MAX;
-    v = warp_max(v);
-    if (lane == 0) red[16] = v;
-  }
-  __syncthreads();
-  mx = red[16];
-  float tot = 0.f;
-  for (int m = tid; m < M; m += kScoreThreads) {
-    const float e = expf(s[m] - mx);
-    pi[m] = e;
-    tot += e;
-  }
-  tot = warp_sum(tot);
-  __syncthreads();
-  if (lane == 0) red[warp] = tot;
-  __syncthreads();
-  if (warp == 0) {
-    float v = lane < nwarp ? red[lane] : 0.f;
-    v = warp_sum(v);
-    if (lane == 0) red[17] = v;
-  }
-  __syncthreads();
-  const float inv = 1.f / red[17];
-  for (int m = tid; m < M; m += kScoreThreads) pi[m] *= inv;
-  __syncthreads();
-  // o_bar = sum_m pi_m v_bar_m
-  for (int c = tid; c < d; c += kScoreThreads) {
-    float acc = 0.f;
-    for (int m = 0; m < M; ++m) acc = fmaf(pi[m], vbar[(int64_t)m * D + h * d + c], acc);
-    ob[c] = acc;
-  }
-  __syncthreads();
-  // delta_m = pi_m / (1 - pi_m + eps) (o_bar - v_bar_m);  u_m = delta^T G delta (Eq. omission)
-  float* e = ew + warp * d;
-  for (int m = warp; m < M; m += nwarp) {
-    const float* vb = vbar + (int64_t)m * D + h * d;
-    const float coef = pi[m] / (1.f - pi[m] + eps);
-    float acc = 0.f;
-    if (gram == nullptr) {
-      for (int c = lane; c < d; c += 32) {
-        const float x = ob[c] - vb[c];
-        acc = fmaf(x, x, acc);
-      }
-    } else {
-      for (int c = lane; c < d; c += 32) e[c] = ob[c] - vb[c];
-      __syncwarp();
-      const float* G = gram + (int64_t)h * d * d;
-      for (int r = lane; r < d; r += 32) {
-        float y = 0.f;
-        for (int c = 0; c < d; ++c) y = fmaf(G[(int64_t)r * d + c], e[c], y);
-        acc = fmaf(e[r], y, acc);
-      }
-      __syncwarp();
-    }
-    acc = warp_sum(acc);
-    if (lane == 0) {
-      const float u = coef * coef * acc;
-      key[m] = (mode == CAST_ROUTE_SIMILARITY) ? s[m] : u;
-      if (u_out) u_out[((int64_t)i * H + h) * M + m] = (mode == CAST_ROUTE_SIMILARITY) ? s[m] : u;
-    }
-  }
-  __syncthreads();
-  // TopK by repeated warp argmax (ties -> lower index), then ascending compaction
-  if (warp == 0) {
-    for (int k = 0; k < K_eff; ++k) {
-      float best = -INFINITY;
-      int bi = 0x7fffffff;   // none yet
-      for (int m = lane; m < M; m += 32) {   // ascending m: strict > keeps the lower index
-        if (sel[m]) continue;
-        const float v = key[m];
-        if (bi == 0x7fffffff || v > best) { best = v; bi = m; }
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, best, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-        if (oi != 0x7fffffff && (bi == 0x7fffffff || ov > best || (ov == best && oi < bi))) {
-          best = ov;
-          bi = oi;
-        }
-      }
-      if (lane == 0 && bi != 0x7fffffff) sel[bi] = 1;
-      __syncwarp();
-    }
-    int base = 0;
-    int32_t* out = idx + ((int64_t)i * H + h) * K_eff;
-    for (int m0 = 0; m0 < M; m0 += 32) {
-      const int m = m0 + lane;
-      const bool on = m < M && sel[m];
-      const unsigned bal = __ballot_sync(0xffffffffu, on);
-      if (on) out[base + __popc(bal & ((1u << lane) - 1u))] = m;
-      base += __popc(bal);
-    }
-  }
-}
-
-// ---------------------------------------------------------------------- refinement
-struct RefineArgs {
-  int n_anchors, M, K_eff, H, passes;
-  float lam_anc, lam_rec, tol;
-  float A[CAST_MAX_ANCHORS], B[CAST_MAX_ANCHORS], C[CAST_MAX_ANCHORS];   // interval (j-1, j)
-  float AL, BL, CL, AR, BR, CR;                                          // boundary sets
-};
-
-constexpr int kRefineThreads = 256;
-
-// Warp 0: mask[m] = 1 for the K largest key[m] (ties to the lower index), 0 elsewhere.
-__device__ void warp_topk_mask(const float* key, float* mask, int M, int K, int lane) {
-  for (int m = lane; m < M; m += 32) mask[m] = 0.f;
-  __syncwarp();
-  for (int k = 0; k < K; ++k) {
-    float best = -INFINITY;
-    int bi = 0x7fffffff;
-    for (int m = lane; m < M; m += 32) {
-      if (mask[m] != 0.f) continue;
-      const float v = key[m];
-      if (bi == 0x7fffffff || v > best) { best = v; bi = m; }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, best, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-      if (oi != 0x7fffffff && (bi == 0x7fffffff || ov > best || (ov == best && oi < bi))) {
-        best = ov;
-        bi = oi;
-      }
-    }
-    if (lane == 0 && bi != 0x7fffffff) mask[bi] = 1.f;
-    __syncwarp();
-  }
-}
-
-// Eq. (risk) term of one block for the anchor pair (p, q) with coefficients (A, B, C)
-__device__ __forceinline__ float pair_risk(float A, float B, float C, float xp, float xq, float up,
-                                           float uq) {
-  return A * (1.f - xp) * up + B * (1.f - xq) * uq + 2.f * C * (1.f - xp) * (1.f - xq) * sqrtf(up * uq);
-}
-
-__device__ float block_sum(float v, float* red) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  __syncthreads();
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  float t = 0.f;
-  if (threadIdx.x < 32) {
-    t = threadIdx.x < kRefineThreads / 32 ? red[threadIdx.x] : 0.f;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (threadIdx.x == 0) red[31] = t;
-  }
-  __syncthreads();
-  return red[31];
-}
-
-// Eq. (objective) of the current masks (block-wide)
-__device__ float objective(const RefineArgs& r, const float* u, const float* x, float* red) {
-  const int na = r.n_anchors, M = r.M;
-  float v = 0.f;
-  for (int m = threadIdx.x; m < M; m += kRefineThreads) {
-    for (int i = 0; i < na; ++i) v += r.lam_anc * (1.f - x[i * M + m]) * u[i * M + m];
-    float rec = 0.f;
-    for (int j = 1; j < na; ++j)
-      rec += pair_risk(r.A[j], r.B[j], r.C[j], x[(j - 1) * M + m], x[j * M + m], u[(j - 1) * M + m],
-                       u[j * M + m]);
-    if (na >= 2) {
-      rec += pair_risk(r.AL, r.BL, r.CL, x[m], x[M + m], u[m], u[M + m]);
-      rec += pair_risk(r.AR, r.BR, r.CR, x[(na - 2) * M + m], x[(na - 1) * M + m], u[(na - 2) * M + m],
-                       u[(na - 1) * M + m]);
-    }
-    v += r.lam_rec * rec;
-  }
-  return block_sum(v, red);
-}
-
-// grid (H).  Dynamic smem: u [na][M], x [na][M], G [M], xn [M] (floats).
-__global__ void __launch_bounds__(kRefineThreads)
-    k_refine(const float* __restrict__ u_all, const __grid_constant__ RefineArgs r,
-             int32_t* __restrict__ idx) {
-  extern __shared__ float sm[];
-  __shared__ float red[32];
-  __shared__ int s_accept;
-  const int h = blockIdx.x, na = r.n_anchors, M = r.M, K = r.K_eff;
+  const int h = blockIdx.x, na = a.n_anchors, M = a.M, d = a.d, K = a.K_eff;
+  const int D = a.H * d;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  float* u = sm;
-  float* x = u + na * M;
+  float* qb = sm;
+  float* ob = qb + na * d;
+  float* pi = ob + na * d;
+  float* key = pi + na * M;
+  float* x = key + na * M;
   float* G = x + na * M;
-  float* xn = G + M;
-  for (int e = tid; e < na * M; e += kRefineThreads) {
-    const int i = e / M, m = e - i * M;
-    u[e] = u_all[((int64_t)i * r.H + h) * M + m];
+  float* ew = G + M;
+  // float4 stores below: the staged means start on a 16-byte boundary
+  float* kb_s = sm + (((ew + kHeadWarps * d) - sm + 3) & ~(ptrdiff_t)3);
+  float* vb_s = kb_s + (size_t)M * d;
+  launch_dependents();
+  grid_dependency_wait();   // the pooled means come from the preceding kernel
+  // this head's slices of q_bar (and of k_bar, v_bar when they fit), all loads in flight at once
+  const float* kb = a.kbar + h * d;
+  const float* vb = a.vbar + h * d;
+  int64_t kv_stride = D;
+  {
+    // rows of d/4 float4: q_bar rows of every anchor, then k_bar and v_bar rows when staged;
+    // each thread issues up to 8 loads before its first store
+    const int q4 = d / 4;
+    const int n_q = na * q4, n_all = n_q + (a.stage_kv ? 2 * M * q4 : 0);
+    for (int e0 = tid; e0 < n_all; e0 += 8 * kHeadThreads) {
+      float4 v[8];
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const int e = e0 + t * kHeadThreads;
+        if (e < n_q) {
+          const int i = e / q4, c = (e - i * q4) * 4;
+          v[t] = __ldcg(reinterpret_cast<const float4*>(a.qbar + (int64_t)i * D + h * d + c));
+        } else if (e < n_all) {
+          const int f = e - n_q, m = (f >> 1) / q4, c = ((f >> 1) - m * q4) * 4;
+          v[t] = __ldcg(reinterpret_cast<const float4*>(((f & 1) ? vb : kb) + (int64_t)m * D + c));
+        }
+      }
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const int e = e0 + t * kHeadThreads;
+        if (e < n_q) {
+          const int i = e / q4, c = (e - i * q4) * 4;
+          *reinterpret_cast<float4*>(qb + i * d + c) = v[t];
+        } else if (e < n_all) {
+          const int f = e - n_q, m = (f >> 1) / q4, c = ((f >> 1) - m * q4) * 4;
+          *reinterpret_cast<float4*>(((f & 1) ? vb_s : kb_s) + (int64_t)m * d + c) = v[t];
+        }
+      }
+    }
+    if (a.stage_kv) {
+      kb = kb_s;
+      vb = vb_s;
+      kv_stride = d;
+    }
   }
   __syncthreads();
-  // initial masks: TopK of u per anchor (one warp per anchor)
-  for (int i = warp; i < na; i += kRefineThreads / 32) warp_topk_mask(u + i * M, x + i * M, M, K, lane);
+  const float scale = rsqrtf((float)d);
+  // s_{i,m} = q_bar_i . k_bar_m / sqrt(d)   (Eq. pooled); eight threads per (i, m), thread k
+  // of a pair takes the float4 chunks k, k+8, ... (conflict-free shared-memory reads)
+  // (rounds are block-uniform so every lane reaches the shuffles)
+  const int sub = tid & 7, n4 = d / 4;
+  const int n_pair = na * M, rounds = (n_pair + kHeadThreads / 8 - 1) / (kHeadThreads / 8);
+  for (int rd = 0; rd < rounds; ++rd) {
+    const int p = rd * (kHeadThreads / 8) + (tid >> 3);
+    const bool live = p < n_pair;
+    const int i = live ? p / M : 0, m = live ? p - i * M : 0;
+    const float4* qv = reinterpret_cast<const float4*>(qb + i * d);
+    const float4* kv = reinterpret_cast<const float4*>(kb + (int64_t)m * kv_stride);
+    float acc = 0.f;
+    for (int c = sub; live && c < n4; c += 8) {
+      const float4 x4 = qv[c], y4 = kv[c];
+      acc = fmaf(x4.x, y4.x, fmaf(x4.y, y4.y, fmaf(x4.z, y4.z, fmaf(x4.w, y4.w, acc))));
+    }
+    acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+    acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+    acc += __shfl_xor_sync(0xffffffffu, acc, 4);
+    if (live && sub == 0) key[p] = acc * scale;
+  }
   __syncthreads();
-  float J = objective(r, u, x, red);
-  for (int pass = 1; pass <= r.passes; ++pass) {
-    bool changed = false;
-    for (int step = 0; step < na; ++step) {
-      const int i = (pass & 1) ? step : na - 1 - step;
-      // retain gains, Eqs. (gain) and (boundarygain)
-      for (int m = tid; m < M; m += kRefineThreads) {
-        const float ui = u[i * M + m];
-        float g = r.lam_anc * ui, rec = 0.f;
-        if (i >= 1) {
-          const float ul = u[(i - 1) * M + m];
-          rec += r.B[i] * ui + 2.f * r.C[i] * (1.f - x[(i - 1) * M + m]) * sqrtf(ul * ui);
+  // pi_i = softmax over blocks, one warp per anchor
+  for (int i = warp; i < na; i += kHeadWarps) {
+    const float* s = key + i * M;
+    float mx = -FLT_MAX;
+    for (int m = lane; m < M; m += 32) mx = fmaxf(mx, s[m]);
+    mx = warp_max(mx);
+    float tot = 0.f;
+    for (int m = lane; m < M; m += 32) {
+      const float e = expf(s[m] - mx);
+      pi[i * M + m] = e;
+      tot += e;
+    }
+    tot = warp_sum(tot);
+    const float inv = 1.f / tot;
+    for (int m = lane; m < M; m += 32) pi[i * M + m] *= inv;
+  }
+  __syncthreads();
+  // o_bar_i = sum_m pi_{i,m} v_bar_m (four independent partial sums)
+  for (int e = tid; e < na * d; e += kHeadThreads) {
+    const int i = e / d, c = e - i * d;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    int m = 0;
+    for (; m + 4 <= M; m += 4)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) acc[t] = fmaf(pi[i * M + m + t], vb[(int64_t)(m + t) * kv_stride + c], acc[t]);
+    for (; m < M; ++m) acc[0] = fmaf(pi[i * M + m], vb[(int64_t)m * kv_stride + c], acc[0]);
+    ob[e] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+  }
+  __syncthreads();
+  // delta_{i,m} = pi/(1 - pi + eps) (o_bar_i - v_bar_m);  u = delta^T G delta  (Eq. omission)
+  if (a.mode == CAST_ROUTE_OMISSION && a.gram == nullptr) {
+    // eight threads per (i, m) as for the scores
+    for (int rd = 0; rd < rounds; ++rd) {
+      const int p = rd * (kHeadThreads / 8) + (tid >> 3);
+      const bool live = p < n_pair;
+      const int i = live ? p / M : 0, m = live ? p - i * M : 0;
+      const float4* ov = reinterpret_cast<const float4*>(ob + i * d);
+      const float4* vv = reinterpret_cast<const float4*>(vb + (int64_t)m * kv_stride);
+      float acc = 0.f;
+      for (int c = sub; live && c < n4; c += 8) {
+        const float4 x4 = ov[c], y4 = vv[c];
+        const float t0 = x4.x - y4.x, t1 = x4.y - y4.y, t2 = x4.z - y4.z, t3 = x4.w - y4.w;
+        acc = fmaf(t0, t0, fmaf(t1, t1, fmaf(t2, t2, fmaf(t3, t3, acc))));
+      }
+      acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+      acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+      acc += __shfl_xor_sync(0xffffffffu, acc, 4);
+      if (live && sub == 0) {
+        const float coef = pi[p] / (1.f - pi[p] + a.eps);
+        key[p] = coef * coef * acc;
+      }
+    }
+    __syncthreads();
+  } else if (a.mode == CAST_ROUTE_OMISSION) {
+    float* e = ew + warp * d;
+    for (int p = warp; p < na * M; p += kHeadWarps) {
+      const int i = p / M, m = p - i * M;
+      const float* vm = vb + (int64_t)m * kv_stride;
+      const float coef = pi[p] / (1.f - pi[p] + a.eps);
+      float acc = 0.f;
+      {
+        for (int c = lane; c < d; c += 32) e[c] = ob[i * d + c] - vm[c];
+        __syncwarp();
+        const float* Gm = a.gram + (int64_t)h * d * d;
+        for (int r = lane; r < d; r += 32) {
+          float y = 0.f;
+          for (int c = 0; c < d; ++c) y = fmaf(Gm[(int64_t)r * d + c], e[c], y);
+          acc = fmaf(e[r], y, acc);
         }
-        if (i + 1 < na) {
-          const float ur = u[(i + 1) * M + m];
-          rec += r.A[i + 1] * ui + 2.f * r.C[i + 1] * (1.f - x[(i + 1) * M + m]) * sqrtf(ui * ur);
+        __syncwarp();
+      }
+      acc = warp_sum(acc);
+      if (lane == 0) key[p] = coef * coef * acc;
+    }
+    __syncthreads();
+  }
+  if (a.u_out)
+    for (int p = tid; p < na * M; p += kHeadThreads) {
+      const int i = p / M, m = p - i * M;
+      a.u_out[((int64_t)i * a.H + h) * M + m] = key[p];
+    }
+  if (K == 0) return;
+  // initial masks: TopK of each anchor's key (Eq. topk)
+  for (int p = tid; p < na * M; p += kHeadThreads) {
+    const int i = p / M, m = p - i * M;
+    x[p] = in_topk(key + i * M, M, K, m) ? 1.f : 0.f;
+  }
+  __syncthreads();
+  if (a.passes > 0 && K < M) {
+    // Alg. (routing) with u = key.  Shared state for the passes: sq[j][m] = sqrt(u_{j-1,m}
+    // u_{j,m}) of every adjacent anchor pair (pi is no longer needed) and the interval
+    // coefficients (o_bar is no longer needed); the boundary sets use the pairs (0, 1) and
+    // (na-2, na-1), i.e. sq[1] and sq[na-1].
+    const float* u = key;
+    float* sq = pi;
+    float* cA = ob;
+    float* cB = ob + na;
+    float* cC = ob + 2 * na;
+    for (int p = tid; p < na * M; p += kHeadThreads)
+      if (p >= M) sq[p] = sqrtf(u[p - M] * u[p]);
+    for (int j = tid; j < na; j += kHeadThreads) {
+      cA[j] = a.A[j];
+      cB[j] = a.B[j];
+      cC[j] = a.C[j];
+    }
+    __syncthreads();
+    if (warp == 0) {
+      // one warp: fixed-budget best responses on J (Eq. objective); lane l owns blocks l, l+32, ...
+      const float AL = a.AL, BL = a.BL, CL = a.CL, AR = a.AR, BR = a.BR, CR = a.CR;
+      const float lam_anc = a.lam_anc, lam_rec = a.lam_rec;
+      float Jl = 0.f;
+      for (int m = lane; m < M; m += 32) {
+        for (int i = 0; i < na; ++i) Jl += lam_anc * (1.f - x[i * M + m]) * u[i * M + m];
+        float rec = 0.f;
+        for (int j = 1; j < na; ++j) {
+          const float xp = 1.f - x[(j - 1) * M + m], xq = 1.f - x[j * M + m];
+          rec += cA[j] * xp * u[(j - 1) * M + m] + cB[j] * xq * u[j * M + m] + 2.f * cC[j] * xp * xq * sq[j * M + m];
         }
         if (na >= 2) {
-          if (i == 0) rec += r.AL * ui + 2.f * r.CL * (1.f - x[M + m]) * sqrtf(ui * u[M + m]);
-          if (i == 1) rec += r.BL * ui + 2.f * r.CL * (1.f - x[m]) * sqrtf(ui * u[m]);
-          if (i == na - 2) rec += r.AR * ui + 2.f * r.CR * (1.f - x[(na - 1) * M + m]) * sqrtf(ui * u[(na - 1) * M + m]);
-          if (i == na - 1) rec += r.BR * ui + 2.f * r.CR * (1.f - x[(na - 2) * M + m]) * sqrtf(ui * u[(na - 2) * M + m]);
+          const float x0 = 1.f - x[m], x1 = 1.f - x[M + m];
+          rec += AL * x0 * u[m] + BL * x1 * u[M + m] + 2.f * CL * x0 * x1 * sq[M + m];
+          const int r0 = (na - 2) * M + m, r1 = (na - 1) * M + m;
+          const float y0 = 1.f - x[r0], y1 = 1.f - x[r1];
+          rec += AR * y0 * u[r0] + BR * y1 * u[r1] + 2.f * CR * y0 * y1 * sq[r1];
         }
-        G[m] = g + r.lam_rec * rec;
+        Jl += lam_rec * rec;
       }
-      __syncthreads();
-      if (warp == 0) warp_topk_mask(G, xn, M, K, lane);
-      __syncthreads();
-      float d = 0.f;
-      for (int m = tid; m < M; m += kRefineThreads) d += G[m] * (xn[m] - x[i * M + m]);
-      const float gain = block_sum(d, red);
-      if (tid == 0) s_accept = gain > r.tol * fmaxf(J, 1e-8f);
-      __syncthreads();
-      if (s_accept) {
-        for (int m = tid; m < M; m += kRefineThreads) x[i * M + m] = xn[m];
-        __syncthreads();
-        J = objective(r, u, x, red);
-        changed = true;
+      float J = warp_total(Jl);
+      for (int pass = 1; pass <= a.passes; ++pass) {
+        bool changed = false;
+        for (int step = 0; step < na; ++step) {
+          const int i = (pass & 1) ? step : na - 1 - step;
+          // retain gains, Eqs. (gain) and (boundarygain)
+          for (int m = lane; m < M; m += 32) {
+            const float ui = u[i * M + m];
+            float rec = 0.f;
+            if (i >= 1) rec += cB[i] * ui + 2.f * cC[i] * (1.f - x[(i - 1) * M + m]) * sq[i * M + m];
+            if (i + 1 < na) rec += cA[i + 1] * ui + 2.f * cC[i + 1] * (1.f - x[(i + 1) * M + m]) * sq[(i + 1) * M + m];
+            if (na >= 2) {
+              if (i == 0) rec += AL * ui + 2.f * CL * (1.f - x[M + m]) * sq[M + m];
+              if (i == 1) rec += BL * ui + 2.f * CL * (1.f - x[m]) * sq[M + m];
+              if (i == na - 2) rec += AR * ui + 2.f * CR * (1.f - x[(na - 1) * M + m]) * sq[(na - 1) * M + m];
+              if (i == na - 1) rec += BR * ui + 2.f * CR * (1.f - x[(na - 2) * M + m]) * sq[(na - 1) * M + m];
+            }
+            G[m] = lam_anc * ui + lam_rec * rec;
+          }
+          __syncwarp();
+          // best response TopK(G) and its gain sum_m G_m (x_new - x_i); J is affine in x_i, so
+          // the accepted step lowers J by exactly that gain
+          float gl = 0.f;
+          for (int m = lane; m < M; m += 32) {
+            const float nx = in_topk(G, M, K, m) ? 1.f : 0.f;
+            gl += G[m] * (nx - x[i * M + m]);
+          }
+          const float gain = warp_total(gl);
+          if (gain > a.tol * fmaxf(J, 1e-8f)) {   // uniform across the warp
+            for (int m = lane; m < M; m += 32) x[i * M + m] = in_topk(G, M, K, m) ? 1.f : 0.f;
+            J -= gain;
+            changed = true;
+          }
+          __syncwarp();
+        }
+        if (!changed) break;
       }
     }
-    if (!changed) break;
   }
   __syncthreads();
   // ascending block indices of every anchor's mask
-  for (int i = warp; i < na; i += kRefineThreads / 32) {
+  for (int i = warp; i < na; i += kHeadWarps) {
     int base = 0;
-    int32_t* out = idx + ((int64_t)i * r.H + h) * K;
+    int32_t* out = a.idx + ((int64_t)i * a.H + h) * K;
     for (int m0 = 0; m0 < M; m0 += 32) {
       const int m = m0 + lane;
       const bool on = m < M && x[i * M + m] != 0.f;
@@ -454,27 +502,42 @@ __global__ void __launch_bounds__(kRefineThreads)
 
 }  // namespace
 
-size_t refine_smem_bytes(const cast_route_args& a) {
-  return (size_t)(2 * a.n_anchors + 2) * (size_t)a.M * sizeof(float);
+size_t route_head_smem_bytes(const cast_route_args& a) {
+  return ((size_t)2 * a.n_anchors * a.d + (size_t)3 * a.n_anchors * a.M + (size_t)a.M +
+          (size_t)kHeadWarps * a.d) * sizeof(float);
+}
+
+namespace {
+constexpr size_t kHeadSmemLimit = 200 * 1024;
+// k_bar and v_bar of one head join the shared state when everything fits
+size_t head_staged_bytes(const cast_route_args& a) {
+  return align_up(route_head_smem_bytes(a), 16) + (size_t)2 * a.M * a.d * sizeof(float);
+}
+bool head_stages_kv(const cast_route_args& a) { return head_staged_bytes(a) <= kHeadSmemLimit; }
+}  // namespace
+
+size_t route_pool_smem_bytes(const cast_route_args& a) {
+  const int D = a.H * a.d;
+  return (size_t)pool_shape(D, a.dtype == CAST_BF16 ? 2 : 4).lanes_r * D * sizeof(float);
 }
 
 RoutePlan route_plan(const cast_route_args& a) {
   RoutePlan p{};
   const int D = a.H * a.d;
   p.n_seg = a.n_anchors + 2 * a.M;
-  // enough CTAs to cover the SMs several times, each streaming >= ~128 rows
-  const int64_t rows = (int64_t)a.n_anchors * a.S + 2LL * a.M * a.B_v;
-  int target = 4 * 152;
-  int nsplit = (int)((target + p.n_seg - 1) / p.n_seg);
+  // a cluster of up to 8 CTAs per segment, enough CTAs to cover the SMs a few times, each
+  // streaming >= 64 rows
+  int dev = 0, nsm = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  const int target = 4 * (nsm > 0 ? nsm : 148);
+  int nsplit = (target + p.n_seg - 1) / p.n_seg;
+  if (nsplit > kMaxClusterSplit) nsplit = kMaxClusterSplit;
   const int maxrows = a.M > 0 ? (a.S > a.B_v ? a.S : a.B_v) : a.S;
   while (nsplit > 1 && (maxrows + nsplit - 1) / nsplit < 64) --nsplit;
   if (nsplit < 1) nsplit = 1;
-  (void)rows;
   p.nsplit = nsplit;
-  p.partial_bytes = align_up((size_t)p.n_seg * nsplit * D * sizeof(float));
   p.pooled_bytes = align_up((size_t)p.n_seg * D * sizeof(float));
-  p.u_bytes = (a.refine_passes > 0 && !a.u) ? align_up((size_t)a.n_anchors * a.H * a.M * sizeof(float)) : 0;
-  p.total_bytes = p.partial_bytes + p.pooled_bytes + p.u_bytes;
+  p.total_bytes = p.pooled_bytes;
   return p;
 }
 
@@ -483,9 +546,7 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   const int D = a.H * a.d;
   const int K_eff = a.K < a.M ? a.K : a.M;
   if (a.M == 0) return CAST_OK;   // nothing to route (App. B.3 bypass)
-  char* w = static_cast<char*>(ws);
-  float* partial = reinterpret_cast<float*>(w);
-  float* pooled = reinterpret_cast<float*>(w + p.partial_bytes);
+  float* pooled = static_cast<float*>(ws);
   float* qbar = a.qbar ? a.qbar : pooled;
   float* kbar = a.kbar ? a.kbar : pooled + (size_t)a.n_anchors * D;
   float* vbar = a.vbar ? a.vbar : pooled + (size_t)(a.n_anchors + a.M) * D;
@@ -494,6 +555,9 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   pa.q = static_cast<const char*>(a.q);
   pa.k = static_cast<const char*>(a.k_hist);
   pa.v = static_cast<const char*>(a.v_hist);
+  pa.qbar = qbar;
+  pa.kbar = kbar;
+  pa.vbar = vbar;
   pa.q_row_stride = a.q_row_stride;
   pa.hist_row_stride = a.hist_row_stride;
   pa.n_anchors = a.n_anchors;
@@ -504,77 +568,98 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   pa.nsplit = p.nsplit;
   pa.elt = a.dtype == CAST_BF16 ? 2 : 4;
   for (int k = 0; k < a.n_anchors; ++k) pa.anchors[k] = a.anchors[k];
-  dim3 grid(p.nsplit, p.n_seg);
-  if (a.dtype == CAST_BF16)
-    k_pool<__nv_bfloat16><<<grid, kPoolThreads, 0, st>>>(pa, partial);
-  else
-    k_pool<float><<<grid, kPoolThreads, 0, st>>>(pa, partial);
+
+  const size_t psm = route_pool_smem_bytes(a);
+  auto pool_fn = a.dtype == CAST_BF16 ? k_pool<__nv_bfloat16> : k_pool<float>;
+  if (psm > 48 * 1024 &&
+      cudaFuncSetAttribute(pool_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psm) != cudaSuccess)
+    return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory for pooling", psm);
+  const PoolShape ps = pool_shape(D, pa.elt);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(p.nsplit, p.n_seg, 1);
+  cfg.blockDim = dim3(ps.cgs * ps.lanes_r, 1, 1);
+  cfg.dynamicSmemBytes = psm;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = p.nsplit;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, pool_fn, pa) != cudaSuccess) return check_launch("routing pool kernel");
   cast_status s = check_launch("routing pool kernel");
   if (s != CAST_OK) return s;
-  dim3 gf((D + 255) / 256, p.n_seg);
-  k_finalize<<<gf, 256, 0, st>>>(partial, qbar, kbar, vbar, a.n_anchors, a.M, a.S, a.B_v, D,
-                                 p.nsplit);
-  s = check_launch("routing finalize kernel");
-  if (s != CAST_OK) return s;
-  const size_t smem = (size_t)(4 * a.M + 2 * a.d + (kScoreThreads / 32) * a.d) * sizeof(float);
-  if (smem > 48 * 1024) {
-    if (cudaFuncSetAttribute(k_score_topk, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem) != cudaSuccess)
-      return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory", smem);
-  }
-  const bool refine = a.refine_passes > 0 && K_eff > 0 && K_eff < a.M;
-  float* u_buf = a.u ? a.u : (p.u_bytes ? reinterpret_cast<float*>(w + p.partial_bytes + p.pooled_bytes) : nullptr);
-  k_score_topk<<<dim3(a.H, a.n_anchors), kScoreThreads, smem, st>>>(
-      qbar, kbar, vbar, a.gram, a.H, a.d, a.M, K_eff, a.eps, a.mode, a.idx, u_buf);
-  s = check_launch("routing score/TopK kernel");
-  if (s != CAST_OK || !refine) return s;
-  // Alg. (routing): interval and boundary coefficients of the anchor layout (Eqs. abc,
-  // boundarycoeff), then the directional best-response passes on the GPU
-  RefineArgs r{};
-  r.n_anchors = a.n_anchors;
-  r.M = a.M;
-  r.K_eff = K_eff;
-  r.H = a.H;
-  r.passes = a.refine_passes;
-  r.lam_anc = a.lambda_anc;
-  r.lam_rec = a.lambda_rec;
-  r.tol = a.refine_tol;
-  for (int j = 1; j < a.n_anchors; ++j) {
-    const int x0 = a.anchors[j - 1], x1 = a.anchors[j];
-    double A = 0, B = 0, C = 0;
-    for (int t = x0 + 1; t < x1; ++t) {
-      const double al = (double)(t - x0) / (double)(x1 - x0);
-      A += (1 - al) * (1 - al);
-      B += al * al;
-      C += al * (1 - al);
-    }
-    r.A[j] = (float)A;
-    r.B[j] = (float)B;
-    r.C[j] = (float)C;
-  }
-  if (a.n_anchors >= 2) {
-    auto bset = [&](int x0, int x1, int t0, int t1, float& A, float& B, float& C) {
-      double sa = 0, sb = 0, sc = 0;
-      for (int t = t0; t < t1; ++t) {
+
+  HeadArgs ha{};
+  ha.qbar = qbar;
+  ha.kbar = kbar;
+  ha.vbar = vbar;
+  ha.gram = a.gram;
+  ha.idx = a.idx;
+  ha.u_out = a.u;
+  ha.H = a.H;
+  ha.d = a.d;
+  ha.M = a.M;
+  ha.n_anchors = a.n_anchors;
+  ha.K_eff = K_eff;
+  ha.mode = a.mode;
+  ha.passes = a.refine_passes;
+  ha.eps = a.eps;
+  ha.lam_anc = a.lambda_anc;
+  ha.lam_rec = a.lambda_rec;
+  ha.tol = a.refine_tol;
+  if (a.refine_passes > 0) {
+    // interval and boundary coefficients of the anchor layout (Eqs. abc, boundarycoeff) with
+    // the alpha of Eq. (block)
+    for (int j = 1; j < a.n_anchors; ++j) {
+      const int x0 = a.anchors[j - 1], x1 = a.anchors[j];
+      double A = 0, B = 0, C = 0;
+      for (int t = x0 + 1; t < x1; ++t) {
         const double al = (double)(t - x0) / (double)(x1 - x0);
-        sa += (1 - al) * (1 - al);
-        sb += al * al;
-        sc += std::fabs(al * (1 - al));
+        A += (1 - al) * (1 - al);
+        B += al * al;
+        C += al * (1 - al);
       }
-      A = (float)sa;
-      B = (float)sb;
-      C = (float)sc;
-    };
-    bset(a.anchors[0], a.anchors[1], 0, a.anchors[0], r.AL, r.BL, r.CL);
-    bset(a.anchors[a.n_anchors - 2], a.anchors[a.n_anchors - 1], a.anchors[a.n_anchors - 1] + 1,
-         a.n_frames, r.AR, r.BR, r.CR);
+      ha.A[j] = (float)A;
+      ha.B[j] = (float)B;
+      ha.C[j] = (float)C;
+    }
+    if (a.n_anchors >= 2) {
+      auto bset = [&](int x0, int x1, int t0, int t1, float& A, float& B, float& C) {
+        double sa = 0, sb = 0, sc = 0;
+        for (int t = t0; t < t1; ++t) {
+          const double al = (double)(t - x0) / (double)(x1 - x0);
+          sa += (1 - al) * (1 - al);
+          sb += al * al;
+          sc += std::fabs(al * (1 - al));
+        }
+        A = (float)sa;
+        B = (float)sb;
+        C = (float)sc;
+      };
+      bset(a.anchors[0], a.anchors[1], 0, a.anchors[0], ha.AL, ha.BL, ha.CL);
+      bset(a.anchors[a.n_anchors - 2], a.anchors[a.n_anchors - 1], a.anchors[a.n_anchors - 1] + 1,
+           a.n_frames, ha.AR, ha.BR, ha.CR);
+    }
   }
-  const size_t rsm = refine_smem_bytes(a);
-  if (rsm > 48 * 1024 &&
-      cudaFuncSetAttribute(k_refine, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsm) != cudaSuccess)
-    return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory for refinement", rsm);
-  k_refine<<<a.H, kRefineThreads, rsm, st>>>(u_buf, r, a.idx);
-  return check_launch("routing refinement kernel");
+  ha.stage_kv = head_stages_kv(a) ? 1 : 0;
+  const size_t hsm = ha.stage_kv ? head_staged_bytes(a) : route_head_smem_bytes(a);
+  if (hsm > 48 * 1024 &&
+      cudaFuncSetAttribute(k_head, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)hsm) != cudaSuccess)
+    return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory", hsm);
+  cudaLaunchConfig_t hc{};
+  hc.gridDim = dim3(a.H, 1, 1);
+  hc.blockDim = dim3(kHeadThreads, 1, 1);
+  hc.dynamicSmemBytes = hsm;
+  hc.stream = st;
+  cudaLaunchAttribute hat[1];
+  hat[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  hat[0].val.programmaticStreamSerializationAllowed = 1;
+  hc.attrs = hat;
+  hc.numAttrs = 1;
+  if (cudaLaunchKernelEx(&hc, k_head, ha) != cudaSuccess) return check_launch("routing head kernel");
+  return check_launch("routing head kernel");
 }
 
 }  // namespace cast

@@ -54,9 +54,10 @@ def test_noalloc_matches_workspace_entry_point_twice(lib):
 
 
 def test_noalloc_rejects_problems_above_its_fixed_scratch(lib):
-    # 64 history blocks x 32 heads x 128 channels of pooled partial sums exceed 16 MiB
+    # the f32 means of 2 anchor frames and 600 key and value blocks of 32 heads x 128 channels
+    # (19.7 MB) exceed 16 MiB
     q = torch.zeros((2, 64, 32, 128), dtype=torch.bfloat16, device="cuda")
-    k = torch.zeros((300, 64, 32, 128), dtype=torch.bfloat16, device="cuda")
+    k = torch.zeros((600, 64, 32, 128), dtype=torch.bfloat16, device="cuda")
     a = lib._route_args(q, [0, 1], k, k, 4)
     assert lib.library().cast_route_workspace_size(C.byref(a)) > (16 << 20)
     idx = torch.empty((2, 32, 4), dtype=torch.int32, device="cuda")
