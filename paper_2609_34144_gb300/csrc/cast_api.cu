@@ -177,6 +177,7 @@ cast_status validate_par(const cast_par_args* a) {
     return fail(CAST_ERR_INVALID_ARG, "%s: bad shape F=%d Hg=%d Wg=%d C=%d", who, a->F, a->Hg,
                 a->Wg, a->C);
   if (a->C % 8 != 0) return fail(CAST_ERR_UNSUPPORTED, "%s: C=%d not a multiple of 8", who, a->C);
+  if (a->C > 4096) return fail(CAST_ERR_UNSUPPORTED, "%s: C=%d above 4096", who, a->C);
   const cast_par_params& p = a->params;
   if (p.tile_h < 1 || p.tile_h > 8 || p.tile_w < 1 || p.tile_w > 8)
     return fail(CAST_ERR_UNSUPPORTED, "%s: tile %dx%d outside 1..8", who, p.tile_h, p.tile_w);
@@ -376,7 +377,7 @@ cast_status cast_par_reconstruct(const cast_par_args* a, void* ws, size_t ws_byt
   if (s) return s;
   const ParPlan p = par_plan(*a);
   if (p.n_target == 0) return CAST_OK;
-  if (ws_bytes < p.total_bytes || !ws)
+  if (ws_bytes < p.total_bytes || (p.total_bytes && !ws))
     return fail(CAST_ERR_INVALID_ARG, "cast_par_reconstruct: workspace %zu B < %zu B", ws_bytes,
                 p.total_bytes);
   if (reinterpret_cast<uintptr_t>(ws) % kWsAlign)

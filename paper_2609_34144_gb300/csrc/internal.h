@@ -58,10 +58,12 @@ unsigned int attention_error_word(cudaStream_t st, bool clear);
 struct ParPlan {
   int n_anchor, n_pair, n_target;
   int tiles_y, tiles_x, n_tile;
-  int chunk;        // channels per work item (= threads per CTA)
-  int n_chunk;
-  int slab_tiles, n_slab;
-  size_t partial_bytes, counter_bytes, total_bytes;
+  int n_full, n_edge;   // 8x8 tiles / truncated (or non-8x8) tiles
+  int chunk;        // channels per CTA (= threads per CTA)
+  int n_chunk;      // channel groups = CTAs per cluster
+  int cl;           // CTAs per cluster
+  int n_tseg;       // time segments (runs of anchor pairs) per tile
+  size_t total_bytes;
 };
 ParPlan par_plan(const cast_par_args& a);
 cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st);

@@ -1,25 +1,25 @@
 // Phase-Aware Reconstruction of skipped frames (Section 4.3, Eqs. cross, confidence, gate,
-// fcpasm; App. A.2), one fused persistent kernel.
+// fcpasm; App. A.2), one fused single-pass kernel.
 //
-// Work is split into items (spectral tile p, channel chunk of 128 channels); one thread owns
-// one channel of the tile.  Thread 0 streams the item's anchor tiles through a TMA 4-D map
-// ([frame][row][col][channel], out-of-range rows/cols/channels arrive as zeros) into a
-// shared-memory stage, issuing anchor j+1 while the CTA transforms anchor j; the current
-// spectrum stays in registers and the previous one in shared memory.
-//   stats item  : walks the anchors in order, forms each anchor's spectrum once, and for every
-//                 adjacent anchor pair with targets reduces Z = sum_c w_c F_b conj(F_a) and
-//                 W = sum_c w_c |F_b||F_a| over the chunk's channels into a partial record.
-//   recon item  : waits until every chunk of its tile has published its partials, walks the
-//                 anchors again (re-read mostly from L2), sums the partial records of each pair
-//                 in a fixed order, derives eta, reliability, principal phases, the tile
-//                 confidence c and the gate g, and for every target t of the pair writes
-//                 R_t = IRFFT2((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
-// Items are claimed from a ticket counter in an order where every stats item of a tile is
-// claimed before any recon item of that tile, so a waiting recon item only ever waits on
-// items already held by running CTAs (no deadlock); the wait is also bounded in time.
+// A thread-block cluster owns one spectral tile position (and a run of consecutive anchor
+// pairs); its CTAs split the channels, one thread per channel.  For each anchor in time order
+// the CTA streams the anchor tile through a TMA 4-D map ([frame][row][col][channel], out-of-
+// range rows/cols/channels arrive as zeros) and forms the channel's tile spectrum in registers
+// (the previous anchor's spectrum stays in shared memory).  For every adjacent pair with
+// targets:
+//   1. each CTA reduces Z = sum_c w_c F_b conj(F_a) and W = sum_c w_c |F_b||F_a| over its
+//      channels (warp transpose reductions) into a record in its shared memory;
+//   2. after a cluster barrier every CTA sums the records of all CTAs of the cluster through
+//      distributed shared memory in rank order (deterministic, identical in every CTA) and
+//      derives eta, reliability, principal phases, the tile confidence c and the gate g;
+//   3. every target t of the pair is written straight from registers:
+//      R_t = IRFFT2((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
+// Each anchor element is read from HBM once and transformed once; each target element is
+// written once; nothing but the output goes through global memory.
 #include <cuda_bf16.h>
 
 #include <cmath>
+#include <mutex>
 
 #include "dft.cuh"
 #include "internal.h"
@@ -28,12 +28,12 @@
 namespace cast {
 namespace {
 
-constexpr int kThreads = 128;      // channels per item
+constexpr int kMaxThreads = 256;   // channels per CTA (one thread each), a multiple of 32
+constexpr int kMaxCluster = 16;    // CTAs per cluster (channel groups of one tile)
 constexpr int kNB = 40;            // stored bins of an 8-wide tile: 8 x 5
 constexpr int kNV = 3 * kNB;       // (Re Z, Im Z, W) per bin, record index = 3 * bin + component
-constexpr int kMaxSeg = 128;
+constexpr int kRec = kNV;          // record slots per CTA (96 + 1 used for 8x8 tiles)
 constexpr int kCoefBatch = 4;
-constexpr int kSpecFloats = 2 * kNB * kThreads;   // one spectrum per thread, [value][thread]
 
 __device__ unsigned int g_par_error;   // 1: a wait gave up
 
@@ -145,18 +145,15 @@ __host__ __device__ __forceinline__ constexpr int fast_value(int n) {
 struct ParKArgs {
   char* r;
   const float* wch;
-  int F, Hg, Wg, C;
-  int th, tw, tiles_x, n_tile, n_chunk;
+  int F, Hg, Wg, C, cl;                  // cl: CTAs per cluster (channel groups)
+  int th, tw, tiles_x, tiles_y, n_tile, n_tseg;
   int n_anchor;
   int anchor_frame[CAST_MAX_ANCHORS];
   int pair_tbeg[CAST_MAX_ANCHORS + 1];   // targets of pair j (anchors j-1, j) in [tbeg[j], tbeg[j+1])
   int target_frame[CAST_MAX_FRAMES];
   float target_alpha[CAST_MAX_FRAMES];
-  int n_seg;
-  int seg_first[kMaxSeg + 1];            // first ticket of each segment
-  int seg_tile0[kMaxSeg];                // first tile of the segment's slab
-  unsigned char seg_recon[kMaxSeg];
-  int total_tickets;
+  int seg_pair0[CAST_MAX_ANCHORS];       // time segment s covers pairs seg_pair0[s] .. seg_pair1[s]
+  int seg_pair1[CAST_MAX_ANCHORS];
   float tau_low, tau_high, q, T, eps, eta_rel, eta_abs, band;
   int gate_mode;
   unsigned long long wait_ns;
@@ -173,23 +170,39 @@ template <>
 __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
 
 
-__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
-  unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
 struct TileGeom {
   int y0, x0, h, w;
 };
 
-__device__ __forceinline__ TileGeom tile_geom(const ParKArgs& a, int tile) {
+// Tile i of one kind.  With 8x8 tiles: full tiles (row-major over the full-tile grid) or edge
+// tiles (the truncated last column of every tile row, then the truncated last row).  Other
+// tile sides: every tile, row-major, in the edge kind.
+__device__ __forceinline__ TileGeom tile_geom(const ParKArgs& a, int i, bool full) {
   TileGeom g;
-  const int ty = tile / a.tiles_x, tx = tile - ty * a.tiles_x;
-  g.y0 = ty * a.th;
-  g.x0 = tx * a.tw;
-  g.h = min(a.th, a.Hg - g.y0);
-  g.w = min(a.tw, a.Wg - g.x0);
+  if (a.th != 8 || a.tw != 8) {
+    const int ty = i / a.tiles_x, tx = i - (i / a.tiles_x) * a.tiles_x;
+    g.y0 = ty * a.th;
+    g.x0 = tx * a.tw;
+    g.h = min(a.th, a.Hg - g.y0);
+    g.w = min(a.tw, a.Wg - g.x0);
+    return g;
+  }
+  const int fy = a.Hg / 8, fx = a.Wg / 8;   // full tiles per column / row
+  int ty, tx;
+  if (full) {
+    ty = i / fx;
+    tx = i - ty * fx;
+  } else if (a.Wg % 8 != 0 && i < a.tiles_y) {
+    ty = i;
+    tx = fx;
+  } else {
+    ty = fy;
+    tx = i - (a.Wg % 8 != 0 ? a.tiles_y : 0);
+  }
+  g.y0 = ty * 8;
+  g.x0 = tx * 8;
+  g.h = min(8, a.Hg - g.y0);
+  g.w = min(8, a.Wg - g.x0);
   return g;
 }
 
@@ -210,24 +223,98 @@ __device__ __forceinline__ float warp_transpose_sum(float (&v)[32], int lane) {
   return v[0];
 }
 
-// Per-tile transport of one anchor pair (warp 0): theta and g per stored bin (App. A.2).
-__device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float* zw, float* th,
-                               float* gate, float* own_th, int* own_rel, int lane) {
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float y;
+  asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// atan2(y, x) in (-pi, pi]: octant reduction to a = min(|x|,|y|) / max(|x|,|y|) in [0, 1] and an
+// odd degree-15 polynomial for atan(a) whose coefficients were fitted (weighted least squares
+// at Chebyshev nodes) for this kernel; |error| < 2e-7 rad in f32.
+__device__ __forceinline__ float atan2_fast(float y, float x) {
+  const float ax = fabsf(x), ay = fabsf(y);
+  const float mx = fmaxf(ax, ay), mn = fminf(ax, ay);
+  const float a = mx > 0.f ? mn * __frcp_rn(mx) : 0.f;
+  const float a2 = a * a;
+  float p = -4.054564983e-03f;
+  p = fmaf(p, a2, 2.186295576e-02f);
+  p = fmaf(p, a2, -5.591233447e-02f);
+  p = fmaf(p, a2, 9.642198682e-02f);
+  p = fmaf(p, a2, -1.390863061e-01f);
+  p = fmaf(p, a2, 1.994656622e-01f);
+  p = fmaf(p, a2, -3.332985938e-01f);
+  p = fmaf(p, a2, 9.999993443e-01f);
+  float r = p * a;
+  if (ay > ax) r = 1.57079632679489662f - r;
+  if (x < 0.f) r = 3.14159265358979324f - r;
+  return signbit(y) ? -r : r;
+}
+
+// sin and cos of x = 2 pi k + r with |r| <= pi (Cody-Waite split of 2 pi into two parts),
+// then the hardware approximations on the reduced argument.
+__device__ __forceinline__ void sincos_reduced(float x, float* s, float* c) {
+  const float k = rintf(x * 0.159154943091895336f);
+  float r = fmaf(-k, 6.28318548202514648f, x);
+  r = fmaf(-k, -1.74845553e-07f, r);
+  __sincosf(r, s, c);
+}
+
+// Geometry of the stored bins of one tile shape (App. A.2), computed once per CTA: per bin
+// b = ky * 5 + kx the representative (mirrors point at their conjugate), the pooling weight
+// kappa (0: not stored, DC, or outside the tile), the flags, the gate threshold tau(nu) and
+// whether the band cut forces g = 0.
+struct BinInfo {
+  float tau[kNB], kap[kNB];
+  int rep[kNB];
+  unsigned char valid[kNB], selfc[kNB], mirror[kNB], cut[kNB];
+};
+
+__device__ void bin_info(const ParKArgs& a, const TileGeom& g, BinInfo& bi, int tid) {
+  if (tid >= kNB) return;
+  const int b = tid, ky = b / 5, kx = b % 5, hw2 = g.w / 2;
+  const bool valid = ky < g.h && kx <= hw2;
+  const bool edge = kx == 0 || ((g.w % 2 == 0) && kx == hw2);
+  const bool selfc = edge && (ky == 0 || ((g.h % 2 == 0) && 2 * ky == g.h));
+  const bool mirror = edge && !selfc && 2 * ky > g.h;
+  bi.valid[b] = valid;
+  bi.selfc[b] = selfc;
+  bi.mirror[b] = mirror;
+  bi.rep[b] = mirror ? (g.h - ky) * 5 + kx : b;
+  bi.kap[b] = (valid && b != 0) ? (edge ? 1.f : 2.f) : 0.f;
+  const int kys = ky <= (g.h - 1) / 2 ? ky : ky - g.h;
+  const float hh = (float)(g.h / 2) / (float)g.h, ww = (float)hw2 / (float)g.w;
+  const float rmax = sqrtf(hh * hh + ww * ww);
+  const float fy = (float)kys / (float)g.h, fx = (float)kx / (float)g.w;
+  const float nu = rmax > 0.f ? sqrtf(fy * fy + fx * fx) / rmax : 0.f;
+  bi.tau[b] = a.tau_low + (a.tau_high - a.tau_low) * powf(nu, a.q);
+  bool cut = false;
+  if (a.band >= 0.f) {
+    const float ry = (float)kys * 8.f / (float)g.h, rx = (float)kx * 8.f / (float)g.w;
+    cut = sqrtf(ry * ry + rx * rx) > a.band;
+  }
+  bi.cut[b] = cut;
+}
+
+// Per-tile transport of one anchor pair (warp 0, two bins per lane): theta and g per stored
+// bin from the pooled Z, W record (App. A.2).
+__device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const BinInfo& bi,
+                               const float* zw, float* th, float* gate, float* own_th,
+                               int* own_rel, int lane) {
   const float inv_hw = 1.f / (float)(g.h * g.w);
-  const int hw2 = g.w / 2;
-  float Zr[2], Zi[2], Wv[2], Za[2];
-  bool valid[2];
+  float Zr[2], Zi[2], Wv[2], Za[2], t[2];
   float wmax = 0.f;
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
     const int b = lane + 32 * s;
-    const int ky = b / 5, kx = b % 5;
-    valid[s] = b < kNB && ky < g.h && kx <= hw2;
-    Zr[s] = valid[s] ? zw[3 * b] * inv_hw : 0.f;
-    Zi[s] = valid[s] ? zw[3 * b + 1] * inv_hw : 0.f;
-    Wv[s] = valid[s] ? zw[3 * b + 2] * inv_hw : 0.f;
-    Za[s] = sqrtf(Zr[s] * Zr[s] + Zi[s] * Zi[s]);
-    if (valid[s]) wmax = fmaxf(wmax, Wv[s]);
+    const bool v = b < kNB && bi.valid[b];
+    Zr[s] = v ? zw[3 * b] * inv_hw : 0.f;
+    Zi[s] = v ? zw[3 * b + 1] * inv_hw : 0.f;
+    Wv[s] = v ? zw[3 * b + 2] * inv_hw : 0.f;
+    Za[s] = sqrt_approx(Zr[s] * Zr[s] + Zi[s] * Zi[s]);
+    t[s] = atan2_fast(Zi[s], Zr[s]);
+    if (t[s] <= -3.14159265358979f) t[s] = 3.14159265358979f;   // principal branch (-pi, pi]
+    if (v) wmax = fmaxf(wmax, Wv[s]);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) wmax = fmaxf(wmax, __shfl_xor_sync(0xffffffffu, wmax, o));
@@ -236,10 +323,8 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float
   for (int s = 0; s < 2; ++s) {
     const int b = lane + 32 * s;
     if (b < kNB) {
-      float t = atan2f(Zi[s], Zr[s]);
-      if (t <= -3.14159265358979f) t = 3.14159265358979f;   // principal branch (-pi, pi]
-      own_th[b] = t;
-      own_rel[b] = valid[s] && Wv[s] > eta && Za[s] > eta;
+      own_th[b] = t[s];
+      own_rel[b] = bi.valid[b] && Wv[s] > eta && Za[s] > eta;
     }
   }
   __syncwarp();
@@ -249,21 +334,18 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
     const int b = lane + 32 * s;
-    const int ky = b / 5, kx = b % 5;
-    const bool edge = kx == 0 || ((g.w % 2 == 0) && kx == hw2);
-    const bool selfc = edge && (ky == 0 || ((g.h % 2 == 0) && 2 * ky == g.h));
-    const bool mirror = edge && !selfc && 2 * ky > g.h;
-    const int rep = mirror ? (g.h - ky) * 5 + kx : b;
-    const bool rel = valid[s] && b < kNB && own_rel[rep < kNB ? rep : 0];
-    float t = (b < kNB) ? own_th[rep < kNB ? rep : 0] : 0.f;
-    if (mirror) t = -t;
-    if (!rel || selfc) t = 0.f;
-    thv[s] = t;
-    if (rel && b != 0) {
-      const float kap = edge ? 1.f : 2.f;
-      num += kap * Za[s];
-      den += kap * Wv[s];
-      any = 1;
+    thv[s] = 0.f;
+    if (b < kNB) {
+      const int rep = bi.rep[b] < kNB ? bi.rep[b] : 0;
+      const bool rel = bi.valid[b] && own_rel[rep];
+      float tv = own_th[rep];
+      if (bi.mirror[b]) tv = -tv;
+      thv[s] = (!rel || bi.selfc[b]) ? 0.f : tv;
+      if (rel && bi.kap[b] > 0.f) {
+        num += bi.kap[b] * Za[s];
+        den += bi.kap[b] * Wv[s];
+        any = 1;
+      }
     }
   }
 #pragma unroll
@@ -272,320 +354,342 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const float
     den += __shfl_xor_sync(0xffffffffu, den, o);
     any |= __shfl_xor_sync(0xffffffffu, any, o);
   }
-  const float c = any ? num / (den + a.eps) : 0.f;
-  const float hh = (float)(g.h / 2) / (float)g.h, ww = (float)hw2 / (float)g.w;
-  const float rmax = sqrtf(hh * hh + ww * ww);
+  const float c = any ? __fdividef(num, den + a.eps) : 0.f;
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
     const int b = lane + 32 * s;
     if (b >= kNB) continue;
-    const int ky = b / 5, kx = b % 5;
-    const int kys = ky <= (g.h - 1) / 2 ? ky : ky - g.h;
-    const float fy = (float)kys / (float)g.h, fx = (float)kx / (float)g.w;
-    const float nu = rmax > 0.f ? sqrtf(fy * fy + fx * fx) / rmax : 0.f;
-    const float tau = a.tau_low + (a.tau_high - a.tau_low) * powf(nu, a.q);
-    float gv = 1.f / (1.f + expf(-(c - tau) / a.T));
+    const float tau = bi.tau[b];
+    float gv = __frcp_rn(1.f + __expf((tau - c) * __frcp_rn(a.T)));
     if (a.gate_mode == CAST_GATE_ZERO) gv = 0.f;
     if (a.gate_mode == CAST_GATE_ONE) gv = 1.f;
-    if (a.band >= 0.f) {
-      const float ry = (float)kys * 8.f / (float)g.h, rx = (float)kx * 8.f / (float)g.w;
-      if (sqrtf(ry * ry + rx * rx) > a.band) gv = 0.f;
-    }
+    if (bi.cut[b]) gv = 0.f;   // outside the band
     th[b] = any ? thv[s] : 0.f;
     gate[b] = gv;
   }
 }
 
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+// Dynamic shared memory of one CTA with cc channels in a cluster of cl: the TMA stage (one
+// anchor tile, 128-byte aligned), the previous anchor's spectrum [value][thread], and the
+// records of every CTA of the cluster for two rounds [round][rank][value].
 template <typename T>
-constexpr size_t stage_bytes() { return (size_t)64 * kThreads * sizeof(T); }
+__host__ __device__ constexpr size_t stage_bytes(int cc) { return (size_t)64 * cc * sizeof(T); }
+__host__ __device__ constexpr size_t spec_bytes(int cc) { return (size_t)2 * kNB * cc * sizeof(float); }
 template <typename T>
-constexpr size_t par_dyn_smem() {
-  return 2 * stage_bytes<T>() + kSpecFloats * sizeof(float) + 128;   // in, out, previous spectrum
+__host__ __device__ constexpr size_t par_dyn_smem(int cc, int cl) {
+  return stage_bytes<T>(cc) + spec_bytes(cc) + (size_t)2 * cl * kRec * sizeof(float) + 128;
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kThreads, 2)
-    k_par(const __grid_constant__ CUtensorMap tm, const __grid_constant__ ParKArgs a,
-          float* __restrict__ partial, unsigned* __restrict__ counters) {
+__device__ __forceinline__ void st_dsmem(float* local, uint32_t rank, float v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+}
+
+// grid (cl, n_tiles_of_kind * n_tseg), cluster (cl, 1, 1), CC threads = channels per CTA.
+// FULL: every tile of the grid is 8x8 (the specialised fast path); otherwise edge tiles.
+template <typename T, int CC, bool FULL>
+__global__ void __launch_bounds__(CC, FULL ? (CC == 128 ? 3 : (CC == 192 ? 2 : 1)) : 1)
+    k_par(const __grid_constant__ CUtensorMap tm, const __grid_constant__ ParKArgs a) {
   extern __shared__ uint8_t dsm_raw[];
   const uint32_t raw = smem_u32(dsm_raw);
   uint8_t* dsm = dsm_raw + (((raw + 127u) & ~127u) - raw);   // TMA boxes without swizzle: 128 B
+  constexpr int cc = CC;
+  constexpr int nwarp = CC / 32;
   const T* stage = reinterpret_cast<const T*>(dsm);          // [y][x][channel] of one anchor tile
-  float* s_fprev = reinterpret_cast<float*>(dsm + stage_bytes<T>());   // [value][thread]
-  T* ostage = reinterpret_cast<T*>(dsm + stage_bytes<T>() + kSpecFloats * sizeof(float));
-  __shared__ float s_red[kThreads / 32][128];
+  float* s_fprev = reinterpret_cast<float*>(dsm + stage_bytes<T>(cc));   // [value][thread]
+  float* s_recv = reinterpret_cast<float*>(dsm + stage_bytes<T>(cc) + spec_bytes(cc));
+  __shared__ float s_red[nwarp][128];
   __shared__ float s_zw[kNV];
   __shared__ float s_th[kNB], s_g[kNB], s_own_th[kNB];
   __shared__ int s_own_rel[kNB];
   __shared__ float4 s_coef[kCoefBatch][kNB];
-  __shared__ int s_ticket;
+  __shared__ BinInfo s_bins;
   __shared__ __align__(8) uint64_t s_full;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // bytes one TMA box delivers: 128 channels x tile_w x tile_h (must match the tensor map)
-  const uint32_t kStageBytes = (uint32_t)(kThreads * a.tw * a.th * sizeof(T));
+  const int rank = blockIdx.x;                        // = rank in the cluster (cluster spans x)
+  const int tile = blockIdx.y / a.n_tseg, seg = blockIdx.y - tile * a.n_tseg;
+  const int j0 = a.seg_pair0[seg] - 1, j1 = a.seg_pair1[seg];   // anchors of this segment
+  const TileGeom g = tile_geom(a, tile, FULL);
+  const int c = rank * cc + tid;
+  const bool active = c < a.C;
+  const float wc = active ? (a.wch ? __ldg(a.wch + c) : 1.f) : 0.f;
+  // bytes one TMA box delivers: cc channels x tile_w x tile_h (must match the tensor map)
+  const uint32_t box_bytes = (uint32_t)(cc * a.tw * a.th * sizeof(T));
   if (tid == 0) {
     mbar_init(&s_full, 1);
     fence_barrier_init();
     tma_prefetch_desc(&tm);
+    mbar_arrive_expect_tx(&s_full, box_bytes);
+    tma_load_4d(const_cast<T*>(stage), &tm, &s_full, rank * cc, g.x0, g.y0, a.anchor_frame[j0]);
   }
+  bin_info(a, g, s_bins, tid);
   __syncthreads();
-  uint32_t n_loaded = 0;   // tiles consumed so far (phase of s_full)
+  bool ok = true;          // CTA-uniform; after a failed wait no more TMA is issued
+  int round = 0;           // pairs reduced so far: the receive buffer alternates per round, and
+                           // every round ends in a cluster barrier, so a buffer is rewritten
+                           // only after every CTA has passed the barrier that follows its reads
+  const int64_t frame_elems = (int64_t)a.Hg * a.Wg * a.C;
+  T* out = reinterpret_cast<T*>(a.r);
 
-  for (;;) {
-    if (tid == 0) s_ticket = (int)atomicAdd(&counters[0], 1u);
-    __syncthreads();
-    const int t = s_ticket;
-    __syncthreads();
-    if (t >= a.total_tickets) break;
-    int q = 0;
-    while (q + 1 < a.n_seg && a.seg_first[q + 1] <= t) ++q;
-    const int local = t - a.seg_first[q];
-    const int tile = a.seg_tile0[q] + local / a.n_chunk;
-    const int chunk = local % a.n_chunk;
-    const bool recon = a.seg_recon[q] != 0;
-    const TileGeom g = tile_geom(a, tile);
-    const int c = chunk * kThreads + tid;
-    const bool active = c < a.C;
-    const float wc = active ? (a.wch ? __ldg(a.wch + c) : 1.f) : 0.f;
-
-    if (tid == 0) {
-      if (recon) {
-        // every chunk of this tile must have published its partial records (bounded wait)
-        const uint64_t t0 = global_ns();
-        while (ld_acquire(&counters[1 + tile]) < (unsigned)a.n_chunk) {
-          if (global_ns() - t0 > a.wait_ns) {
-            atomicExch(&g_par_error, 1u);
-            break;
-          }
-          __nanosleep(128);
-        }
+  for (int j = j0; j <= j1; ++j) {
+    float re[8][5], im[8][5];
+    {
+      const bool got = ok && mbar_wait(&s_full, (uint32_t)(j - j0) & 1u, a.wait_ns);
+      float x[8][8];
+      if (FULL) {
+#pragma unroll
+        for (int y = 0; y < 8; ++y)
+#pragma unroll
+          for (int xx = 0; xx < 8; ++xx) x[y][xx] = to_f32(stage[(y * 8 + xx) * cc + tid]);
+      } else {
+#pragma unroll
+        for (int y = 0; y < 8; ++y)
+#pragma unroll
+          for (int xx = 0; xx < 8; ++xx)
+            x[y][xx] = (y < g.h && xx < g.w) ? to_f32(stage[(y * a.tw + xx) * cc + tid]) : 0.f;
       }
-      mbar_arrive_expect_tx(&s_full, kStageBytes);
-      tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * kThreads, g.x0, g.y0, a.anchor_frame[0]);
+      // the stage is free: prefetch the next anchor while this one is transformed
+      if (__syncthreads_or(ok && !got)) {
+        if (tid == 0) atomicExch(&g_par_error, 1u);
+        ok = false;
+      }
+      if (ok && tid == 0 && j + 1 <= j1) {
+        mbar_arrive_expect_tx(&s_full, box_bytes);
+        tma_load_4d(const_cast<T*>(stage), &tm, &s_full, rank * cc, g.x0, g.y0, a.anchor_frame[j + 1]);
+      }
+      if (FULL) dft::fwd2d(x, 8, 8, re, im);
+      else dft::fwd2d(x, g.h, g.w, re, im);
     }
-    if (recon) __syncthreads();
-
-    for (int j = 0; j < a.n_anchor; ++j) {
-      float re[8][5], im[8][5];
-      {
-        const bool ok = mbar_wait(&s_full, n_loaded & 1u, a.wait_ns);
-        ++n_loaded;
-        float x[8][8];
-        if (a.tw == 8 && a.th == 8) {
+    const bool has_targets = j > j0 && a.pair_tbeg[j + 1] > a.pair_tbeg[j];
+    const float* fa = s_fprev;   // spectrum of anchor j-1 (this thread's column)
+    if (has_targets) {
+      float* recv = s_recv + (size_t)(round & 1) * a.cl * kRec;   // [rank][value]
+      ++round;
+      // ---- 1. this CTA's Z = sum w F_b conj(F_a), W = sum w |F_b||F_a| (Eq. cross)
+      if (FULL) {
+        // the 96 non-redundant values in three transpose groups, W at DC by a warp sum
 #pragma unroll
-          for (int y = 0; y < 8; ++y)
+        for (int grp = 0; grp < 3; ++grp) {
+          float v[32];
 #pragma unroll
-            for (int xx = 0; xx < 8; ++xx) x[y][xx] = to_f32(stage[(y * 8 + xx) * kThreads + tid]);
-        } else {
-#pragma unroll
-          for (int y = 0; y < 8; ++y)
-#pragma unroll
-            for (int xx = 0; xx < 8; ++xx)
-              x[y][xx] = (y < a.th && xx < a.tw) ? to_f32(stage[(y * a.tw + xx) * kThreads + tid]) : 0.f;
+          for (int e = 0; e < 32; ++e) {
+            const int code = fast_value(grp * 32 + e);
+            const int b = code >> 2, comp = code & 3;
+            const float ar = fa[(2 * b) * cc + tid], ai = fa[(2 * b + 1) * cc + tid];
+            const float br = re[b / 5][b % 5], bi = im[b / 5][b % 5];
+            v[e] = comp == 0 ? wc * (br * ar + bi * ai)
+                 : comp == 1 ? wc * (bi * ar - br * ai)
+                             : wc * sqrt_approx((ar * ar + ai * ai) * (br * br + bi * bi));
+          }
+          s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
         }
-        // the stage is free: prefetch the next anchor while transforming this one.  A tile
-        // that never arrived ends the kernel for every thread of the CTA (error word set);
-        // the barrier is never re-armed in an incomplete phase.
-        if (__syncthreads_or(!ok)) {
-          if (tid == 0) atomicExch(&g_par_error, 1u);
-          return;
-        }
-        if (tid == 0 && j + 1 < a.n_anchor) {
-          mbar_arrive_expect_tx(&s_full, kStageBytes);
-          tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * kThreads, g.x0, g.y0,
-                      a.anchor_frame[j + 1]);
-        }
-        dft::fwd2d(x, g.h, g.w, re, im);
-      }
-      const bool has_targets = j > 0 && a.pair_tbeg[j + 1] > a.pair_tbeg[j];
-      const float* fa = s_fprev;   // spectrum of anchor j-1 (this thread's column)
-      if (has_targets && !recon) {
-        // ---- partial Z = sum w F_b conj(F_a), W = sum w |F_b||F_a| over the chunk (Eq. cross)
-        if (g.h == 8 && g.w == 8) {
-          // the 96 non-redundant values in three transpose groups, W at DC by a warp sum
+        float wdc = wc * fabsf(re[0][0]) * fabsf(fa[tid]);
 #pragma unroll
-          for (int grp = 0; grp < 3; ++grp) {
-            float v[32];
+        for (int o = 16; o > 0; o >>= 1) wdc += __shfl_xor_sync(0xffffffffu, wdc, o);
+        if (lane == 0) s_red[warp][96] = wdc;
+      } else {
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const int code = fast_value(grp * 32 + e);
-              const int b = code >> 2, comp = code & 3;
-              const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
+        for (int grp = 0; grp < 4; ++grp) {
+          float v[32];
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const int vi = grp * 32 + e;
+            if (vi < kNV) {
+              const int b = vi / 3, comp = vi % 3;
+              const float ar = fa[(2 * b) * cc + tid], ai = fa[(2 * b + 1) * cc + tid];
               const float br = re[b / 5][b % 5], bi = im[b / 5][b % 5];
               v[e] = comp == 0 ? wc * (br * ar + bi * ai)
                    : comp == 1 ? wc * (bi * ar - br * ai)
-                               : wc * sqrtf((ar * ar + ai * ai) * (br * br + bi * bi));
-            }
-            s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
-          }
-          float wdc = wc * fabsf(re[0][0]) * fabsf(fa[tid]);
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) wdc += __shfl_xor_sync(0xffffffffu, wdc, o);
-          if (lane == 0) s_red[warp][96] = wdc;
-          __syncthreads();
-          if (tid < kNV) {
-            const int src = a.fast_src[tid];
-            float sum = 0.f;
-            if (src != 0) {
-              const int k = (src > 0 ? src : -src) - 1;
-#pragma unroll
-              for (int w = 0; w < kThreads / 32; ++w) sum += s_red[w][k];
-              if (src < 0) sum = -sum;
-            }
-            partial[(((int64_t)j * a.n_tile + tile) * a.n_chunk + chunk) * kNV + tid] = sum;
-          }
-          __syncthreads();
-        } else {
-#pragma unroll
-          for (int grp = 0; grp < 4; ++grp) {
-            float v[32];
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const int vi = grp * 32 + e;
-              if (vi < kNV) {
-                const int b = vi / 3, comp = vi % 3;
-                const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
-                const float br = re[b / 5][b % 5], bi = im[b / 5][b % 5];
-                v[e] = comp == 0 ? wc * (br * ar + bi * ai)
-                     : comp == 1 ? wc * (bi * ar - br * ai)
-                                 : wc * sqrtf((ar * ar + ai * ai) * (br * br + bi * bi));
-              } else {
-                v[e] = 0.f;
-              }
-            }
-            s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
-          }
-          __syncthreads();
-          if (tid < kNV) {
-            float sum = 0.f;
-#pragma unroll
-            for (int w = 0; w < kThreads / 32; ++w) sum += s_red[w][tid];
-            partial[(((int64_t)j * a.n_tile + tile) * a.n_chunk + chunk) * kNV + tid] = sum;
-          }
-          __syncthreads();
-        }
-      } else if (has_targets && recon) {
-        // ---- transport of pair (j-1, j) on this tile
-        if (tid < kNV) {
-          // fixed-order sum over the chunks, 4 independent loads in flight
-          const float* p = partial + ((int64_t)j * a.n_tile + tile) * a.n_chunk * kNV + tid;
-          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-          int k = 0;
-          for (; k + 3 < a.n_chunk; k += 4) {
-            s0 += __ldcg(p + (int64_t)k * kNV);
-            s1 += __ldcg(p + (int64_t)(k + 1) * kNV);
-            s2 += __ldcg(p + (int64_t)(k + 2) * kNV);
-            s3 += __ldcg(p + (int64_t)(k + 3) * kNV);
-          }
-          for (; k < a.n_chunk; ++k) s0 += __ldcg(p + (int64_t)k * kNV);
-          s_zw[tid] = (s0 + s1) + (s2 + s3);
-        }
-        __syncthreads();
-        if (warp == 0) tile_transport(a, g, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
-        __syncthreads();
-        const float inv_hw = 1.f / (float)(g.h * g.w);
-        for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += kCoefBatch) {
-          const int nt = min(kCoefBatch, a.pair_tbeg[j + 1] - t0);
-          for (int e = tid; e < nt * kNB; e += kThreads) {
-            const int k = e / kNB, b = e % kNB;
-            const float al = a.target_alpha[t0 + k];
-            float sa, ca, sb, cb;
-            sincosf(s_g[b] * al * s_th[b], &sa, &ca);
-            sincosf(-s_g[b] * (1.f - al) * s_th[b], &sb, &cb);
-            const float fa_ = (1.f - al) * inv_hw, fb_ = al * inv_hw;
-            s_coef[k][b] = make_float4(fa_ * ca, fa_ * sa, fb_ * cb, fb_ * sb);
-          }
-          __syncthreads();
-          for (int k = 0; k < nt; ++k) {
-            // Eq. (fcpasm): (1-alpha) F_a U^{g alpha} + alpha F_b U^{-g (1-alpha)}, ortho scale folded
-            float hr[8][5], hi[8][5];
-#pragma unroll
-            for (int b = 0; b < kNB; ++b) {
-              const int ky = b / 5, kx = b % 5;
-              const float4 cf = s_coef[k][b];
-              const float ar = fa[(2 * b) * kThreads + tid], ai = fa[(2 * b + 1) * kThreads + tid];
-              const float br = re[ky][kx], bi = im[ky][kx];
-              hr[ky][kx] = cf.x * ar - cf.y * ai + cf.z * br - cf.w * bi;
-              hi[ky][kx] = cf.x * ai + cf.y * ar + cf.z * bi + cf.w * br;
-            }
-            // the previous tile store must have finished reading the out stage
-            if (tid == 0) bulk_wait_read_all();
-            __syncthreads();
-            const int tw = a.tw;
-            dft::inv2d_emit(hr, hi, g.h, g.w, [&](int yy, const float* row) {
-              if (tw == 8) {
-#pragma unroll
-                for (int xx = 0; xx < 8; ++xx) ostage[(yy * 8 + xx) * kThreads + tid] = T(row[xx]);
-              } else {
-#pragma unroll
-                for (int xx = 0; xx < 8; ++xx)
-                  if (xx < tw) ostage[(yy * tw + xx) * kThreads + tid] = T(row[xx]);
-              }
-            });
-            fence_proxy_async_smem();
-            __syncthreads();
-            if (tid == 0) {
-              tma_store_4d(&tm, ostage, chunk * kThreads, g.x0, g.y0, a.target_frame[t0 + k]);
-              bulk_commit();
+                               : wc * sqrt_approx((ar * ar + ai * ai) * (br * br + bi * bi));
+            } else {
+              v[e] = 0.f;
             }
           }
-          __syncthreads();
+          s_red[warp][grp * 32 + lane] = warp_transpose_sum(v, lane);
         }
       }
-      // this anchor's spectrum becomes the previous one (thread-private column)
-      if (j + 1 < a.n_anchor) {
+      __syncthreads();
+      // the CTA's record, pushed into slot `rank` of every CTA of the cluster
+      constexpr int nrec = FULL ? 97 : kNV;
+      if (tid < nrec) {
+        float sum = 0.f;
 #pragma unroll
-        for (int b = 0; b < kNB; ++b) {
-          s_fprev[(2 * b) * kThreads + tid] = re[b / 5][b % 5];
-          s_fprev[(2 * b + 1) * kThreads + tid] = im[b / 5][b % 5];
+        for (int w = 0; w < nwarp; ++w) sum += s_red[w][tid];
+        for (int r = 0; r < a.cl; ++r) st_dsmem(recv + rank * kRec + tid, (uint32_t)r, sum);
+      }
+      // ---- 2. cluster-wide sums in rank order (local reads), then the tile's transport
+      cluster_sync_all();
+      if (tid < kNV) {
+        float sum = 0.f;
+        int k = tid, sign = 1;
+        if (FULL) {
+          const int src = a.fast_src[tid];
+          k = (src > 0 ? src : -src) - 1;
+          sign = src < 0 ? -1 : 1;
         }
+        if (k >= 0)
+          for (int r = 0; r < a.cl; ++r) sum += recv[r * kRec + k];
+        s_zw[tid] = sign < 0 ? -sum : sum;
+      }
+      __syncthreads();
+      if (warp == 0) tile_transport(a, g, s_bins, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
+      __syncthreads();
+      // ---- 3. every target of the pair (Eq. fcpasm), ortho scale folded into the coefficients
+      const float inv_hw = 1.f / (float)(g.h * g.w);
+      for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += kCoefBatch) {
+        const int nt = min(kCoefBatch, a.pair_tbeg[j + 1] - t0);
+        for (int e = tid; e < nt * kNB; e += cc) {
+          const int k = e / kNB, b = e % kNB;
+          const float al = a.target_alpha[t0 + k];
+          float sa, ca, sb, cb;
+          sincos_reduced(s_g[b] * al * s_th[b], &sa, &ca);
+          sincos_reduced(-s_g[b] * (1.f - al) * s_th[b], &sb, &cb);
+          const float fa_ = (1.f - al) * inv_hw, fb_ = al * inv_hw;
+          s_coef[k][b] = make_float4(fa_ * ca, fa_ * sa, fb_ * cb, fb_ * sb);
+        }
+        __syncthreads();
+        for (int k = 0; k < nt; ++k) {
+          float hr[8][5], hi[8][5];
+#pragma unroll
+          for (int b = 0; b < kNB; ++b) {
+            const int ky = b / 5, kx = b % 5;
+            const float4 cf = s_coef[k][b];
+            const float ar = fa[(2 * b) * cc + tid], ai = fa[(2 * b + 1) * cc + tid];
+            const float br = re[ky][kx], bi = im[ky][kx];
+            hr[ky][kx] = cf.x * ar - cf.y * ai + cf.z * br - cf.w * bi;
+            hi[ky][kx] = cf.x * ai + cf.y * ar + cf.z * bi + cf.w * br;
+          }
+          T* dst = out + (int64_t)a.target_frame[t0 + k] * frame_elems +
+                   ((int64_t)g.y0 * a.Wg + g.x0) * a.C + c;
+          const int64_t row_step = (int64_t)a.Wg * a.C;
+          const int w = FULL ? 8 : g.w, C = a.C;
+          // keeps the compiler from hoisting the stores over the blend (register pressure)
+          asm volatile("" ::: "memory");
+          auto emit = [&](int yy, const float* row) {
+            if (!active) return;
+            T* d = dst + yy * row_step;
+#pragma unroll
+            for (int xx = 0; xx < 8; ++xx)
+              if (xx < w) d[(int64_t)xx * C] = T(row[xx]);
+          };
+          if (FULL) dft::inv2d_emit(hr, hi, 8, 8, emit);
+          else dft::inv2d_emit(hr, hi, g.h, g.w, emit);
+        }
+        __syncthreads();   // s_coef is rewritten by the next batch
       }
     }
-    if (!recon) {
-      __syncthreads();
-      if (tid == 0) {
-        __threadfence();
-        atomicAdd(&counters[1 + tile], 1u);
+    // this anchor's spectrum becomes the previous one (thread-private column)
+    if (j < j1) {
+#pragma unroll
+      for (int b = 0; b < kNB; ++b) {
+        s_fprev[(2 * b) * cc + tid] = re[b / 5][b % 5];
+        s_fprev[(2 * b + 1) * cc + tid] = im[b / 5][b % 5];
       }
     }
   }
-  if (tid == 0) bulk_wait_all();   // tile stores complete before the CTA's shared memory goes
+  cluster_sync_all();   // no CTA leaves while a peer may still write its records
 }
 
-// 4-D map [F][Hg][Wg][C], box (128 channels, tw, th, 1), zero fill out of range
-bool make_r_map(CUtensorMap* m, const cast_par_args& a) {
+// 4-D map [F][Hg][Wg][C], box (cc channels, tw, th, 1), zero fill out of range
+bool make_r_map(CUtensorMap* m, const cast_par_args& a, int cc) {
   EncodeTiledFn fn = tensor_map_encoder();
   if (!fn) return false;
   const cuuint64_t elt = a.dtype == CAST_BF16 ? 2 : 4;
   cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.Wg, (cuuint64_t)a.Hg, (cuuint64_t)a.F};
   cuuint64_t strides[3] = {a.C * elt, (cuuint64_t)a.Wg * a.C * elt, (cuuint64_t)a.Hg * a.Wg * a.C * elt};
-  cuuint32_t box[4] = {(cuuint32_t)kThreads, (cuuint32_t)a.params.tile_w, (cuuint32_t)a.params.tile_h, 1};
+  cuuint32_t box[4] = {(cuuint32_t)cc, (cuuint32_t)a.params.tile_w, (cuuint32_t)a.params.tile_h, 1};
   cuuint32_t es[4] = {1, 1, 1, 1};
   return fn(m, a.dtype == CAST_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
             4, a.r, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <typename T>
-cast_status launch_typed(const CUtensorMap& tm, const ParKArgs& k, int tickets, float* partial,
-                         unsigned* counters, cudaStream_t st) {
+template <typename T, int CC, bool FULL>
+cast_status launch_kind(const CUtensorMap& tm, const ParKArgs& k, const ParPlan& p, int n_tiles,
+                        cudaStream_t st) {
+  const size_t smem = par_dyn_smem<T>(CC, p.cl);
   static bool attr_set = false;
-  constexpr size_t smem = par_dyn_smem<T>();
   if (!attr_set) {
-    if (cudaFuncSetAttribute(k_par<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-        cudaSuccess)
-      return check_launch("PAR smem attribute");
+    if (cudaFuncSetAttribute(k_par<T, CC, FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)par_dyn_smem<T>(CC, kMaxCluster)) != cudaSuccess ||
+        cudaFuncSetAttribute(k_par<T, CC, FULL>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+            cudaSuccess)
+      return check_launch("PAR kernel attributes");
     attr_set = true;
   }
-  int dev = 0, nsm = 0, occ = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_par<T>, kThreads, smem);
-  if (occ < 1) occ = 1;
-  int grid = nsm * occ;
-  if (grid > tickets) grid = tickets;
-  k_par<T><<<grid, kThreads, smem, st>>>(tm, k, partial, counters);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(p.cl, n_tiles * p.n_tseg, 1);
+  cfg.blockDim = dim3(CC, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = p.cl;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, k_par<T, CC, FULL>, &cfg) != cudaSuccess || clusters < 1) {
+    cudaGetLastError();
+    return fail(CAST_ERR_UNSUPPORTED, "PAR: a cluster of %d CTAs x %d channels cannot be resident",
+                p.cl, CC);
+  }
+  if (cudaLaunchKernelEx(&cfg, k_par<T, CC, FULL>, tm, k) != cudaSuccess) return check_launch("PAR kernel");
   return check_launch("PAR kernel");
+}
+
+// A second stream per device (and the events that fork it from and join it back into the
+// caller's stream) for the edge-tile launch, created on first use.
+struct ForkStream {
+  cudaStream_t side = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+cast_status fork_stream(ForkStream*& out) {
+  static std::mutex mu;
+  static ForkStream per_dev[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return check_launch("PAR device");
+  std::lock_guard<std::mutex> lock(mu);
+  ForkStream& f = per_dev[dev];
+  if (!f.side) {
+    if (cudaStreamCreateWithFlags(&f.side, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&f.fork, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&f.join, cudaEventDisableTiming) != cudaSuccess)
+      return check_launch("PAR side stream");
+  }
+  out = &f;
+  return CAST_OK;
+}
+
+template <typename T, int CC>
+cast_status launch_typed(const CUtensorMap& tm, const ParKArgs& k, const ParPlan& p, cudaStream_t st) {
+  if (p.n_edge == 0) return launch_kind<T, CC, true>(tm, k, p, p.n_full, st);
+  if (p.n_full == 0) return launch_kind<T, CC, false>(tm, k, p, p.n_edge, st);
+  // full tiles on the caller's stream, edge tiles concurrently on the side stream
+  ForkStream* f = nullptr;
+  cast_status s = fork_stream(f);
+  if (s != CAST_OK) return s;
+  if (cudaEventRecord(f->fork, st) != cudaSuccess || cudaStreamWaitEvent(f->side, f->fork, 0) != cudaSuccess)
+    return check_launch("PAR fork");
+  s = launch_kind<T, CC, false>(tm, k, p, p.n_edge, f->side);
+  if (s != CAST_OK) return s;
+  s = launch_kind<T, CC, true>(tm, k, p, p.n_full, st);
+  if (cudaEventRecord(f->join, f->side) != cudaSuccess || cudaStreamWaitEvent(st, f->join, 0) != cudaSuccess)
+    return check_launch("PAR join");
+  return s;
+}
+
+template <typename T>
+cast_status launch_cc(const CUtensorMap& tm, const ParKArgs& k, const ParPlan& p, cudaStream_t st) {
+  if (p.chunk == 128) return launch_typed<T, 128>(tm, k, p, st);
+  if (p.chunk == 192) return launch_typed<T, 192>(tm, k, p, st);
+  return launch_typed<T, 256>(tm, k, p, st);
 }
 
 }  // namespace
@@ -601,20 +705,32 @@ ParPlan par_plan(const cast_par_args& a) {
   p.tiles_y = (a.Hg + th - 1) / th;
   p.tiles_x = (a.Wg + tw - 1) / tw;
   p.n_tile = p.tiles_y * p.tiles_x;
-  p.chunk = kThreads;
-  p.n_chunk = (a.C + kThreads - 1) / kThreads;
-  // slab: tiles whose anchor bytes stay well inside L2 between the stats and recon passes
-  const double elt = a.dtype == CAST_BF16 ? 2.0 : 4.0;
-  const double tile_bytes = (double)na * th * tw * a.C * elt;
-  int slab = (int)(24.0e6 / (tile_bytes > 1 ? tile_bytes : 1));
-  if (slab < 1) slab = 1;
-  if (slab > p.n_tile) slab = p.n_tile;
-  while ((p.n_tile + slab - 1) / slab > kMaxSeg / 2) ++slab;
-  p.slab_tiles = slab;
-  p.n_slab = (p.n_tile + slab - 1) / slab;
-  p.partial_bytes = align_up((size_t)(na > 0 ? na : 1) * p.n_tile * p.n_chunk * kNV * sizeof(float));
-  p.counter_bytes = align_up((size_t)(1 + p.n_tile) * sizeof(unsigned));
-  p.total_bytes = p.partial_bytes + p.counter_bytes;
+  // 8x8 tiles take the specialised kernel; with smaller tile sides every tile is an edge tile
+  if (th == 8 && tw == 8) {
+    p.n_full = (a.Hg / 8) * (a.Wg / 8);
+    p.n_edge = p.n_tile - p.n_full;
+  } else {
+    p.n_full = 0;
+    p.n_edge = p.n_tile;
+  }
+  // channel groups: CTAs of 128 channels, or of 192 / 256 when more than kMaxCluster CTAs of
+  // 128 would be needed; a cluster spans the groups
+  int cc = 128;
+  while (cc < kMaxThreads && (a.C + cc - 1) / cc > kMaxCluster) cc += 64;
+  const int cl = (a.C + cc - 1) / cc;
+  p.cl = cl;
+  p.chunk = cc;
+  p.n_chunk = cl;
+  // time segments: split the anchor pairs so that the clusters cover the GPU about twice
+  int dev = 0, nsm = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  const int want_clusters = 2 * (nsm > 0 ? nsm : 148) / (cl < 2 ? 2 : cl) + 1;
+  const int n_big = p.n_full > p.n_edge ? p.n_full : p.n_edge;
+  int nseg = (want_clusters + n_big - 1) / n_big;
+  if (nseg > p.n_pair) nseg = p.n_pair;
+  if (nseg < 1) nseg = 1;
+  p.n_tseg = nseg;
+  p.total_bytes = 0;   // no workspace: the reduction stays in the cluster's shared memory
   return p;
 }
 
@@ -631,8 +747,10 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
   k.th = a.params.tile_h;
   k.tw = a.params.tile_w;
   k.tiles_x = p.tiles_x;
+  k.tiles_y = p.tiles_y;
   k.n_tile = p.n_tile;
-  k.n_chunk = p.n_chunk;
+  k.n_tseg = p.n_tseg;
+  k.cl = p.cl;
   int anchors[CAST_MAX_FRAMES];
   int na = 0;
   for (int f = 0; f < a.F; ++f)
@@ -657,26 +775,18 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
       for (int t = a1 + 1; t < a.F; ++t) add(t);
   }
   k.pair_tbeg[na] = nt;
-  // ticket schedule: S(0), S(1), R(0), S(2), R(1), ..., R(n-1)
-  int nseg = 0, ticket = 0;
-  auto seg = [&](int slab, bool recon) {
-    const int t0 = slab * p.slab_tiles;
-    const int nt_ = (t0 + p.slab_tiles <= p.n_tile ? p.slab_tiles : p.n_tile - t0);
-    k.seg_first[nseg] = ticket;
-    k.seg_tile0[nseg] = t0;
-    k.seg_recon[nseg] = recon ? 1 : 0;
-    ticket += nt_ * p.n_chunk;
-    ++nseg;
-  };
-  seg(0, false);
-  for (int s = 1; s < p.n_slab; ++s) {
-    seg(s, false);
-    seg(s - 1, true);
+  // time segments of consecutive pairs, balanced by their target counts (pairs 1 .. na-1)
+  {
+    const int npair = na - 1, nseg = p.n_tseg;
+    int pair = 1;
+    for (int sg = 0; sg < nseg; ++sg) {
+      const int left = npair - (pair - 1), segs_left = nseg - sg;
+      const int take = (left + segs_left - 1) / segs_left;
+      k.seg_pair0[sg] = pair;
+      k.seg_pair1[sg] = pair + take - 1;
+      pair += take;
+    }
   }
-  seg(p.n_slab - 1, true);
-  k.n_seg = nseg;
-  k.seg_first[nseg] = ticket;
-  k.total_tickets = ticket;
   const cast_par_params& pp = a.params;
   k.tau_low = pp.tau_low;
   k.tau_high = pp.tau_high;
@@ -707,15 +817,11 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
     }
   }
 
+  (void)ws;
   CUtensorMap tm;
-  if (!make_r_map(&tm, a)) return fail(CAST_ERR_CUDA, "PAR: cuTensorMapEncodeTiled failed");
-  char* w = static_cast<char*>(ws);
-  float* partial = reinterpret_cast<float*>(w);
-  unsigned* counters = reinterpret_cast<unsigned*>(w + p.partial_bytes);
-  if (cudaMemsetAsync(counters, 0, (size_t)(1 + p.n_tile) * sizeof(unsigned), st) != cudaSuccess)
-    return check_launch("PAR counter reset");
-  if (a.dtype == CAST_BF16) return launch_typed<__nv_bfloat16>(tm, k, ticket, partial, counters, st);
-  return launch_typed<float>(tm, k, ticket, partial, counters, st);
+  if (!make_r_map(&tm, a, p.chunk)) return fail(CAST_ERR_CUDA, "PAR: cuTensorMapEncodeTiled failed");
+  if (a.dtype == CAST_BF16) return launch_cc<__nv_bfloat16>(tm, k, p, st);
+  return launch_cc<float>(tm, k, p, st);
 }
 
 unsigned int par_error_word(cudaStream_t st, bool clear) {
