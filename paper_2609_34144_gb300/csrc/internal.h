@@ -62,7 +62,7 @@ struct ParPlan {
   int chunk;        // channels per CTA (= threads per CTA)
   int n_chunk;      // channel groups = CTAs per cluster
   int cl;           // CTAs per cluster
-  int n_tseg;       // time segments (runs of anchor pairs) per tile
+  int n_tseg_full, n_tseg_edge;   // time segments (runs of anchor pairs) per tile, per kind
   size_t total_bytes;
 };
 ParPlan par_plan(const cast_par_args& a);

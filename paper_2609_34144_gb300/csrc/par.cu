@@ -623,7 +623,7 @@ cast_status launch_kind(const CUtensorMap& tm, const ParKArgs& k, const ParPlan&
     attr_set = true;
   }
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(p.cl, n_tiles * p.n_tseg, 1);
+  cfg.gridDim = dim3(p.cl, n_tiles * k.n_tseg, 1);
   cfg.blockDim = dim3(CC, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
@@ -667,19 +667,36 @@ cast_status fork_stream(ForkStream*& out) {
   return CAST_OK;
 }
 
+// Time segments of consecutive anchor pairs (pairs 1 .. n_anchor-1), as even as possible.
+ParKArgs with_segments(const ParKArgs& k0, int nseg) {
+  ParKArgs k = k0;
+  const int npair = k.n_anchor - 1;
+  k.n_tseg = nseg;
+  int pair = 1;
+  for (int sg = 0; sg < nseg; ++sg) {
+    const int left = npair - (pair - 1), segs_left = nseg - sg;
+    const int take = (left + segs_left - 1) / segs_left;
+    k.seg_pair0[sg] = pair;
+    k.seg_pair1[sg] = pair + take - 1;
+    pair += take;
+  }
+  return k;
+}
+
 template <typename T, int CC>
-cast_status launch_typed(const CUtensorMap& tm, const ParKArgs& k, const ParPlan& p, cudaStream_t st) {
-  if (p.n_edge == 0) return launch_kind<T, CC, true>(tm, k, p, p.n_full, st);
-  if (p.n_full == 0) return launch_kind<T, CC, false>(tm, k, p, p.n_edge, st);
+cast_status launch_typed(const CUtensorMap& tm, const ParKArgs& k0, const ParPlan& p, cudaStream_t st) {
+  const ParKArgs kf = with_segments(k0, p.n_tseg_full), ke = with_segments(k0, p.n_tseg_edge);
+  if (p.n_edge == 0) return launch_kind<T, CC, true>(tm, kf, p, p.n_full, st);
+  if (p.n_full == 0) return launch_kind<T, CC, false>(tm, ke, p, p.n_edge, st);
   // full tiles on the caller's stream, edge tiles concurrently on the side stream
   ForkStream* f = nullptr;
   cast_status s = fork_stream(f);
   if (s != CAST_OK) return s;
   if (cudaEventRecord(f->fork, st) != cudaSuccess || cudaStreamWaitEvent(f->side, f->fork, 0) != cudaSuccess)
     return check_launch("PAR fork");
-  s = launch_kind<T, CC, false>(tm, k, p, p.n_edge, f->side);
+  s = launch_kind<T, CC, false>(tm, ke, p, p.n_edge, f->side);
   if (s != CAST_OK) return s;
-  s = launch_kind<T, CC, true>(tm, k, p, p.n_full, st);
+  s = launch_kind<T, CC, true>(tm, kf, p, p.n_full, st);
   if (cudaEventRecord(f->join, f->side) != cudaSuccess || cudaStreamWaitEvent(st, f->join, 0) != cudaSuccess)
     return check_launch("PAR join");
   return s;
@@ -725,11 +742,13 @@ ParPlan par_plan(const cast_par_args& a) {
   int dev = 0, nsm = 148;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
   const int want_clusters = 2 * (nsm > 0 ? nsm : 148) / (cl < 2 ? 2 : cl) + 1;
-  const int n_big = p.n_full > p.n_edge ? p.n_full : p.n_edge;
-  int nseg = (want_clusters + n_big - 1) / n_big;
-  if (nseg > p.n_pair) nseg = p.n_pair;
-  if (nseg < 1) nseg = 1;
-  p.n_tseg = nseg;
+  auto segs = [&](int n_tiles) {
+    int nseg = n_tiles > 0 ? (want_clusters + n_tiles - 1) / n_tiles : 1;
+    if (nseg > p.n_pair) nseg = p.n_pair;
+    return nseg < 1 ? 1 : nseg;
+  };
+  p.n_tseg_full = segs(p.n_full);
+  p.n_tseg_edge = segs(p.n_edge);
   p.total_bytes = 0;   // no workspace: the reduction stays in the cluster's shared memory
   return p;
 }
@@ -749,7 +768,6 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
   k.tiles_x = p.tiles_x;
   k.tiles_y = p.tiles_y;
   k.n_tile = p.n_tile;
-  k.n_tseg = p.n_tseg;
   k.cl = p.cl;
   int anchors[CAST_MAX_FRAMES];
   int na = 0;
@@ -775,18 +793,6 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
       for (int t = a1 + 1; t < a.F; ++t) add(t);
   }
   k.pair_tbeg[na] = nt;
-  // time segments of consecutive pairs, balanced by their target counts (pairs 1 .. na-1)
-  {
-    const int npair = na - 1, nseg = p.n_tseg;
-    int pair = 1;
-    for (int sg = 0; sg < nseg; ++sg) {
-      const int left = npair - (pair - 1), segs_left = nseg - sg;
-      const int take = (left + segs_left - 1) / segs_left;
-      k.seg_pair0[sg] = pair;
-      k.seg_pair1[sg] = pair + take - 1;
-      pair += take;
-    }
-  }
   const cast_par_params& pp = a.params;
   k.tau_low = pp.tau_low;
   k.tau_high = pp.tau_high;
