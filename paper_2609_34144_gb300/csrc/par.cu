@@ -223,6 +223,11 @@ __device__ __forceinline__ float warp_transpose_sum(float (&v)[32], int lane) {
   return v[0];
 }
 
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 __device__ __forceinline__ float sqrt_approx(float x) {
   float y;
   asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -235,7 +240,7 @@ __device__ __forceinline__ float sqrt_approx(float x) {
 __device__ __forceinline__ float atan2_fast(float y, float x) {
   const float ax = fabsf(x), ay = fabsf(y);
   const float mx = fmaxf(ax, ay), mn = fminf(ax, ay);
-  const float a = mx > 0.f ? mn * __frcp_rn(mx) : 0.f;
+  const float a = mx > 0.f ? mn * rcp_approx(mx) : 0.f;
   const float a2 = a * a;
   float p = -4.054564983e-03f;
   p = fmaf(p, a2, 2.186295576e-02f);
@@ -360,7 +365,7 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const BinIn
     const int b = lane + 32 * s;
     if (b >= kNB) continue;
     const float tau = bi.tau[b];
-    float gv = __frcp_rn(1.f + __expf((tau - c) * __frcp_rn(a.T)));
+    float gv = rcp_approx(1.f + __expf((tau - c) * rcp_approx(a.T)));
     if (a.gate_mode == CAST_GATE_ZERO) gv = 0.f;
     if (a.gate_mode == CAST_GATE_ONE) gv = 1.f;
     if (bi.cut[b]) gv = 0.f;   // outside the band
