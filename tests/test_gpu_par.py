@@ -50,6 +50,11 @@ CASES = [
     (5, 9, 9, 128, (2, 4), "f32", {"tile": (4, 6)}),
     (9, 8, 8, 136, (0, 8), "f32", {}),
     (9, 8, 8, 136, (0, 8), "bf16", {"band_radius": 4.0}),
+    # one tile and three anchor pairs (one time segment per pair); 1096 channels: a cluster of
+    # 9 CTAs whose last CTA is partly empty
+    (8, 8, 8, 1096, (0, 2, 5, 7), "f32", {}),
+    # the channel maximum: 16 CTAs of 256 channels
+    (5, 16, 24, 4096, (0, 4), "bf16", {}),
 ]
 
 
