@@ -524,3 +524,64 @@ def coupled_routing(u, anchors, n_frames, K, passes=2, lam_anc=1.0, lam_rec=1.0,
     if with_info:
         return idx, {"trace": trace, "ambiguous": ambiguous, "x": x, "coefficients": co}
     return idx
+
+
+# ===========================================================================
+# Control-aware frame selection (Section 3 "Interaction sensitivity" and "Coverage debt",
+# Eqs. sensitivity, debt, score; App. B.1 Eq. normalization)
+# ===========================================================================
+
+
+def control_rms(delta) -> np.ndarray:
+    """r_{i,k}: root mean square of the control update Delta_{i,k} over the frame's spatial and
+    channel coordinates (App. B.1).  delta [N_cur, ...] -> [N_cur]."""
+    d = np.asarray(delta, dtype=np.float64)
+    d = d.reshape(d.shape[0], -1)
+    return np.sqrt(np.mean(d * d, axis=1))
+
+
+def minmax_norm(r, eps=1e-8) -> np.ndarray:
+    """Eq. (normalization): (r_i - min_j r_j) / (max_j r_j - min_j r_j + eps) over the chunk."""
+    r = np.asarray(r, dtype=np.float64)
+    return (r - r.min()) / (r.max() - r.min() + eps)
+
+
+def sensitivity(deltas, eps=1e-8):
+    """Eq. (sensitivity): d_i = mean over the available control branches of Norm(Delta_{i,k});
+    None when no branch supplies a fresh response."""
+    if deltas is None or len(deltas) == 0:
+        return None
+    return np.mean([minmax_norm(control_rms(dk), eps) for dk in deltas], axis=0)
+
+
+def refresh_ages(ages, anchor_mask) -> np.ndarray:
+    """Eq. (debt): h^{l+1}_i = 0 for the anchors of block l, h^l_i + 1 for the other frames."""
+    ages = np.asarray(ages, dtype=np.int64)
+    m = np.asarray(anchor_mask).astype(bool)
+    return np.where(m, 0, ages + 1)
+
+
+def select_frames(deltas, ages, anchor_mask, K_f, lam_cov=0.5, eps=1e-8):
+    """Eqs. (debt) and (score), then the deterministic TopK_f over all current frames with ties
+    to the lower frame index.  deltas: list of the available branches' updates [N_cur, ...]
+    (empty: no fresh response, the score is the debt term alone); ages, anchor_mask: [N_cur]
+    refresh ages and anchors of block l.  Returns (anchors of block l+1 ascending, ages h^{l+1},
+    scores S^{l+1})."""
+    h = refresh_ages(ages, anchor_mask)
+    N = h.shape[0]
+    H_cov = -(-N // K_f)                      # ceil(N_cur / K_f)
+    D = h / H_cov
+    d = sensitivity(deltas, eps)
+    S = lam_cov * D if d is None else d + lam_cov * D
+    K = min(K_f, N)
+    order = sorted(range(N), key=lambda i: (-S[i], i))
+    return np.array(sorted(order[:K]), dtype=np.int64), h, S
+
+
+def selection_margin(S, K_f) -> float:
+    """Relative gap between the K_f-th and (K_f+1)-th largest score (inf when all frames are
+    selected): a selection whose gap is tiny can flip with rounding."""
+    s = np.sort(np.asarray(S, dtype=np.float64))[::-1]
+    if K_f >= len(s):
+        return np.inf
+    return (s[K_f - 1] - s[K_f]) / max(abs(s[K_f - 1]), 1e-30)

@@ -8,6 +8,7 @@ CUDA path.
 from __future__ import annotations
 
 import itertools
+import math
 import os
 
 import numpy as np
@@ -538,6 +539,100 @@ def check_coupled_routing():
                 assert O.routing_objective(u, y, co) >= J0 - 1e-6 * max(J0, 1e-8) - 1e-12
     u = r.exponential(size=(3, 4))
     assert np.array_equal(O.coupled_routing(u, [0, 2, 4], 5, 7), np.tile(np.arange(4), (3, 1)))
+
+
+
+
+# ----------------------------------------------------------------------------------------------
+# Control-aware frame selection (Eqs. sensitivity, normalization, debt, score)
+# ----------------------------------------------------------------------------------------------
+
+def check_control_rms_brute_force():
+    """r_{i,k} against pure-Python loops over every coordinate of each frame (App. B.1)."""
+    rng = np.random.default_rng(11)
+    delta = rng.standard_normal((3, 4, 5, 2))
+    r = O.control_rms(delta)
+    for i in range(3):
+        acc, n = 0.0, 0
+        for a in range(4):
+            for b in range(5):
+                for c in range(2):
+                    acc += float(delta[i, a, b, c]) ** 2
+                    n += 1
+        assert abs(r[i] - math.sqrt(acc / n)) < 1e-12
+
+
+def check_minmax_normalization():
+    """Eq. (normalization): closed forms, a constant response contributes zero, range [0, 1)."""
+    got = O.minmax_norm([1.0, 2.0, 3.0], eps=0.0)
+    assert np.allclose(got, [0.0, 0.5, 1.0])
+    got = O.minmax_norm([5.0, 1.0, 3.0], eps=1e-8)
+    assert np.allclose(got, [4.0 / (4.0 + 1e-8), 0.0, 2.0 / (4.0 + 1e-8)], rtol=0, atol=1e-15)
+    assert np.all(O.minmax_norm([2.5, 2.5, 2.5]) == 0.0)
+    rng = np.random.default_rng(3)
+    v = O.minmax_norm(rng.random(50) * 7 + 3)
+    assert v.min() == 0.0 and 0.99 < v.max() < 1.0
+
+
+def check_sensitivity_branches():
+    """Eq. (sensitivity): one branch is its own normalized score (not halved by the absent
+    branch), two branches average, no branch gives no score."""
+    rng = np.random.default_rng(5)
+    cam = rng.standard_normal((6, 3, 4)) * np.arange(1, 7)[:, None, None]
+    act = rng.standard_normal((6, 3, 4)) * np.arange(6, 0, -1)[:, None, None]
+    n_cam = O.minmax_norm(O.control_rms(cam))
+    n_act = O.minmax_norm(O.control_rms(act))
+    assert np.allclose(O.sensitivity([cam]), n_cam)
+    assert np.allclose(O.sensitivity([cam, act]), 0.5 * (n_cam + n_act))
+    assert O.sensitivity([]) is None
+    d = O.sensitivity([cam, act])
+    assert d.min() >= 0.0 and d.max() <= 1.0
+
+
+def check_frame_selection_worked_example():
+    """Eqs. (debt), (score), TopK_f worked by hand for N_cur = 4, K_f = 2 (H_cov = 2):
+    ages (0, 1, 2, 0) with anchors {0, 3} -> h = (0, 2, 3, 0), D = (0, 1, 1.5, 0);
+    one branch with r = (1, 3, 2, 1) -> Norm = (0, 1, 0.5, 0) (eps = 0);
+    S = d + 0.5 D = (0, 1.5, 1.25, 0) -> anchors {1, 2}."""
+    delta = np.array([1.0, 3.0, 2.0, 1.0])[:, None] * np.ones((4, 6))
+    anchors, h, S = O.select_frames([delta], [0, 1, 2, 0], [1, 0, 0, 1], 2, eps=0.0)
+    assert list(h) == [0, 2, 3, 0]
+    assert np.allclose(S, [0.0, 1.5, 1.25, 0.0])
+    assert list(anchors) == [1, 2]
+    # without a fresh response only the debt term: S = (0, 0.5, 0.75, 0) -> {1, 2} as well
+    anchors, _, S = O.select_frames([], [0, 1, 2, 0], [1, 0, 0, 1], 2)
+    assert np.allclose(S, [0.0, 0.5, 0.75, 0.0]) and list(anchors) == [1, 2]
+    # ties go to the lower frame index: equal ages, no response -> the first K_f frames
+    anchors, _, _ = O.select_frames([], [4, 4, 4, 4, 4], [0] * 5, 2)
+    assert list(anchors) == [0, 1]
+    # H_cov = ceil(5 / 2) = 3: ages (2, 0, 0, 0, 0), anchors {} -> D_0 = 3 / 3 = 1
+    _, h, S = O.select_frames([], [2, 0, 0, 0, 0], [0] * 5, 2)
+    assert np.allclose(S, 0.5 * h / 3.0) and S[0] == 0.5
+
+
+def check_frame_selection_brute_force():
+    """TopK_f against enumeration of every K_f-subset (largest score sum, ties to the
+    lexicographically smallest index set), including all-frames and tied scores."""
+    import itertools
+    rng = np.random.default_rng(21)
+    for trial in range(40):
+        N = int(rng.integers(2, 8))
+        K = int(rng.integers(1, N + 2))
+        ages = rng.integers(0, 4, N)
+        mask = rng.random(N) < 0.4
+        deltas = [rng.standard_normal((N, 5)) * rng.integers(1, 3, N)[:, None]
+                  for _ in range(int(rng.integers(0, 3)))]
+        if trial % 5 == 0:
+            deltas = []                                   # debt only: many ties
+        anchors, h, S = O.select_frames(deltas, ages, mask, K)
+        Ke = min(K, N)
+        best = None
+        for sub in itertools.combinations(range(N), Ke):
+            key = (-round(sum(S[list(sub)]), 12), sub)
+            if best is None or key < best:
+                best = key
+        assert tuple(anchors) == best[1], (anchors, best)
+        assert len(anchors) == Ke and np.all(np.diff(anchors) > 0)
 
 
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

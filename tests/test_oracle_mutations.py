@@ -107,7 +107,52 @@ def _coeffs_signed_boundary_cross(anchors, n_frames):
     return co
 
 
+_orig_norm = O.minmax_norm
+_orig_sens = O.sensitivity
+
+
+def _norm_from_max(r, eps=1e-8):
+    r = np.asarray(r, dtype=np.float64)
+    return (r.max() - r) / (r.max() - r.min() + eps)           # distance from the maximum
+
+
+def _sens_absent_branch_as_zero(deltas, eps=1e-8):
+    if deltas is None or len(deltas) == 0:
+        return None
+    n = [_orig_norm(O.control_rms(dk), eps) for dk in deltas]
+    return np.sum(n, axis=0) / 2.0                              # always divides by both branches
+
+
+def _ages_never_reset(ages, anchor_mask):
+    return np.asarray(ages, dtype=np.int64) + 1
+
+
+def _select_floor_hcov(deltas, ages, anchor_mask, K_f, lam_cov=0.5, eps=1e-8):
+    h = O.refresh_ages(ages, anchor_mask)
+    N = h.shape[0]
+    D = h / max(N // K_f, 1)                                    # floor instead of ceil
+    d = O.sensitivity(deltas, eps)
+    S = lam_cov * D if d is None else d + lam_cov * D
+    order = sorted(range(N), key=lambda i: (-S[i], i))
+    return np.array(sorted(order[:min(K_f, N)])), h, S
+
+
+def _select_ties_high(deltas, ages, anchor_mask, K_f, lam_cov=0.5, eps=1e-8):
+    h = O.refresh_ages(ages, anchor_mask)
+    N = h.shape[0]
+    D = h / (-(-N // K_f))
+    d = O.sensitivity(deltas, eps)
+    S = lam_cov * D if d is None else d + lam_cov * D
+    order = sorted(range(N), key=lambda i: (-S[i], -i))         # ties to the higher index
+    return np.array(sorted(order[:min(K_f, N)])), h, S
+
+
 MUTATIONS = {
+    "norm_measured_from_max": ("minmax_norm", _norm_from_max),
+    "single_branch_halved": ("sensitivity", _sens_absent_branch_as_zero),
+    "ages_never_reset": ("refresh_ages", _ages_never_reset),
+    "coverage_scale_floor": ("select_frames", _select_floor_hcov),
+    "frame_ties_high": ("select_frames", _select_ties_high),
     "gain_neighbour_mask_dropped": ("retain_gains", _gains_no_neighbour_mask),
     "gain_interval_coefficients_swapped": ("retain_gains", _gains_swapped_ab),
     "boundary_cross_without_abs": ("routing_coefficients", _coeffs_signed_boundary_cross),
