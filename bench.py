@@ -283,7 +283,7 @@ def run_gpu(args):
 
 
 # ------------------------------------------------------------------------------ scale points
-SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy")
+SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy", "select_mg")
 
 
 def _scale_setup(name, lib, torch, dev):
@@ -328,6 +328,17 @@ def _scale_setup(name, lib, torch, dev):
         return (lambda: lib.cast_anchor_attention(q, kc, vc, list(wl.anchors), kh, vh, idx, out=o,
                                                   workspace=aws),
                 flop, "FLOP")
+    if name == "select_mg":
+        w = W.SELECT_MG
+        S = w.grid[0] * w.grid[1]
+        deltas = [rnd(w.n_cur, S, w.D) for _ in range(w.n_branch)]
+        ages = torch.zeros(w.n_cur, dtype=torch.int32, device=dev)
+        mask = torch.zeros(w.n_cur, dtype=torch.uint8, device=dev)
+        mask[::2] = 1
+        ws = torch.empty(max(lib.select_workspace_size(deltas, ages, mask, w.K_f), 256),
+                         dtype=torch.uint8, device=dev)
+        return (lambda: lib.cast_select_frames(deltas, ages, mask, w.K_f, workspace=ws),
+                w.n_branch * w.n_cur * S * w.D * 2, "B")
     raise ValueError(name)
 
 

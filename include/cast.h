@@ -258,6 +258,46 @@ cast_status cast_block_step(const cast_block_args* args, void* workspace,
 size_t cast_block_workspace_size(const cast_block_args* args);
 
 /* ------------------------------------------------------------------------ */
+/* Control-aware frame selection: Section 3 ("Interaction sensitivity",      */
+/* "Coverage debt"), Eqs. (sensitivity), (debt), (score); App. B.1 Eq.      */
+/* (normalization).  Picks the anchors of block l+1 from the control-branch  */
+/* updates of block l and the frames' refresh ages.                          */
+/* ------------------------------------------------------------------------ */
+#define CAST_MAX_BRANCHES 2       /* control branches (camera, action) */
+
+typedef struct {
+  /* device [N_cur, frame_elems] feature updates of the available control branches (the
+     frame's S spatial x D channel coordinates, contiguous, 16-byte aligned); entries past
+     n_branch are ignored */
+  const void* delta[CAST_MAX_BRANCHES];
+  int32_t n_branch;               /* 0..2; 0 = no fresh response: the score is the debt term alone */
+  int32_t dtype;                  /* CAST_F32 | CAST_BF16 (of delta) */
+  int32_t n_frames;               /* N_cur, 1..CAST_MAX_FRAMES */
+  int64_t frame_elems;            /* S * D; frame_elems * element size a multiple of 16 bytes */
+  const int32_t* ages;            /* device [N_cur] refresh ages h^l */
+  const uint8_t* anchor_mask;     /* device [N_cur] anchors of block l (nonzero = anchor) */
+  int32_t K_f;                    /* anchors to select, >= 1 (K_f >= N_cur selects every frame) */
+  float lambda_cov;               /* debt weight, 0.5 in the paper */
+  float eps;                      /* epsilon of Eq. (normalization), 1e-8 */
+  int32_t* ages_out;              /* device [N_cur] h^{l+1} (may alias ages) */
+  int32_t* anchors_out;           /* device [min(K_f, N_cur)] frame indices of block l+1, ascending */
+  uint8_t* mask_out;              /* optional device [N_cur] anchor mask of block l+1 */
+  float* rms_out;                 /* optional device [n_branch, N_cur] RMS of each update (App. B.1) */
+  float* score_out;               /* optional device [N_cur] scores S^{l+1} (Eq. score) */
+} cast_select_args;
+
+/* r_{i,k} = RMS(delta_k[i]); Norm = (r - min r) / (max r - min r + eps) over the chunk per
+ * branch; d_i = mean over the given branches; h^{l+1} = 0 for anchors of block l, h^l + 1
+ * otherwise; D = h^{l+1} / ceil(N_cur / K_f); S = d + lambda_cov D (debt alone without a
+ * branch); anchors of block l+1 = the K_f largest S, ties to the lower frame index, written in
+ * ascending order.  Errors: INVALID_ARG for NULL required pointers, n_frames outside
+ * 1..CAST_MAX_FRAMES, K_f < 1, n_branch outside 0..2, misaligned delta, frame_elems < 1,
+ * negative lambda_cov or eps, a short workspace. */
+cast_status cast_select_frames(const cast_select_args* args, void* workspace,
+                               size_t workspace_bytes, void* stream);
+size_t cast_select_workspace_size(const cast_select_args* args);
+
+/* ------------------------------------------------------------------------ */
 /* Status                                                                    */
 /* ------------------------------------------------------------------------ */
 const char* cast_status_string(cast_status s);

@@ -14,7 +14,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libcast.so")
-SOURCES = ["cast_api.cu", "route.cu", "attention.cu", "par.cu", "noalloc.cu"]
+SOURCES = ["cast_api.cu", "route.cu", "attention.cu", "par.cu", "noalloc.cu", "select.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr", "-Xcompiler", "-fPIC",
          "-Xcompiler", "-fno-strict-aliasing", "-I", os.path.join(ROOT, "include"), "-I", CSRC]

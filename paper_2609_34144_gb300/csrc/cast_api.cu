@@ -14,6 +14,8 @@ namespace cast {
 
 static thread_local char g_detail[512] = "";
 
+void clear_error_detail() { g_detail[0] = 0; }
+
 cast_status fail(cast_status s, const char* fmt, ...) {
   va_list ap;
   va_start(ap, fmt);

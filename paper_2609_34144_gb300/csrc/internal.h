@@ -12,6 +12,8 @@ namespace cast {
 
 // Records a printf-style message for cast_last_error_detail() and returns `s`.
 cast_status fail(cast_status s, const char* fmt, ...);
+// Empties the message cast_last_error_detail() returns (at the start of every entry point).
+void clear_error_detail();
 // Converts a pending launch error into CAST_ERR_CUDA.
 cast_status check_launch(const char* what);
 

@@ -72,6 +72,16 @@ class BlockArgs(C.Structure):
                 ("x", _vp), ("idx_out", _vp), ("channel_weight", _vp), ("par", ParParams)]
 
 
+class SelectArgs(C.Structure):
+    _fields_ = [("delta", _vp * 2), ("n_branch", _i32), ("dtype", _i32), ("n_frames", _i32),
+                ("frame_elems", _i64), ("ages", _vp), ("anchor_mask", _vp), ("K_f", _i32),
+                ("lambda_cov", _f32), ("eps", _f32), ("ages_out", _vp), ("anchors_out", _vp),
+                ("mask_out", _vp), ("rms_out", _vp), ("score_out", _vp)]
+
+
+_lib.cast_select_frames.argtypes = [C.POINTER(SelectArgs), _vp, C.c_size_t, _vp]
+_lib.cast_select_workspace_size.argtypes = [C.POINTER(SelectArgs)]
+_lib.cast_select_workspace_size.restype = C.c_size_t
 _lib.cast_route_topk.argtypes = [C.POINTER(RouteArgs), _vp, C.c_size_t, _vp]
 _lib.cast_route_workspace_size.argtypes = [C.POINTER(RouteArgs)]
 _lib.cast_route_workspace_size.restype = C.c_size_t
@@ -95,7 +105,8 @@ for _f in ("cast_route_topk", "cast_route_topk_noalloc", "cast_anchor_attention"
            "cast_check_device"):
     getattr(_lib, _f).restype = C.c_int
 
-EXPORTED = ["cast_route_topk", "cast_route_workspace_size", "cast_route_topk_noalloc",
+EXPORTED = ["cast_select_frames", "cast_select_workspace_size",
+            "cast_route_topk", "cast_route_workspace_size", "cast_route_topk_noalloc",
             "cast_anchor_attention", "cast_attention_workspace_size",
             "cast_par_reconstruct", "cast_par_workspace_size", "cast_par_params_default",
             "cast_block_step", "cast_block_workspace_size", "cast_status_string",
@@ -368,3 +379,51 @@ def version():
 
 def library():
     return _lib
+
+
+# --------------------------------------------------------------------------- frame selection
+def select_args(deltas, ages, anchor_mask, K_f, lambda_cov=0.5, eps=1e-8):
+    """deltas: list of 0..2 device tensors [N_cur, ...] (same dtype, contiguous); ages int32 and
+    anchor_mask uint8 device tensors [N_cur]."""
+    a = SelectArgs()
+    N = ages.shape[0]
+    a.n_branch = len(deltas)
+    for k, dk in enumerate(deltas):
+        if not dk.is_contiguous():
+            raise ValueError("control updates must be contiguous")
+        a.delta[k] = dk.data_ptr()
+    a.dtype = (F32 if deltas[0].dtype == torch.float32 else BF16) if deltas else F32
+    a.n_frames = N
+    a.frame_elems = deltas[0][0].numel() if deltas else 0
+    a.ages, a.anchor_mask = _ptr(ages), _ptr(anchor_mask)
+    a.K_f, a.lambda_cov, a.eps = K_f, lambda_cov, eps
+    return a
+
+
+def cast_select_frames(deltas, ages, anchor_mask, K_f, lambda_cov=0.5, eps=1e-8, want_rms=False,
+                       want_score=False, workspace=None, stream=None):
+    """Anchors of the next block (Eqs. sensitivity, normalization, debt, score).  Returns
+    (anchors int32 [min(K_f, N)] ascending, ages int32 [N], mask uint8 [N]) plus the RMS
+    [n_branch, N] and the scores [N] when asked; all on the device."""
+    a = select_args(deltas, ages, anchor_mask, K_f, lambda_cov, eps)
+    N, dev = ages.shape[0], ages.device
+    anchors = torch.empty(min(K_f, N), dtype=torch.int32, device=dev)
+    ages_out = torch.empty(N, dtype=torch.int32, device=dev)
+    mask = torch.empty(N, dtype=torch.uint8, device=dev)
+    rms = torch.empty((len(deltas), N), dtype=torch.float32, device=dev) if want_rms else None
+    score = torch.empty(N, dtype=torch.float32, device=dev) if want_score else None
+    a.ages_out, a.anchors_out, a.mask_out = _ptr(ages_out), _ptr(anchors), _ptr(mask)
+    a.rms_out, a.score_out = _ptr(rms), _ptr(score)
+    need = _lib.cast_select_workspace_size(C.byref(a))
+    ws = workspace if workspace is not None else _workspace(need, dev)
+    _check(_lib.cast_select_frames(C.byref(a), _ptr(ws), ws.numel(), _stream(stream)))
+    out = [anchors, ages_out, mask]
+    if want_rms:
+        out.append(rms)
+    if want_score:
+        out.append(score)
+    return tuple(out)
+
+
+def select_workspace_size(deltas, ages, anchor_mask, K_f):
+    return _lib.cast_select_workspace_size(C.byref(select_args(deltas, ages, anchor_mask, K_f)))

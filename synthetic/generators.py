@@ -164,3 +164,18 @@ def planted_history(seed_seq, M: int, B_v: int, H: int, d: int, n_planted: int =
     k += koff[:, None, :, :]
     v += _gen(s_voff).standard_normal((M, 1, H, d), dtype=np.float32)
     return g, planted, k, v
+
+
+def control_updates(seed_seq, n_branch: int, N: int, S: int, D: int, lo: float = 0.2,
+                    hi: float = 2.0):
+    """Control-branch feature updates: n_branch arrays [N, S, D] float32, frame i of branch k
+    drawn N(0, a_{k,i}^2) with amplitudes a_{k,i} ~ U[lo, hi) so the frames' response
+    magnitudes differ (the conditioning-path updates of camera / action branches)."""
+    out = []
+    for child in seed_seq.spawn(n_branch):
+        ca, cn = child.spawn(2)
+        amp = _gen(ca).uniform(lo, hi, N).astype(np.float32)
+        x = normal(cn, (N, S, D))
+        x *= amp[:, None, None]
+        out.append(x)
+    return out

@@ -167,3 +167,32 @@ def stress_inputs(w: StressWorkload = STRESS):
     out["anchor_mask"] = np.ones(w.n_cur, dtype=np.uint8)
     out["planted"] = planted
     return out
+
+
+@dataclass(frozen=True)
+class SelectWorkload:
+    """Control-aware frame selection at a block of the Matrix-Game-shaped chunk: two control
+    branches (camera, action) of [N_cur, S, D] bf16 updates, K_f of N_cur frames."""
+    name: str = "select_mg_bf16_8f_30x52_c1536_k4"
+    seed: int = 5
+    n_cur: int = 8
+    grid: tuple = (30, 52)
+    D: int = 1536
+    n_branch: int = 2
+    K_f: int = 4
+
+
+SELECT_MG = SelectWorkload()
+
+
+def select_inputs(w: SelectWorkload = SELECT_MG):
+    """bf16-rounded control updates, refresh ages and the previous block's anchor mask."""
+    ss = np.random.SeedSequence(w.seed)
+    sd, sa = ss.spawn(2)
+    S = w.grid[0] * w.grid[1]
+    deltas = [G.round_bf16(x) for x in G.control_updates(sd, w.n_branch, w.n_cur, S, w.D)]
+    rng = G._gen(sa)
+    ages = rng.integers(0, 4, w.n_cur).astype(np.int32)
+    mask = np.zeros(w.n_cur, dtype=np.uint8)
+    mask[rng.choice(w.n_cur, w.K_f, replace=False)] = 1
+    return deltas, ages, mask

@@ -154,3 +154,42 @@ def test_attention_validation(lib):
     assert lib.library().cast_anchor_attention(C.byref(a), None, 0, None) == 1
     a.K_eff, a.d = 0, 80
     assert lib.library().cast_anchor_attention(C.byref(a), None, 0, None) == 2
+
+
+def _select(lib, **kw):
+    a = lib.SelectArgs()
+    a.delta[0], a.delta[1] = 0x10000, 0x20000
+    a.n_branch, a.dtype, a.n_frames, a.frame_elems = 2, lib.BF16, 8, 1560 * 1536
+    a.ages, a.anchor_mask = 0x30000, 0x40000
+    a.K_f, a.lambda_cov, a.eps = 4, 0.5, 1e-8
+    a.ages_out, a.anchors_out = 0x50000, 0x60000
+    for k, v in kw.items():
+        setattr(a, k, v)
+    return a
+
+
+@pytest.mark.parametrize("bad,status", [
+    ({"K_f": 0}, 1),
+    ({"n_frames": 0}, 1),
+    ({"n_frames": 257}, 1),
+    ({"n_branch": 3}, 1),
+    ({"frame_elems": 7}, 1),             # 14 bytes per frame: not a multiple of 16
+    ({"lambda_cov": -1.0}, 1),
+    ({"anchors_out": None}, 1),
+])
+def test_select_validation(lib, bad, status):
+    a = _select(lib, **bad)
+    assert lib.library().cast_select_frames(C.byref(a), _fake(0x100000), 1 << 20, None) == status
+    assert lib.library().cast_last_error_detail() != b""
+
+
+def test_select_misaligned_update_rejected(lib):
+    a = _select(lib)
+    a.delta[1] = 0x20008
+    assert lib.library().cast_select_frames(C.byref(a), _fake(0x100000), 1 << 20, None) == 1
+
+
+def test_select_workspace(lib):
+    assert lib.library().cast_select_workspace_size(C.byref(_select(lib, n_branch=0))) == 0
+    assert lib.library().cast_select_workspace_size(C.byref(_select(lib))) > 0
+
