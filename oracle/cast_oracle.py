@@ -585,3 +585,50 @@ def selection_margin(S, K_f) -> float:
     if K_f >= len(s):
         return np.inf
     return (s[K_f - 1] - s[K_f]) / max(abs(s[K_f - 1]), 1e-30)
+
+
+# ===========================================================================
+# Residual sites beyond the attention output (App. B.1, B.4): the output projection W_O of
+# the anchor rows, and the anchor FFN whose skipped-frame residuals PAR reconstructs
+# ===========================================================================
+
+
+def gelu_tanh(x):
+    """GELU in its tanh form, 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3)))."""
+    x = np.asarray(x, dtype=np.float64)
+    return 0.5 * x * (1.0 + np.tanh(np.sqrt(2.0 / np.pi) * (x + 0.044715 * x ** 3)))
+
+
+def linear(x, w, b=None):
+    """Rows of x times w^T (+ b): x [..., D_in], w [D_out, D_in] (the layer's weight layout)."""
+    y = np.asarray(x, np.float64) @ np.asarray(w, np.float64).T
+    return y if b is None else y + np.asarray(b, np.float64)
+
+
+def anchor_ffn(x, anchors, w1, b1, w2, b2):
+    """The FFN residual of the anchor frames: GELU(x_a W1^T + b1) W2^T + b2 for every anchor
+    frame a; x [F, S, D] -> [K_f, S, D]."""
+    return np.stack([linear(gelu_tanh(linear(x[a], w1, b1)), w2, b2) for a in anchors])
+
+
+def block_step_projected(inp, K, grid, w_o, b_o=None, p: ParParams = ParParams(), eps=1e-8,
+                         idx=None, O=None):
+    """Eq. (block) at the attention site with the output projection: anchor rows carry
+    O_a W_O^T (+ b_O), skipped rows are PAR of those rows (App. B.1: PAR acts on the site's
+    residual).  Returns (idx, O, r [N, S, D])."""
+    q = inp["q"]
+    N, S, H, d = q.shape
+    anchors = [int(a) for a in inp["anchors"]]
+    if idx is None:
+        rt = pooled_routing(q, anchors, inp["k_hist"], inp["v_hist"], eps=eps)
+        idx = topk_blocks(rt.u, K)
+    if O is None:
+        O = routed_attention(q, inp["k_cur"], inp["v_cur"], inp["k_hist"], inp["v_hist"],
+                             anchors, idx)
+    r = np.zeros((N, S, H * d))
+    for i, a in enumerate(anchors):
+        r[a] = linear(np.asarray(O[i], np.float64).reshape(S, H * d), w_o, b_o)
+    mask = np.zeros(N, dtype=np.uint8)
+    mask[anchors] = 1
+    r = par_reconstruct(r.reshape(N, grid[0], grid[1], H * d), mask, None, p)
+    return idx, O, r.reshape(N, S, H * d)

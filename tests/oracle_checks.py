@@ -635,4 +635,70 @@ def check_frame_selection_brute_force():
         assert len(anchors) == Ke and np.all(np.diff(anchors) > 0)
 
 
+
+
+# ----------------------------------------------------------------------------------------------
+# Output projection and anchor FFN
+# ----------------------------------------------------------------------------------------------
+
+def check_gelu_tanh_values():
+    """The tanh form at printed values of 0.5 x (1 + tanh(sqrt(2/pi)(x + 0.044715 x^3))):
+    gelu(1) = 0.8411919906, gelu(-1) = -0.1588080094, gelu(0) = 0, odd-part identity
+    gelu(x) - gelu(-x) = x, and it lies within 1e-3 of the erf form on [-4, 4]."""
+    assert abs(O.gelu_tanh(1.0) - 0.8411919906082768) < 1e-12
+    assert abs(O.gelu_tanh(-1.0) + 0.15880800939172324) < 1e-12
+    assert O.gelu_tanh(0.0) == 0.0
+    x = np.linspace(-6, 6, 101)
+    assert np.allclose(O.gelu_tanh(x) - O.gelu_tanh(-x), x, atol=1e-12)
+    erf_form = 0.5 * x * (1.0 + scipy.special.erf(x / np.sqrt(2.0)))
+    assert np.max(np.abs(O.gelu_tanh(x[np.abs(x) <= 4]) - erf_form[np.abs(x) <= 4])) < 1e-3
+
+
+def check_linear_and_ffn_loops():
+    """linear and anchor_ffn against explicit loops over every output (tiny sizes), reading
+    only the anchor frames."""
+    rng = np.random.default_rng(9)
+    F, S, D, Dff = 4, 3, 5, 7
+    x = rng.standard_normal((F, S, D))
+    w1, b1 = rng.standard_normal((Dff, D)), rng.standard_normal(Dff)
+    w2, b2 = rng.standard_normal((D, Dff)), rng.standard_normal(D)
+    anchors = [0, 2]
+    y = O.anchor_ffn(x, anchors, w1, b1, w2, b2)
+    assert y.shape == (2, S, D)
+    for ia, a in enumerate(anchors):
+        for s in range(S):
+            hid = []
+            for j in range(Dff):
+                acc = b1[j]
+                for c in range(D):
+                    acc += x[a, s, c] * w1[j, c]
+                hid.append(0.5 * acc * (1.0 + math.tanh(math.sqrt(2.0 / math.pi) * (acc + 0.044715 * acc ** 3))))
+            for o in range(D):
+                acc = b2[o]
+                for j in range(Dff):
+                    acc += hid[j] * w2[o, j]
+                assert abs(y[ia, s, o] - acc) < 1e-10
+    wsq = rng.standard_normal((D, D))            # a square weight (W_O): out = x W^T
+    ysq = O.linear(x[0], wsq)
+    for s_ in range(S):
+        for o in range(D):
+            assert abs(ysq[s_, o] - sum(x[0, s_, c] * wsq[o, c] for c in range(D))) < 1e-10
+    x2 = x.copy()
+    x2[1] += 100.0
+    x2[3] -= 7.0                                   # skipped frames are not read
+    assert np.array_equal(O.anchor_ffn(x2, anchors, w1, b1, w2, b2), y)
+
+
+def check_projected_block_step_identity():
+    """With W_O = I and no bias the projected block step equals the plain one (Eq. block)."""
+    from synthetic import workloads as W
+    wl = W.TINY
+    inp = W.block_step_inputs(wl)
+    D = wl.H * wl.d
+    p = O.ParParams(band_radius=wl.band_radius)
+    idx, Oa, r = O.block_step(inp, wl.K, wl.grid, p)
+    _, _, r2 = O.block_step_projected(inp, wl.K, wl.grid, np.eye(D), None, p, idx=idx, O=Oa)
+    assert np.allclose(r, r2, atol=1e-12)
+
+
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

@@ -147,7 +147,26 @@ def _select_ties_high(deltas, ages, anchor_mask, K_f, lam_cov=0.5, eps=1e-8):
     return np.array(sorted(order[:min(K_f, N)])), h, S
 
 
+def _gelu_erf(x):
+    import scipy.special
+    x = np.asarray(x, dtype=np.float64)
+    return 0.5 * x * (1.0 + scipy.special.erf(x / np.sqrt(2.0)))     # the erf form instead
+
+
+def _linear_no_bias(x, w, b=None):
+    return np.asarray(x, np.float64) @ np.asarray(w, np.float64).T
+
+
+def _linear_untransposed_square(x, w, b=None):
+    w = np.asarray(w, np.float64)
+    y = np.asarray(x, np.float64) @ (w if w.shape[0] == w.shape[1] else w.T)
+    return y if b is None else y + b
+
+
 MUTATIONS = {
+    "gelu_erf_form": ("gelu_tanh", _gelu_erf),
+    "linear_bias_dropped": ("linear", _linear_no_bias),
+    "linear_square_untransposed": ("linear", _linear_untransposed_square),
     "norm_measured_from_max": ("minmax_norm", _norm_from_max),
     "single_branch_halved": ("sensitivity", _sens_absent_branch_as_zero),
     "ages_never_reset": ("refresh_ages", _ages_never_reset),
