@@ -283,7 +283,7 @@ def run_gpu(args):
 
 
 # ------------------------------------------------------------------------------ scale points
-SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy", "select_mg")
+SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy", "select_mg", "ffn_mg")
 
 
 def _scale_setup(name, lib, torch, dev):
@@ -339,6 +339,19 @@ def _scale_setup(name, lib, torch, dev):
                          dtype=torch.uint8, device=dev)
         return (lambda: lib.cast_select_frames(deltas, ages, mask, w.K_f, workspace=ws),
                 w.n_branch * w.n_cur * S * w.D * 2, "B")
+    if name == "ffn_mg":
+        wl = W.MG
+        N, S, D = wl.n_cur, wl.S, wl.H * wl.d
+        Dff = 4 * D
+        x = rnd(N, S, D)
+        w1, w2 = rnd(Dff, D) * (D ** -0.5), rnd(D, Dff) * (Dff ** -0.5)
+        b1, b2 = rnd(Dff), rnd(D)
+        r = torch.zeros((N, S, D), dtype=torch.bfloat16, device=dev)
+        an = list(wl.anchors)
+        ws = torch.empty(lib.ffn_workspace_size(x, an, w1, b1, w2, b2, wl.grid, r), dtype=torch.uint8,
+                         device=dev)
+        return (lambda: lib.cast_ffn_step(x, an, w1, b1, w2, b2, wl.grid, r, workspace=ws),
+                4.0 * len(an) * S * D * Dff, "FLOP")
     raise ValueError(name)
 
 

@@ -249,13 +249,50 @@ typedef struct {
   int32_t* idx_out;               /* optional device [n_anchors, H, min(K, M)] */
   const float* channel_weight;    /* optional device [H*d] PAR channel weights */
   cast_par_params par;
+  /* Optional output projection (App. B.1: PAR acts on the site's residual): with w_o the
+     anchor rows of r_out are O_a W_O^T + b_O and PAR reconstructs the skipped rows of that
+     projected residual; NULL = the attention output itself (pre-W_O). */
+  const void* w_o;                /* optional device bf16 [H*d, H*d], layer layout [out, in] */
+  const void* b_o;                /* optional device [H*d] of r_dtype */
 } cast_block_args;
 
-/* route_topk -> anchor_attention -> par_reconstruct on one stream, then the optional
- * residual update x += r_out.  Errors: those of the three steps. */
+/* route_topk -> anchor_attention -> (output projection) -> par_reconstruct on one stream,
+ * then the optional residual update x += r_out.  The projection is a plain GEMM run through
+ * cuBLASLt with the caller's workspace.  Errors: those of the steps; INVALID_ARG for a
+ * misaligned w_o / b_o. */
 cast_status cast_block_step(const cast_block_args* args, void* workspace,
                             size_t workspace_bytes, void* stream);
 size_t cast_block_workspace_size(const cast_block_args* args);
+
+/* ------------------------------------------------------------------------ */
+/* The FFN residual site (App. B.1, B.4): the anchors' FFN is computed, the  */
+/* skipped frames' FFN residuals are reconstructed by PAR with the same      */
+/* anchors.                                                                   */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  const void* x;                  /* device bf16 [n_frames, S, D] FFN input (anchor frames read) */
+  int64_t x_row_stride;           /* elements between token rows, >= D, multiple of 8 */
+  int32_t n_frames, Hg, Wg, D, D_ff;   /* S = Hg * Wg; D and D_ff multiples of 8 */
+  const int32_t* anchors;         /* HOST, strictly ascending, as in cast_block_args */
+  int32_t n_anchors;
+  const void* w1;                 /* device bf16 [D_ff, D] */
+  const void* b1;                 /* optional device bf16 [D_ff] */
+  const void* w2;                 /* device bf16 [D, D_ff] */
+  const void* b2;                 /* optional device [D] of r_dtype */
+  void* r_out;                    /* device [n_frames, S, D]: anchor rows = FFN(x), skipped rows = PAR */
+  int32_t r_dtype;                /* CAST_BF16 or CAST_F32 */
+  const float* channel_weight;    /* optional device [D] PAR channel weights */
+  cast_par_params par;
+} cast_ffn_args;
+
+/* For every anchor frame a: r_out[a] = GELU(x[a] W1^T + b1) W2^T + b2 (GELU in its tanh
+ * form, the hidden activations rounded to bf16 between the two GEMMs), then
+ * par_reconstruct(r_out) over the skipped frames.  The two GEMMs are plain GEMMs run through
+ * cuBLASLt with the caller's workspace.  Errors: INVALID_ARG for bad shapes, strides or
+ * pointers, anchors as in cast_block_step, a short workspace; those of par_reconstruct. */
+cast_status cast_ffn_step(const cast_ffn_args* args, void* workspace, size_t workspace_bytes,
+                          void* stream);
+size_t cast_ffn_workspace_size(const cast_ffn_args* args);
 
 /* ------------------------------------------------------------------------ */
 /* Control-aware frame selection: Section 3 ("Interaction sensitivity",      */

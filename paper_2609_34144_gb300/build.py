@@ -14,7 +14,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libcast.so")
-SOURCES = ["cast_api.cu", "route.cu", "attention.cu", "par.cu", "noalloc.cu", "select.cu"]
+SOURCES = ["cast_api.cu", "route.cu", "attention.cu", "par.cu", "noalloc.cu", "select.cu", "dense.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr", "-Xcompiler", "-fPIC",
          "-Xcompiler", "-fno-strict-aliasing", "-I", os.path.join(ROOT, "include"), "-I", CSRC]
@@ -46,7 +46,9 @@ def build(verbose_ptxas: bool = False, quiet: bool = True) -> str:
                 print(log, file=sys.stderr)
     objs = [o for (o, _) in results]
     tmp = LIB + ".tmp"
-    cmd = [nvcc(), *ARCH, "-shared", "-o", tmp, *objs, "-lrt", "-lpthread", "-ldl"]
+    cuda_lib = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "lib64")
+    cmd = [nvcc(), *ARCH, "-shared", "-o", tmp, *objs, "-L", cuda_lib, "-lcublasLt",
+           "-Xlinker", "-rpath=" + cuda_lib, "-lrt", "-lpthread", "-ldl"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")

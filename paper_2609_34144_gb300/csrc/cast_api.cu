@@ -273,7 +273,7 @@ cast_attn_args attn_of_block(const cast_block_args* a, const int32_t* idx) {
 
 // block-step workspace: [route ws][idx (when idx_out is NULL)][attention ws][par ws]
 struct BlockPlan {
-  size_t route_bytes, idx_bytes, attn_bytes, par_bytes, total;
+  size_t route_bytes, idx_bytes, attn_bytes, par_bytes, proj_bytes, total;
 };
 BlockPlan block_plan(const cast_block_args* a) {
   BlockPlan b{};
@@ -287,7 +287,9 @@ BlockPlan block_plan(const cast_block_args* a) {
   uint8_t mask[CAST_MAX_FRAMES];
   cast_par_args p = par_of_block(a, mask);
   b.par_bytes = par_plan(p).total_bytes;
-  b.total = b.route_bytes + b.idx_bytes + b.attn_bytes + b.par_bytes;
+  // with W_O: the attention output [n_anchors, S, H*d] bf16, then the GEMM scratch
+  b.proj_bytes = a->w_o ? align_up((size_t)a->n_anchors * a->Hg * a->Wg * a->H * a->d * 2) + kGemmWorkspace : 0;
+  b.total = b.route_bytes + b.idx_bytes + b.attn_bytes + b.par_bytes + b.proj_bytes;
   return b;
 }
 
@@ -416,6 +418,9 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
   cast_par_args p = par_of_block(a, mask);
   if ((s = validate_par(&p))) return s;
   if (a->x && !aligned16(a->x)) return fail(CAST_ERR_INVALID_ARG, "%s: x misaligned", who);
+  if (a->w_o && (!aligned16(a->w_o) || (a->b_o && !aligned16(a->b_o))))
+    return fail(CAST_ERR_INVALID_ARG, "%s: w_o / b_o misaligned", who);
+  if (!a->w_o && a->b_o) return fail(CAST_ERR_INVALID_ARG, "%s: b_o given without w_o", who);
   if (ws_bytes < bp.total || (bp.total && !ws))
     return fail(CAST_ERR_INVALID_ARG, "%s: workspace %zu B < %zu B", who, ws_bytes, bp.total);
   if (reinterpret_cast<uintptr_t>(ws) % kWsAlign)
@@ -424,7 +429,36 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
   if (a->M > 0 && a->K > 0) {
     if ((s = launch_route(r, w, st))) return s;
   }
-  if ((s = launch_attention(t, 1, w + bp.route_bytes + bp.idx_bytes, st))) return s;
+  if (!a->w_o) {
+    if ((s = launch_attention(t, 1, w + bp.route_bytes + bp.idx_bytes, st))) return s;
+  } else {
+    // attention output of the anchors into the workspace, then r_out[a] = O_a W_O^T + b_O
+    char* proj = w + bp.route_bytes + bp.idx_bytes + bp.attn_bytes + bp.par_bytes;
+    const int S = a->Hg * a->Wg, D = a->H * a->d;
+    const size_t o_bytes = align_up((size_t)a->n_anchors * S * D * 2);
+    t.o = proj;
+    t.o_dtype = CAST_BF16;
+    if ((s = launch_attention(t, 0, w + bp.route_bytes + bp.idx_bytes, st))) return s;
+    const size_t elt = a->r_dtype == CAST_BF16 ? 2 : 4;
+    for (int i = 0; i < a->n_anchors; ++i) {
+      GemmRows g{};
+      g.a = proj + (size_t)i * S * D * 2;
+      g.lda = D;
+      g.w = a->w_o;
+      g.ldw = D;
+      g.bias = a->b_o;
+      g.c = static_cast<char*>(a->r_out) + (size_t)a->anchors[i] * S * D * elt;
+      g.ldc = D;
+      g.c_dtype = a->r_dtype;
+      g.M = S;
+      g.N = D;
+      g.K = D;
+      g.gelu = false;
+      g.ws = proj + o_bytes;
+      g.ws_bytes = kGemmWorkspace;
+      if ((s = gemm_rows(g, st))) return s;
+    }
+  }
   if (par_plan(p).n_target > 0) {
     if ((s = launch_par(p, w + bp.route_bytes + bp.idx_bytes + bp.attn_bytes, st))) return s;
   }
@@ -432,6 +466,91 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
     const size_t n = (size_t)a->n_frames * a->Hg * a->Wg * a->H * a->d;
     if ((s = launch_residual_add(a->x, a->r_out, a->r_dtype, n, st))) return s;
   }
+  return CAST_OK;
+}
+
+size_t cast_ffn_workspace_size(const cast_ffn_args* a) {
+  if (!a || a->Hg < 1 || a->Wg < 1 || a->D_ff < 1) return 0;
+  return align_up((size_t)a->Hg * a->Wg * a->D_ff * 2) + kGemmWorkspace;
+}
+
+cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, void* stream) {
+  g_detail[0] = 0;
+  const char* who = "cast_ffn_step";
+  if (!a) return fail(CAST_ERR_INVALID_ARG, "%s: args is NULL", who);
+  if (a->n_frames < 1 || a->n_frames > CAST_MAX_FRAMES || a->Hg < 1 || a->Wg < 1 || a->D < 8 ||
+      a->D_ff < 8 || a->D % 8 || a->D_ff % 8)
+    return fail(CAST_ERR_INVALID_ARG, "%s: bad shape (frames %d, grid %dx%d, D %d, D_ff %d)", who,
+                a->n_frames, a->Hg, a->Wg, a->D, a->D_ff);
+  if (a->r_dtype != CAST_BF16 && a->r_dtype != CAST_F32)
+    return fail(CAST_ERR_INVALID_ARG, "%s: r_dtype %d", who, a->r_dtype);
+  cast_status s = validate_anchors(a->anchors, a->n_anchors, a->n_frames, who);
+  if (s) return s;
+  if (!a->x || !aligned16(a->x) || a->x_row_stride < a->D || a->x_row_stride % 8)
+    return fail(CAST_ERR_INVALID_ARG, "%s: x NULL, misaligned or with a bad row stride", who);
+  if (!a->w1 || !a->w2 || !aligned16(a->w1) || !aligned16(a->w2) || (a->b1 && !aligned16(a->b1)) ||
+      (a->b2 && !aligned16(a->b2)))
+    return fail(CAST_ERR_INVALID_ARG, "%s: weights or biases NULL or misaligned", who);
+  uint8_t mask[CAST_MAX_FRAMES];
+  cast_par_args p{};
+  p.r = a->r_out;
+  p.dtype = a->r_dtype;
+  p.F = a->n_frames;
+  p.Hg = a->Hg;
+  p.Wg = a->Wg;
+  p.C = a->D;
+  for (int f = 0; f < a->n_frames; ++f) mask[f] = 0;
+  for (int k = 0; k < a->n_anchors; ++k) mask[a->anchors[k]] = 1;
+  p.anchor_mask = mask;
+  p.channel_weight = a->channel_weight;
+  p.params = a->par;
+  if ((s = validate_par(&p))) return s;
+  const size_t need = cast_ffn_workspace_size(a);
+  if (ws_bytes < need || !ws)
+    return fail(CAST_ERR_INVALID_ARG, "%s: workspace %zu B < %zu B", who, ws_bytes, need);
+  if (reinterpret_cast<uintptr_t>(ws) % kWsAlign)
+    return fail(CAST_ERR_INVALID_ARG, "%s: workspace not 256-byte aligned", who);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int S = a->Hg * a->Wg;
+  char* hid = static_cast<char*>(ws);
+  char* gws = hid + align_up((size_t)S * a->D_ff * 2);
+  const size_t elt = a->r_dtype == CAST_BF16 ? 2 : 4;
+  for (int i = 0; i < a->n_anchors; ++i) {
+    const int f = a->anchors[i];
+    GemmRows g1{};
+    g1.a = static_cast<const char*>(a->x) + (size_t)f * S * a->x_row_stride * 2;
+    g1.lda = a->x_row_stride;
+    g1.w = a->w1;
+    g1.ldw = a->D;
+    g1.bias = a->b1;
+    g1.c = hid;
+    g1.ldc = a->D_ff;
+    g1.c_dtype = CAST_BF16;
+    g1.M = S;
+    g1.N = a->D_ff;
+    g1.K = a->D;
+    g1.gelu = true;
+    g1.ws = gws;
+    g1.ws_bytes = kGemmWorkspace;
+    if ((s = gemm_rows(g1, st))) return s;
+    GemmRows g2{};
+    g2.a = hid;
+    g2.lda = a->D_ff;
+    g2.w = a->w2;
+    g2.ldw = a->D_ff;
+    g2.bias = a->b2;
+    g2.c = static_cast<char*>(a->r_out) + (size_t)f * S * a->D * elt;
+    g2.ldc = a->D;
+    g2.c_dtype = a->r_dtype;
+    g2.M = S;
+    g2.N = a->D;
+    g2.K = a->D_ff;
+    g2.gelu = false;
+    g2.ws = gws;
+    g2.ws_bytes = kGemmWorkspace;
+    if ((s = gemm_rows(g2, st))) return s;
+  }
+  if (par_plan(p).n_target > 0) return launch_par(p, nullptr, st);
   return CAST_OK;
 }
 

@@ -71,6 +71,26 @@ ParPlan par_plan(const cast_par_args& a);
 cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st);
 unsigned int par_error_word(cudaStream_t st, bool clear);
 
+// ------------------------------------------------------------------ dense projections
+constexpr size_t kGemmWorkspace = (size_t)32 << 20;   // cuBLASLt scratch per GEMM call
+// Row-major C[M, N] = act(A[M, K] W[N, K]^T + bias[N]), A and W bf16 (16-byte aligned rows),
+// C and bias of c_dtype; act = GELU (cuBLASLt epilogue) when gelu.
+struct GemmRows {
+  const void* a;
+  int64_t lda;
+  const void* w;
+  int64_t ldw;
+  const void* bias;
+  void* c;
+  int64_t ldc;
+  int c_dtype;
+  int M, N, K;
+  bool gelu;
+  void* ws;
+  size_t ws_bytes;
+};
+cast_status gemm_rows(const GemmRows& g, cudaStream_t st);
+
 // ------------------------------------------------------------------ residual update
 cast_status launch_residual_add(void* x, const void* r, int dtype, size_t n, cudaStream_t st);
 

@@ -69,7 +69,15 @@ class BlockArgs(C.Structure):
                 ("route_mode", _i32), ("route_refine_passes", _i32), ("route_lambda_anc", _f32),
                 ("route_lambda_rec", _f32), ("route_refine_tol", _f32), ("scale", _f32),
                 ("r_out", _vp), ("r_dtype", _i32),
-                ("x", _vp), ("idx_out", _vp), ("channel_weight", _vp), ("par", ParParams)]
+                ("x", _vp), ("idx_out", _vp), ("channel_weight", _vp), ("par", ParParams),
+                ("w_o", _vp), ("b_o", _vp)]
+
+
+class FfnArgs(C.Structure):
+    _fields_ = [("x", _vp), ("x_row_stride", _i64), ("n_frames", _i32), ("Hg", _i32), ("Wg", _i32),
+                ("D", _i32), ("D_ff", _i32), ("anchors", C.POINTER(_i32)), ("n_anchors", _i32),
+                ("w1", _vp), ("b1", _vp), ("w2", _vp), ("b2", _vp), ("r_out", _vp), ("r_dtype", _i32),
+                ("channel_weight", _vp), ("par", ParParams)]
 
 
 class SelectArgs(C.Structure):
@@ -79,6 +87,9 @@ class SelectArgs(C.Structure):
                 ("mask_out", _vp), ("rms_out", _vp), ("score_out", _vp)]
 
 
+_lib.cast_ffn_step.argtypes = [C.POINTER(FfnArgs), _vp, C.c_size_t, _vp]
+_lib.cast_ffn_workspace_size.argtypes = [C.POINTER(FfnArgs)]
+_lib.cast_ffn_workspace_size.restype = C.c_size_t
 _lib.cast_select_frames.argtypes = [C.POINTER(SelectArgs), _vp, C.c_size_t, _vp]
 _lib.cast_select_workspace_size.argtypes = [C.POINTER(SelectArgs)]
 _lib.cast_select_workspace_size.restype = C.c_size_t
@@ -105,7 +116,8 @@ for _f in ("cast_route_topk", "cast_route_topk_noalloc", "cast_anchor_attention"
            "cast_check_device"):
     getattr(_lib, _f).restype = C.c_int
 
-EXPORTED = ["cast_select_frames", "cast_select_workspace_size",
+EXPORTED = ["cast_select_frames", "cast_select_workspace_size", "cast_ffn_step",
+            "cast_ffn_workspace_size",
             "cast_route_topk", "cast_route_workspace_size", "cast_route_topk_noalloc",
             "cast_anchor_attention", "cast_attention_workspace_size",
             "cast_par_reconstruct", "cast_par_workspace_size", "cast_par_params_default",
@@ -326,7 +338,7 @@ def cast_par_reconstruct(r, anchor_mask, channel_weight=None, params=None, works
 # --------------------------------------------------------------------------- block step
 def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None, idx_out=None,
                gram=None, route_eps=1e-8, route_mode=ROUTE_OMISSION, scale=0.0,
-               channel_weight=None, params=None, refine=None):
+               channel_weight=None, params=None, refine=None, w_o=None, b_o=None):
     N, S, H, d = q.shape
     M = k_hist.shape[0]
     a = BlockArgs()
@@ -348,6 +360,7 @@ def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None,
     a.idx_out = _ptr(idx_out)
     a.channel_weight = _ptr(channel_weight)
     a.par = params if params is not None else default_par_params()
+    a.w_o, a.b_o = _ptr(w_o), _ptr(b_o)
     return a
 
 
@@ -427,3 +440,37 @@ def cast_select_frames(deltas, ages, anchor_mask, K_f, lambda_cov=0.5, eps=1e-8,
 
 def select_workspace_size(deltas, ages, anchor_mask, K_f):
     return _lib.cast_select_workspace_size(C.byref(select_args(deltas, ages, anchor_mask, K_f)))
+
+
+# --------------------------------------------------------------------------- FFN site
+def ffn_args(x, anchors, w1, b1, w2, b2, grid, r_out, channel_weight=None, params=None):
+    """x bf16 [F, S, D] (token rows contiguous per frame); w1 bf16 [D_ff, D], w2 bf16 [D, D_ff];
+    b1 bf16 [D_ff] or None; b2 [D] of r_out's dtype or None; r_out [F, S, D] f32 or bf16."""
+    F, S, D = x.shape[0], x.shape[1], x.shape[-1]
+    a = FfnArgs()
+    a.x, a.x_row_stride = _ptr(x), x.stride(1) if x.dim() == 3 else D
+    a.n_frames, a.Hg, a.Wg, a.D, a.D_ff = F, grid[0], grid[1], D, w1.shape[0]
+    a._anchors = _host_i32(anchors)
+    a.anchors = C.cast(a._anchors, C.POINTER(_i32))
+    a.n_anchors = len(anchors)
+    a.w1, a.b1, a.w2, a.b2 = _ptr(w1), _ptr(b1), _ptr(w2), _ptr(b2)
+    a.r_out = _ptr(r_out)
+    a.r_dtype = F32 if r_out.dtype == torch.float32 else BF16
+    a.channel_weight = _ptr(channel_weight)
+    a.par = params if params is not None else default_par_params()
+    return a
+
+
+def cast_ffn_step(x, anchors, w1, b1, w2, b2, grid, r_out, channel_weight=None, params=None,
+                  workspace=None, stream=None):
+    """Anchor FFN residuals into r_out's anchor rows, PAR for the skipped rows."""
+    a = ffn_args(x, anchors, w1, b1, w2, b2, grid, r_out, channel_weight, params)
+    need = _lib.cast_ffn_workspace_size(C.byref(a))
+    ws = workspace if workspace is not None else _workspace(need, x.device)
+    _check(_lib.cast_ffn_step(C.byref(a), _ptr(ws), ws.numel(), _stream(stream)))
+    return r_out
+
+
+def ffn_workspace_size(x, anchors, w1, b1, w2, b2, grid, r_out):
+    return _lib.cast_ffn_workspace_size(C.byref(ffn_args(x, anchors, w1, b1, w2, b2, grid, r_out)))
+

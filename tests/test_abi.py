@@ -193,3 +193,21 @@ def test_select_workspace(lib):
     assert lib.library().cast_select_workspace_size(C.byref(_select(lib, n_branch=0))) == 0
     assert lib.library().cast_select_workspace_size(C.byref(_select(lib))) > 0
 
+
+def test_ffn_validation(lib):
+    a = lib.FfnArgs()
+    a.x, a.x_row_stride = _fake(), 64
+    a.n_frames, a.Hg, a.Wg, a.D, a.D_ff = 3, 4, 4, 64, 256
+    an = (C.c_int32 * 2)(0, 2)
+    a.anchors, a.n_anchors = C.cast(an, C.POINTER(C.c_int32)), 2
+    a.w1, a.w2, a.r_out, a.r_dtype = _fake(0x20000), _fake(0x30000), _fake(0x40000), lib.F32
+    a.par = lib.default_par_params()
+    so = lib.library()
+    need = so.cast_ffn_workspace_size(C.byref(a))
+    assert need > 32 << 20
+    assert so.cast_ffn_step(C.byref(a), _fake(0x100000), need - 1, None) == 1      # short workspace
+    a.D = 60
+    assert so.cast_ffn_step(C.byref(a), _fake(0x100000), need, None) == 1          # D not a multiple of 8
+    a.D, a.w1 = 64, _fake(0x20004)
+    assert so.cast_ffn_step(C.byref(a), _fake(0x100000), need, None) == 1          # misaligned weight
+
