@@ -275,15 +275,15 @@ class Routing:
 
 
 def pooled_routing(q, anchors, k_hist, v_hist, proj=None, eps=1e-8) -> Routing:
-    """q [N, S, H, d]; k_hist, v_hist [M, B_v, H, d]; proj: P = W_O head slices
-    [H, d_out, d] (None: P = I).  Means over tokens pool the statistics."""
+    """q [N, S, H, d]; k_hist, v_hist: the M history blocks, either an array [M, B_v, H, d]
+    or a list of M arrays [n_m, H, d] (blocks of different sizes, e.g. truncated spatial
+    blocks); proj: P = W_O head slices [H, d_out, d] (None: P = I).  Means over a block's
+    tokens pool the statistics."""
     q = np.asarray(q, dtype=np.float64)
-    kh = np.asarray(k_hist, dtype=np.float64)
-    vh = np.asarray(v_hist, dtype=np.float64)
     d = q.shape[-1]
     qbar = np.stack([q[a].mean(axis=0) for a in anchors])          # [K_f, H, d]
-    kbar = kh.mean(axis=1)                                          # [M, H, d]
-    vbar = vh.mean(axis=1)
+    kbar = np.stack([np.asarray(b, dtype=np.float64).mean(axis=0) for b in k_hist])   # [M, H, d]
+    vbar = np.stack([np.asarray(b, dtype=np.float64).mean(axis=0) for b in v_hist])
     s = np.einsum("ihd,mhd->ihm", qbar, kbar) / np.sqrt(d)          # Eq. (pooled)
     e = np.exp(s - s.max(axis=-1, keepdims=True))
     pi = e / e.sum(axis=-1, keepdims=True)
@@ -331,7 +331,8 @@ def topk_margin(score: np.ndarray, K: int) -> np.ndarray:
 def routed_attention(q, k_cur, v_cur, k_hist, v_hist, anchors, idx, scale=None,
                      rows=None, heads=None, with_lse=False):
     """O[i, s, h, :] = sum_j softmax_j(q . k_j * scale) v_j over the current chunk
-    (all N_cur * S tokens) followed by the routed history blocks idx[i, h, :].
+    (all N_cur * S tokens) followed by the routed history blocks idx[i, h, :] (k_hist, v_hist
+    as in pooled_routing: an array of equal blocks or a list of blocks).
 
     Explicit max-subtracted softmax in float64.  `rows` / `heads` restrict the
     query rows / heads computed (others stay NaN)."""
@@ -349,8 +350,8 @@ def routed_attention(q, k_cur, v_cur, k_hist, v_hist, anchors, idx, scale=None,
     for i, a in enumerate(anchors):
         for h in heads:
             blocks = [int(m) for m in idx[i, h]] if idx is not None else []
-            keys = [kc[:, h]] + [np.asarray(k_hist[m, :, h], dtype=np.float64) for m in blocks]
-            vals = [vc[:, h]] + [np.asarray(v_hist[m, :, h], dtype=np.float64) for m in blocks]
+            keys = [kc[:, h]] + [np.asarray(k_hist[m], dtype=np.float64)[:, h] for m in blocks]
+            vals = [vc[:, h]] + [np.asarray(v_hist[m], dtype=np.float64)[:, h] for m in blocks]
             kk = np.concatenate(keys)
             vv = np.concatenate(vals)
             qq = np.asarray(q[a, rows, h], dtype=np.float64)
@@ -632,3 +633,37 @@ def block_step_projected(inp, K, grid, w_o, b_o=None, p: ParParams = ParParams()
     mask[anchors] = 1
     r = par_reconstruct(r.reshape(N, grid[0], grid[1], H * d), mask, None, p)
     return idx, O, r.reshape(N, S, H * d)
+
+
+# ===========================================================================
+# Paper-granularity history blocks (App. C, Tab. config_cast: (1, 8, 8) blocks of 64
+# tokens, K = ceil(0.2 M)); a block never spans frames, edge blocks are truncated
+# ===========================================================================
+
+
+def spatial_blocks(n_frames, Hg, Wg, bh=8, bw=8):
+    """The (1, bh, bw) blocks of n_frames history frames of Hg x Wg tokens: block
+    m = (f * nby + by) * nbx + bx (frame-major, then row-major over the block grid), each a
+    token index array into the frame's row-major Hg * Wg tokens (rows y0..y0+h-1, columns
+    x0..x0+w-1, truncated at the grid edge).  Returns [(frame, tokens), ...]."""
+    nby, nbx = -(-Hg // bh), -(-Wg // bw)
+    out = []
+    for f in range(n_frames):
+        for by in range(nby):
+            for bx in range(nbx):
+                ys = np.arange(by * bh, min(Hg, by * bh + bh))
+                xs = np.arange(bx * bw, min(Wg, bx * bw + bw))
+                out.append((f, (ys[:, None] * Wg + xs[None, :]).reshape(-1)))
+    return out
+
+
+def gather_blocks(frames, blocks):
+    """frames [F_h, Hg * Wg, H, d] -> list of the blocks' token arrays [n_m, H, d]."""
+    fr = np.asarray(frames)
+    return [fr[f, tok] for f, tok in blocks]
+
+
+def paper_budget(M):
+    """K_KV = ceil(0.2 M) (Tab. config_cast)."""
+    return int(-(-2 * M // 10))
+

@@ -701,4 +701,71 @@ def check_projected_block_step_identity():
     assert np.allclose(r, r2, atol=1e-12)
 
 
+
+
+# ----------------------------------------------------------------------------------------------
+# Paper-granularity history blocks: (1, 8, 8) token blocks, partial blocks, K = ceil(0.2 M)
+# ----------------------------------------------------------------------------------------------
+
+def check_spatial_blocks_partition():
+    """Blocks cover every token of every history frame exactly once; full blocks hold 64
+    tokens, edge blocks h x w with h = Hg mod 8 or 8 and w = Wg mod 8 or 8; the count is
+    F * ceil(Hg / 8) * ceil(Wg / 8)."""
+    F, Hg, Wg = 2, 30, 52
+    bl = O.spatial_blocks(F, Hg, Wg)
+    assert len(bl) == F * 4 * 7
+    for f in range(F):
+        toks = np.concatenate([t for g, t in bl if g == f])
+        assert np.array_equal(np.sort(toks), np.arange(Hg * Wg))
+    sizes = sorted({len(t) for _, t in bl})
+    assert sizes == sorted([6 * 4, 6 * 8, 8 * 4, 64])
+    f, t = bl[7 * 3 + 6]                 # frame 0, last block row and column: 6 x 4 tokens
+    assert f == 0 and list(t) == [y * Wg + x for y in range(24, 30) for x in range(48, 52)]
+
+
+def check_spatial_blocks_reduce_to_token_ranges():
+    """With an 8-token-wide history grid a (1, 8, 8) block is 64 consecutive tokens, so routing
+    and attention over the spatial blocks equal the token-range forms with B_v = 64."""
+    rng = np.random.default_rng(13)
+    N, S, H, d = 2, 24, 2, 16
+    Fh, Hg, Wg = 3, 24, 8                 # 3 frames x 3 blocks of 64 tokens
+    q = rng.standard_normal((N, S, H, d))
+    kc, vc = rng.standard_normal((N, S, H, d)), rng.standard_normal((N, S, H, d))
+    kf = rng.standard_normal((Fh, Hg * Wg, H, d))
+    vf = rng.standard_normal((Fh, Hg * Wg, H, d))
+    bl = O.spatial_blocks(Fh, Hg, Wg)
+    kb, vb = O.gather_blocks(kf, bl), O.gather_blocks(vf, bl)
+    krange = kf.reshape(Fh * 3, 64, H, d)
+    vrange = vf.reshape(Fh * 3, 64, H, d)
+    a = O.pooled_routing(q, [0, 1], kb, vb)
+    b = O.pooled_routing(q, [0, 1], krange, vrange)
+    assert np.allclose(a.u, b.u, rtol=1e-12, atol=1e-14)
+    idx = O.topk_blocks(a.u, 4)
+    oa = O.routed_attention(q, kc, vc, kb, vb, [0, 1], idx)
+    ob = O.routed_attention(q, kc, vc, krange, vrange, [0, 1], idx)
+    assert np.allclose(oa, ob, rtol=1e-12, atol=1e-14)
+
+
+def check_partial_block_statistics():
+    """A truncated block pools over its own tokens only (no padding): brute-force means of an
+    edge block; attention over it equals attention over exactly its tokens."""
+    rng = np.random.default_rng(17)
+    Hg, Wg, H, d = 10, 11, 1, 4
+    kf = rng.standard_normal((1, Hg * Wg, H, d))
+    bl = O.spatial_blocks(1, Hg, Wg)
+    f, tok = bl[-1]                      # rows 8..9, columns 8..10: 6 tokens
+    assert len(tok) == 6
+    blk = O.gather_blocks(kf, bl)[-1]
+    ref = np.zeros((H, d))
+    for y in (8, 9):
+        for x in (8, 9, 10):
+            ref += kf[0, y * Wg + x]
+    ref /= 6.0
+    q = rng.standard_normal((1, 3, H, d))
+    r = O.pooled_routing(q, [0], O.gather_blocks(kf, bl), O.gather_blocks(kf, bl))
+    assert np.allclose(r.kbar[-1], ref, atol=1e-14)
+    assert blk.shape[0] == 6
+    assert O.paper_budget(448) == 90 and O.paper_budget(10) == 2 and O.paper_budget(1) == 1
+
+
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

@@ -163,7 +163,26 @@ def _linear_untransposed_square(x, w, b=None):
     return y if b is None else y + b
 
 
+_orig_spatial = O.spatial_blocks
+
+
+def _spatial_blocks_padded(n_frames, Hg, Wg, bh=8, bw=8):
+    # edge blocks padded to full size by repeating their first token (no partial-block mask)
+    out = []
+    for f, tok in _orig_spatial(n_frames, Hg, Wg, bh, bw):
+        if len(tok) < bh * bw:
+            tok = np.concatenate([tok, np.full(bh * bw - len(tok), tok[0])])
+        out.append((f, tok))
+    return out
+
+
+def _budget_floor(M):
+    return int(2 * M // 10)
+
+
 MUTATIONS = {
+    "partial_blocks_padded": ("spatial_blocks", _spatial_blocks_padded),
+    "budget_floor": ("paper_budget", _budget_floor),
     "gelu_erf_form": ("gelu_tanh", _gelu_erf),
     "linear_bias_dropped": ("linear", _linear_no_bias),
     "linear_square_untransposed": ("linear", _linear_untransposed_square),
