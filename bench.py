@@ -283,7 +283,17 @@ def run_gpu(args):
 
 
 # ------------------------------------------------------------------------------ scale points
-SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy", "select_mg", "ffn_mg")
+SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy", "select_mg", "ffn_mg",
+                "route_mg64", "attn_mg64", "attn_hy64", "block_mg64")
+
+
+def _block_tokens(wl):
+    """Tokens of each (1, 8, 8) block of the workload's history frames (edge blocks truncated)."""
+    hg, wg = wl.grid
+    ys = [min(8, hg - 8 * by) for by in range(-(-hg // 8))]
+    xs = [min(8, wg - 8 * bx) for bx in range(-(-wg // 8))]
+    per_frame = [h * w for h in ys for w in xs]
+    return per_frame * wl.hist_frames
 
 
 def _scale_setup(name, lib, torch, dev):
@@ -352,6 +362,34 @@ def _scale_setup(name, lib, torch, dev):
                          device=dev)
         return (lambda: lib.cast_ffn_step(x, an, w1, b1, w2, b2, wl.grid, r, workspace=ws),
                 4.0 * len(an) * S * D * Dff, "FLOP")
+    if name in ("route_mg64", "attn_mg64", "attn_hy64", "block_mg64"):
+        wl = W.HY64 if name == "attn_hy64" else W.MG64
+        N, S, H, d = wl.n_cur, wl.S, wl.H, wl.d
+        an = list(wl.anchors)
+        Kf = len(an)
+        hist = (wl.hist_frames, wl.grid[0], wl.grid[1], H, d)
+        q, kc, vc = rnd(N, S, H, d), rnd(N, S, H, d), rnd(N, S, H, d)
+        kh, vh = rnd(*hist), rnd(*hist)
+        if name == "route_mg64":
+            ws = torch.empty(lib.route_workspace_size(q, an, kh, vh, wl.K), dtype=torch.uint8, device=dev)
+            return (lambda: lib.cast_route_topk(q, an, kh, vh, wl.K, workspace=ws),
+                    (Kf * S + 2 * wl.hist_frames * S) * H * d * 2, "B")
+        if name == "block_mg64":
+            r = torch.zeros((N, S, H * d), dtype=torch.bfloat16, device=dev)
+            a = lib.block_args(q, kc, vc, an, kh, vh, wl.K, wl.grid, r, refine=lib.REFINE_PAPER)
+            ws = torch.empty(lib.block_workspace_size(a), dtype=torch.uint8, device=dev)
+            return (lambda: lib.cast_block_step_args(a, ws), N, "frames")
+        perm = torch.stack([torch.randperm(wl.M, generator=torch.Generator().manual_seed(k))[:wl.K]
+                            for k in range(Kf * H)]).view(Kf, H, wl.K)
+        sizes = torch.tensor(_block_tokens(wl), dtype=torch.float64)
+        routed_tokens = float(sizes[perm].sum())          # keys of the routed blocks, all (i, h)
+        flop = 4.0 * S * d * (Kf * H * N * S + routed_tokens)
+        idx = perm.int().to(dev)
+        o = torch.empty((Kf, S, H * d), dtype=torch.bfloat16, device=dev)
+        aws = torch.empty(max(lib.attention_workspace_size(q, kc, vc, an, kh, vh, idx), 256),
+                          dtype=torch.uint8, device=dev)
+        return (lambda: lib.cast_anchor_attention(q, kc, vc, an, kh, vh, idx, out=o, workspace=aws),
+                flop, "FLOP")
     raise ValueError(name)
 
 
@@ -378,6 +416,8 @@ def scale_points(lib, torch, dev, flush, reps=10):
             rate = work / ms / 1e6
             out[name] = {"ms": round(ms, 4), "GB/s": round(rate, 1), "frac_hbm": round(rate / hbm, 4),
                          "bytes": work}
+        elif unit == "frames":
+            out[name] = {"ms": round(ms, 4), "frames/s": round(work / ms * 1e3, 1)}
         else:
             rate = work / ms / 1e9
             out[name] = {"ms": round(ms, 4), "TFLOP/s": round(rate, 1),

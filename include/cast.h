@@ -69,6 +69,24 @@ typedef int cast_status;
 #define CAST_MAX_ANCHORS 64
 
 /* ------------------------------------------------------------------------ */
+/* Layout of the historical KV blocks (Section 4.4; App. B.5 Tab. config:    */
+/* blocks (t, h, w) = (1, 8, 8) in token coordinates, partial blocks masked). */
+/* ------------------------------------------------------------------------ */
+#define CAST_HIST_BLOCKS 0        /* k_hist/v_hist [M, B_v, H, d]: block m = rows m*B_v .. m*B_v+B_v-1 */
+#define CAST_HIST_FRAMES 1        /* k_hist/v_hist [frames, Hg, Wg, H, d]: (1, 8, 8) blocks */
+
+typedef struct {
+  int32_t kind;                   /* CAST_HIST_BLOCKS (zero-initialised default) or CAST_HIST_FRAMES */
+  /* CAST_HIST_FRAMES only: the history frames and their token grid.  Block
+     m = (f * ceil(Hg/8) + by) * ceil(Wg/8) + bx holds the tokens of frame f in rows
+     8by .. min(8by+8, Hg)-1 and columns 8bx .. min(8bx+8, Wg)-1 (a block never spans frames;
+     blocks at the right and bottom edges are truncated).  M must equal
+     frames * ceil(Hg/8) * ceil(Wg/8) and B_v must be 64 (the nominal block size); a truncated
+     block pools over its own tokens and its missing key positions are masked in attention. */
+  int32_t frames, Hg, Wg;
+} cast_hist_layout;
+
+/* ------------------------------------------------------------------------ */
 /* Routing: Section 4.4, Eqs. (pooled), (omission), (topk); App. B.1.        */
 /* ------------------------------------------------------------------------ */
 typedef struct {
@@ -79,7 +97,8 @@ typedef struct {
   int32_t dtype;                  /* dtype of q, k_hist, v_hist: CAST_BF16 or CAST_F32 */
   const int32_t* anchors;         /* HOST, n_anchors strictly ascending frame indices */
   int32_t n_anchors;
-  /* history blocks, [M, B_v, H, d]: block m is rows m*B_v .. m*B_v+B_v-1 */
+  /* history blocks, [M, B_v, H, d] (block m is rows m*B_v .. m*B_v+B_v-1), or history frames
+     in (1, 8, 8) blocks as given by hist */
   const void* k_hist;
   const void* v_hist;
   int64_t hist_row_stride;
@@ -104,6 +123,7 @@ typedef struct {
      2 passes, (1, 1), 1e-6.  0 passes = independent TopK.  Needs CAST_ROUTE_OMISSION. */
   int32_t refine_passes;
   float lambda_anc, lambda_rec, refine_tol;
+  cast_hist_layout hist;          /* layout of k_hist/v_hist; zero = CAST_HIST_BLOCKS */
 } cast_route_args;
 
 /* Pooled mean statistics q_bar, k_bar, v_bar (mean over a frame's S tokens and over a
@@ -112,8 +132,12 @@ typedef struct {
  * u = delta^T G delta; then per (anchor, head) the K_eff largest scores (ties to the
  * lower block index), written in ascending block order.  K >= M keeps every block and
  * M == 0 writes nothing (routing bypass, App. B.3).
+ * With CAST_HIST_FRAMES a block's means run over its own tokens (64, or fewer at the grid
+ * edge).
  * Errors: INVALID_ARG for NULL required pointers, n_anchors < 1 or > CAST_MAX_ANCHORS,
  * anchors not ascending / out of range, K < 0, M < 0, B_v < 1 with M > 0, bad strides,
+ * an unknown hist.kind, or CAST_HIST_FRAMES with a non-positive grid, M different from its
+ * block count or B_v != 64,
  * a workspace smaller than cast_route_workspace_size(), refinement with a negative weight or
  * tolerance or outside CAST_ROUTE_OMISSION; UNSUPPORTED for d not 64/128, M > 16384,
  * H*d > 51200 channels (pooling shared memory) or 4*(2*K_f*d + 3*K_f*M + M + 8*d) bytes of
@@ -149,7 +173,7 @@ typedef struct {
   int32_t n_frames, S, H, d;      /* d in {64, 128} */
   const int32_t* anchors;         /* HOST, strictly ascending */
   int32_t n_anchors;
-  const void* k_hist;             /* bf16 [M, B_v, H, d] */
+  const void* k_hist;             /* bf16 [M, B_v, H, d], or frames as given by hist */
   const void* v_hist;
   int64_t hist_row_stride;
   int32_t M, B_v;
@@ -160,6 +184,7 @@ typedef struct {
   int32_t o_dtype;                /* CAST_BF16 or CAST_F32 */
   float* lse;                     /* optional device f32 [n_anchors, H, S]: natural-log
                                      log-sum-exp of the scaled logits of each query row */
+  cast_hist_layout hist;          /* layout of k_hist/v_hist; zero = CAST_HIST_BLOCKS */
 } cast_attn_args;
 
 /* O[i, s, h, :] = sum_j softmax_j(scale * q_i,s,h . k_j) v_j, where j runs over every
@@ -168,9 +193,13 @@ typedef struct {
  * The workspace (cast_attention_workspace_size() bytes; 0 and NULL allowed when that is 0)
  * holds the partial results of query tiles whose keys are split over several SMs to fill the
  * last round of work.
+ * With CAST_HIST_FRAMES the routed blocks are taken two at a time (two 8x8 token boxes per
+ * 128-key tile); key positions outside a truncated block, and the empty second half of the
+ * last tile when K_eff is odd, are masked (-inf logits).
  * Errors: INVALID_ARG for NULL pointers, bad shapes or strides, anchors not ascending,
- * K_eff > 0 with M == 0, a short workspace; UNSUPPORTED for d not 64/128 or
- * S*n_frames >= 2^31.  Block indices outside [0, M) make the kernel record an error and
+ * K_eff > 0 with M == 0, a short workspace, a history layout as in cast_route_topk;
+ * UNSUPPORTED for d not 64/128, S*n_frames >= 2^31, or CAST_HIST_FRAMES with
+ * frames * Hg * Wg >= 2^31 tokens.  Block indices outside [0, M) make the kernel record an error and
  * read block 0 instead. */
 cast_status cast_anchor_attention(const cast_attn_args* args, void* workspace,
                                   size_t workspace_bytes, void* stream);
@@ -231,7 +260,7 @@ typedef struct {
   const int32_t* anchors;         /* HOST, strictly ascending; n_anchors >= 2 unless
                                      every frame is an anchor */
   int32_t n_anchors;
-  const void* k_hist;             /* bf16 [M, B_v, H, d] */
+  const void* k_hist;             /* bf16 [M, B_v, H, d], or frames as given by hist */
   const void* v_hist;
   int64_t hist_row_stride;
   int32_t M, B_v;
@@ -254,6 +283,7 @@ typedef struct {
      projected residual; NULL = the attention output itself (pre-W_O). */
   const void* w_o;                /* optional device bf16 [H*d, H*d], layer layout [out, in] */
   const void* b_o;                /* optional device [H*d] of r_dtype */
+  cast_hist_layout hist;          /* layout of k_hist/v_hist; zero = CAST_HIST_BLOCKS */
 } cast_block_args;
 
 /* route_topk -> anchor_attention -> (output projection) -> par_reconstruct on one stream,

@@ -10,7 +10,10 @@
 //   warp 0       TMA producers: lane 0 loads Q0/Q1 and the K tiles, lane 1 the V tiles, each
 //                into a two-stage ring (128 tokens x d, 128-byte swizzle, 64-element boxes);
 //                current-chunk tiles come from a 2-D map, history tiles from a 3-D map
-//                [block, token, channel] so a tile never reads past its block.
+//                [block, token, channel] so a tile never reads past its block, or, with
+//                (1, 8, 8) spatial blocks of history frames, from a 4-D map
+//                [frame, y, x, channel] whose 8 x 8-token boxes put two routed blocks in one
+//                tile (rows 0-63 and 64-127; grid-edge tokens read as zero and are masked).
 //   warp 1       TMEM owner and single-thread UMMA issuer, order
 //                S0_0 S1_0 | PV0_0 S0_1 PV1_0 S1_1 | PV0_1 S0_2 PV1_1 S1_2 | ...
 //                (S_t = Q_t K^T, kind::f16, M=N=128, f32 in TMEM; PV_t: O_t += P_t V with P_t
@@ -65,6 +68,8 @@ struct Cfg {
 
 struct AttnKArgs {
   int S, H, n_pairs, n_single, n_anchors, n_cur_tiles, tiles_per_block, K_eff, M, cur_rows, B_v;
+  int n_hist_tiles;                 // history K/V tiles
+  int spatial, hHg, hWg, nby, nbx;  // CAST_HIST_FRAMES: frame grid, 8x8 block grid
   int n_full;        // units run whole (CTAs 0 .. n_full-1)
   int n_split;       // parts of every remaining unit
   int chunk;         // K/V tiles per part
@@ -117,26 +122,62 @@ __device__ __forceinline__ void set_abort(Bars* b) {
   atomicExch(&g_attn_error, 1u);
 }
 
-// (tensor map, row, block) of K/V tile j: current-chunk tiles first, then the routed blocks
+// Routed block k of (anchor i, head h); an index outside [0, M) records an error and reads 0.
+__device__ __forceinline__ int routed_block(const AttnKArgs& a, int i, int h, int k) {
+  int m = __ldg(a.idx + ((int64_t)i * a.H + h) * a.K_eff + k);
+  if (m < 0 || m >= a.M) {
+    atomicExch(&g_attn_error, 2u);
+    m = 0;
+  }
+  return m;
+}
+
+// Spatial block m: (frame, first row, first column) in the history frames and the mask of its
+// 64 key positions (bit 8 yl + xl set iff row yl, column xl lie inside the frame grid).
+struct SpatialBlock {
+  int f, y0, x0;
+  uint64_t valid;
+};
+__device__ __forceinline__ SpatialBlock spatial_block(const AttnKArgs& a, int m) {
+  SpatialBlock b;
+  const int per_frame = a.nby * a.nbx;
+  b.f = m / per_frame;
+  const int rem = m - b.f * per_frame;
+  const int by = rem / a.nbx, bx = rem - by * a.nbx;
+  b.y0 = 8 * by;
+  b.x0 = 8 * bx;
+  const int hv = min(8, a.hHg - b.y0), wv = min(8, a.hWg - b.x0);
+  const uint64_t row = (1ull << wv) - 1ull;                 // columns 0 .. wv-1 of one row
+  const uint64_t rows = row * 0x0101010101010101ull;        // ... of every row
+  b.valid = hv >= 8 ? rows : rows & ((1ull << (8 * hv)) - 1ull);
+  return b;
+}
+
+// (tensor map, row, block) of K/V tile j: current-chunk tiles first, then the routed blocks.
+// Spatial history: tile jj holds routed blocks 2jj (rows 0-63) and 2jj+1 (rows 64-127); when
+// K_eff is odd the last tile repeats block 2jj in its second half, which is masked.
 struct TileCoord {
   bool cur;
   int y, z;
+  int m0, m1;   // spatial: the two blocks
 };
 __device__ __forceinline__ TileCoord tile_coord(const AttnKArgs& a, int i, int h, int j) {
   TileCoord c;
   c.cur = j < a.n_cur_tiles;
+  c.m0 = c.m1 = 0;
   if (c.cur) {
     c.y = j * BN;
     c.z = 0;
+  } else if (a.spatial) {
+    const int jj = j - a.n_cur_tiles;
+    c.y = c.z = 0;
+    c.m0 = routed_block(a, i, h, 2 * jj);
+    c.m1 = 2 * jj + 1 < a.K_eff ? routed_block(a, i, h, 2 * jj + 1) : c.m0;
   } else {
     const int jj = j - a.n_cur_tiles;
     const int blk = jj / a.tiles_per_block;
     c.y = (jj - blk * a.tiles_per_block) * BN;
-    c.z = a.idx[((int64_t)i * a.H + h) * a.K_eff + blk];
-    if (c.z < 0 || c.z >= a.M) {
-      atomicExch(&g_attn_error, 2u);
-      c.z = 0;
-    }
+    c.z = routed_block(a, i, h, blk);
   }
   return c;
 }
@@ -160,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // first: every pair of query tiles, then the single remainder tiles (S mod 256 <= 128).
   // Head slowest within each group: CTAs resident together share the head's current-chunk
   // K/V in L2.
-  const int n_tiles_all = a.n_cur_tiles + a.K_eff * a.tiles_per_block;
+  const int n_tiles_all = a.n_cur_tiles + a.n_hist_tiles;
   int u, part = 0, k0 = 0, k1 = n_tiles_all;
   const bool split = (int)blockIdx.x >= a.n_full;
   if (!split) {
@@ -239,11 +280,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         mbar_arrive_expect_tx(&bars->k_full[s], C::KV_BYTES);
+        if (!c.cur && a.spatial) {
+          const SpatialBlock b0 = spatial_block(a, c.m0), b1 = spatial_block(a, c.m1);
 #pragma unroll
-        for (int b = 0; b < HD / 64; ++b) {
-          uint8_t* dst = sK + s * C::KV_BYTES + b * BN * 128;
-          if (c.cur) tma_load_2d(dst, &tm_kc, &bars->k_full[s], h * HD + b * 64, c.y);
-          else tma_load_3d(dst, &tm_kh, &bars->k_full[s], h * HD + b * 64, c.y, c.z);
+          for (int b = 0; b < HD / 64; ++b) {
+            uint8_t* dst = sK + s * C::KV_BYTES + b * BN * 128;
+            tma_load_4d(dst, &tm_kh, &bars->k_full[s], h * HD + b * 64, b0.x0, b0.y0, b0.f);
+            tma_load_4d(dst + 64 * 128, &tm_kh, &bars->k_full[s], h * HD + b * 64, b1.x0, b1.y0, b1.f);
+          }
+        } else {
+#pragma unroll
+          for (int b = 0; b < HD / 64; ++b) {
+            uint8_t* dst = sK + s * C::KV_BYTES + b * BN * 128;
+            if (c.cur) tma_load_2d(dst, &tm_kc, &bars->k_full[s], h * HD + b * 64, c.y);
+            else tma_load_3d(dst, &tm_kh, &bars->k_full[s], h * HD + b * 64, c.y, c.z);
+          }
         }
       }
     } else if (lane == 1) {
@@ -257,11 +308,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         mbar_arrive_expect_tx(&bars->v_full[s], C::KV_BYTES);
+        if (!c.cur && a.spatial) {
+          const SpatialBlock b0 = spatial_block(a, c.m0), b1 = spatial_block(a, c.m1);
 #pragma unroll
-        for (int b = 0; b < HD / 64; ++b) {
-          uint8_t* dst = sV + s * C::KV_BYTES + b * BN * 128;
-          if (c.cur) tma_load_2d(dst, &tm_vc, &bars->v_full[s], h * HD + b * 64, c.y);
-          else tma_load_3d(dst, &tm_vh, &bars->v_full[s], h * HD + b * 64, c.y, c.z);
+          for (int b = 0; b < HD / 64; ++b) {
+            uint8_t* dst = sV + s * C::KV_BYTES + b * BN * 128;
+            tma_load_4d(dst, &tm_vh, &bars->v_full[s], h * HD + b * 64, b0.x0, b0.y0, b0.f);
+            tma_load_4d(dst + 64 * 128, &tm_vh, &bars->v_full[s], h * HD + b * 64, b1.x0, b1.y0, b1.f);
+          }
+        } else {
+#pragma unroll
+          for (int b = 0; b < HD / 64; ++b) {
+            uint8_t* dst = sV + s * C::KV_BYTES + b * BN * 128;
+            if (c.cur) tma_load_2d(dst, &tm_vc, &bars->v_full[s], h * HD + b * 64, c.y);
+            else tma_load_3d(dst, &tm_vh, &bars->v_full[s], h * HD + b * 64, c.y, c.z);
+          }
         }
       }
     }
@@ -351,25 +412,44 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
+      const int jg = k0 + j;   // global K/V tile
+      // spatial history tile: the routed block indices are fetched before the wait
+      int sm0 = -1, sm1 = -1;
+      if (a.spatial && jg >= a.n_cur_tiles) {
+        const int jj = jg - a.n_cur_tiles;
+        sm0 = routed_block(a, i, h, 2 * jj);
+        sm1 = 2 * jj + 1 < a.K_eff ? routed_block(a, i, h, 2 * jj + 1) : -1;
+      }
       bool w = !aborted(bars) && mbar_wait(&bars->s_full[t], (uint32_t)j & 1u, lim);
       if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
       tc_fence_after();
       uint32_t sr[BN];
       tmem_ld_x64(tl + colS, sr);
       tmem_ld_x64(tl + colS + 64, sr + 64);
-      int valid;
-      const int jg = k0 + j;   // global K/V tile
-      if (jg < a.n_cur_tiles) {
-        valid = min(BN, a.cur_rows - jg * BN);
-      } else {
-        const int jj = jg - a.n_cur_tiles;
-        valid = min(BN, a.B_v - (jj % a.tiles_per_block) * BN);
-      }
-      // columns past the chunk / block end (only in a ragged last tile) get -inf
-      if (valid < BN) {
+      if (sm0 >= 0) {
+        // key positions outside a truncated block, and the unused half of a last odd tile
+        const uint64_t v0 = spatial_block(a, sm0).valid;
+        const uint64_t v1 = sm1 >= 0 ? spatial_block(a, sm1).valid : 0ull;
+        if ((v0 & v1) != ~0ull) {
+          const uint32_t w4[4] = {(uint32_t)v0, (uint32_t)(v0 >> 32), (uint32_t)v1, (uint32_t)(v1 >> 32)};
 #pragma unroll
-        for (int c = 0; c < BN; ++c)
-          if (c >= valid) sr[c] = __float_as_uint(-INFINITY);
+          for (int c = 0; c < BN; ++c)
+            if (!((w4[c >> 5] >> (c & 31)) & 1u)) sr[c] = __float_as_uint(-INFINITY);
+        }
+      } else {
+        int valid;
+        if (jg < a.n_cur_tiles) {
+          valid = min(BN, a.cur_rows - jg * BN);
+        } else {
+          const int jj = jg - a.n_cur_tiles;
+          valid = min(BN, a.B_v - (jj % a.tiles_per_block) * BN);
+        }
+        // columns past the chunk / block end (only in a ragged last tile) get -inf
+        if (valid < BN) {
+#pragma unroll
+          for (int c = 0; c < BN; ++c)
+            if (c >= valid) sr[c] = __float_as_uint(-INFINITY);
+        }
       }
       // raw-logit max (scale > 0 commutes with max): 3-input max, 8 independent chains
       float m8[8];
@@ -554,6 +634,21 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// bf16 history frames [frames][Hg][Wg][inner], box 64 channels x 8 x 8 tokens x 1 frame
+// (one (1, 8, 8) block), 128-B swizzle; tokens outside the grid read as zero
+bool make_map_frames(CUtensorMap* m, const void* base, uint64_t inner, uint64_t Wg, uint64_t Hg,
+                     uint64_t frames, uint64_t row_stride_bytes) {
+  EncodeTiledFn fn = tensor_map_encoder();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {inner, Wg, Hg, frames};
+  cuuint64_t strides[3] = {row_stride_bytes, row_stride_bytes * Wg, row_stride_bytes * Wg * Hg};
+  cuuint32_t box[4] = {64, 8, 8, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int HD>
 cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_of_anchor, void* ws,
                       cudaStream_t st) {
@@ -564,7 +659,11 @@ cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_o
   bool ok = make_map(&mq, a.q, D, a.S, a.q_row_stride * 2, a.n_frames, (uint64_t)a.S * a.q_row_stride * 2) &&
             make_map(&mkc, a.k_cur, D, cur_rows, a.cur_row_stride * 2, 0, 0) &&
             make_map(&mvc, a.v_cur, D, cur_rows, a.cur_row_stride * 2, 0, 0);
-  if (ok && a.M > 0) {
+  const HistGeom hg = hist_geom(a.hist);
+  if (ok && a.M > 0 && hg.spatial) {
+    ok = make_map_frames(&mkh, a.k_hist, D, hg.Wg, hg.Hg, hg.frames, a.hist_row_stride * 2) &&
+         make_map_frames(&mvh, a.v_hist, D, hg.Wg, hg.Hg, hg.frames, a.hist_row_stride * 2);
+  } else if (ok && a.M > 0) {
     ok = make_map(&mkh, a.k_hist, D, a.B_v, a.hist_row_stride * 2, a.M,
                   (uint64_t)a.B_v * a.hist_row_stride * 2) &&
          make_map(&mvh, a.v_hist, D, a.B_v, a.hist_row_stride * 2, a.M,
@@ -582,6 +681,12 @@ cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_o
   k.n_anchors = a.n_anchors;
   k.n_cur_tiles = pl.n_cur_tiles;
   k.tiles_per_block = pl.tiles_per_block;
+  k.n_hist_tiles = pl.n_hist_tiles;
+  k.spatial = hg.spatial ? 1 : 0;
+  k.hHg = hg.Hg;
+  k.hWg = hg.Wg;
+  k.nby = hg.nby;
+  k.nbx = hg.nbx;
   k.K_eff = a.M > 0 ? a.K_eff : 0;
   k.M = a.M;
   k.cur_rows = (int)cur_rows;
@@ -633,7 +738,9 @@ AttnPlan attention_plan(const cast_attn_args& a) {
   p.n_single = (a.S % (2 * BM) > 0 && a.S % (2 * BM) <= BM) ? 1 : 0;
   p.n_cur_tiles = (int)(((int64_t)a.n_frames * a.S + BN - 1) / BN);
   p.tiles_per_block = a.M > 0 ? (a.B_v + BN - 1) / BN : 0;
-  const int n_tiles = p.n_cur_tiles + (a.M > 0 ? a.K_eff : 0) * p.tiles_per_block;
+  const int keff = a.M > 0 ? a.K_eff : 0;
+  p.n_hist_tiles = hist_geom(a.hist).spatial ? (keff + 1) / 2 : keff * p.tiles_per_block;
+  const int n_tiles = p.n_cur_tiles + p.n_hist_tiles;
   const int units = (p.n_pairs + p.n_single) * a.n_anchors * a.H;
   int dev = 0, nsm = 148;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);

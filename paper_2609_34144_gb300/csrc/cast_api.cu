@@ -99,6 +99,26 @@ cast_status validate_tokens(const void* p, int64_t row_stride, int H, int d, con
   return CAST_OK;
 }
 
+// History layout (App. B.5 Tab. config): CAST_HIST_FRAMES needs a positive grid, M equal to
+// its (1, 8, 8) block count and the nominal block size B_v = 64.
+cast_status validate_hist(const cast_hist_layout& h, int M, int B_v, const char* who) {
+  if (h.kind == CAST_HIST_BLOCKS) return CAST_OK;
+  if (h.kind != CAST_HIST_FRAMES) return fail(CAST_ERR_INVALID_ARG, "%s: hist.kind %d", who, h.kind);
+  if (h.frames < 1 || h.Hg < 1 || h.Wg < 1)
+    return fail(CAST_ERR_INVALID_ARG, "%s: history grid %d x %d x %d must be positive", who, h.frames,
+                h.Hg, h.Wg);
+  if ((int64_t)h.frames * h.Hg * h.Wg >= (1LL << 31))
+    return fail(CAST_ERR_UNSUPPORTED, "%s: history of %lld tokens", who,
+                (long long)h.frames * h.Hg * h.Wg);
+  const HistGeom g = hist_geom(h);
+  if (g.blocks() != M)
+    return fail(CAST_ERR_INVALID_ARG, "%s: M=%d but the history frames hold %lld (1,8,8) blocks", who, M,
+                (long long)g.blocks());
+  if (B_v != kSpatialBlock * kSpatialBlock)
+    return fail(CAST_ERR_INVALID_ARG, "%s: B_v=%d with (1,8,8) blocks (must be 64)", who, B_v);
+  return CAST_OK;
+}
+
 cast_status validate_route(const cast_route_args* a) {
   const char* who = "cast_route_topk";
   if (!a) return fail(CAST_ERR_INVALID_ARG, "%s: args is NULL", who);
@@ -112,6 +132,7 @@ cast_status validate_route(const cast_route_args* a) {
   if (a->M > 16384) return fail(CAST_ERR_UNSUPPORTED, "%s: M=%d above 16384", who, a->M);
   cast_status s = validate_anchors(a->anchors, a->n_anchors, a->n_frames, who);
   if (s) return s;
+  if ((s = validate_hist(a->hist, a->M, a->B_v, who))) return s;
   s = validate_tokens(a->q, a->q_row_stride, a->H, a->d, "q", who);
   if (s) return s;
   if (a->M > 0) {
@@ -155,6 +176,7 @@ cast_status validate_attn(const cast_attn_args* a) {
   if (a->M > 0 && a->B_v < 1) return fail(CAST_ERR_INVALID_ARG, "%s: B_v must be >= 1", who);
   cast_status s = validate_anchors(a->anchors, a->n_anchors, a->n_frames, who);
   if (s) return s;
+  if ((s = validate_hist(a->hist, a->M, a->B_v, who))) return s;
   if ((s = validate_tokens(a->q, a->q_row_stride, a->H, a->d, "q", who))) return s;
   if ((s = validate_tokens(a->k_cur, a->cur_row_stride, a->H, a->d, "k_cur", who))) return s;
   if ((s = validate_tokens(a->v_cur, a->cur_row_stride, a->H, a->d, "v_cur", who))) return s;
@@ -240,6 +262,7 @@ cast_route_args route_of_block(const cast_block_args* a, int32_t* idx) {
   r.lambda_anc = a->route_lambda_anc;
   r.lambda_rec = a->route_lambda_rec;
   r.refine_tol = a->route_refine_tol;
+  r.hist = a->hist;
   r.idx = idx;
   return r;
 }
@@ -268,6 +291,7 @@ cast_attn_args attn_of_block(const cast_block_args* a, const int32_t* idx) {
   t.o = a->r_out;
   t.o_dtype = a->r_dtype;
   t.lse = nullptr;
+  t.hist = a->hist;
   return t;
 }
 

@@ -28,6 +28,27 @@ EncodeTiledFn tensor_map_encoder();
 constexpr size_t kWsAlign = 256;
 inline size_t align_up(size_t x, size_t a = kWsAlign) { return (x + a - 1) / a * a; }
 
+// ------------------------------------------------------------------ history layout
+// Geometry of CAST_HIST_FRAMES: (1, 8, 8) blocks over frames of an Hg x Wg token grid.
+constexpr int kSpatialBlock = 8;
+struct HistGeom {
+  bool spatial;
+  int frames, Hg, Wg, nby, nbx;   // nby x nbx blocks per frame
+  int64_t blocks() const { return (int64_t)frames * nby * nbx; }
+};
+inline HistGeom hist_geom(const cast_hist_layout& h) {
+  HistGeom g{};
+  g.spatial = h.kind == CAST_HIST_FRAMES;
+  if (g.spatial) {
+    g.frames = h.frames;
+    g.Hg = h.Hg;
+    g.Wg = h.Wg;
+    g.nby = h.Hg > 0 ? (h.Hg + kSpatialBlock - 1) / kSpatialBlock : 0;
+    g.nbx = h.Wg > 0 ? (h.Wg + kSpatialBlock - 1) / kSpatialBlock : 0;
+  }
+  return g;
+}
+
 // ------------------------------------------------------------------ routing
 struct RoutePlan {
   int n_seg;        // n_anchors + 2 M pooled segments
@@ -45,6 +66,7 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st);
 // ------------------------------------------------------------------ attention
 struct AttnPlan {
   int n_pairs, n_single, n_cur_tiles, tiles_per_block;
+  int n_hist_tiles;   // K/V tiles of the routed history (two (1,8,8) blocks per tile when spatial)
   int n_full, n_tail, n_split, chunk, grid;
   size_t part_o_bytes, part_ml_bytes, counter_bytes, total_bytes;
 };

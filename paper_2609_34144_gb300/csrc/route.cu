@@ -49,6 +49,7 @@ struct PoolArgs {
   float* vbar;            // [M, D]
   int64_t q_row_stride, hist_row_stride;   // elements
   int n_anchors, M, S, B_v, D, nsplit, elt;
+  int Hg, Wg, nby, nbx;   // CAST_HIST_FRAMES: history frame grid and its 8x8 block grid
   int anchors[CAST_MAX_ANCHORS];
 };
 
@@ -92,8 +93,10 @@ __device__ __forceinline__ void launch_dependents() {
 }
 
 // grid (nsplit, n_seg), cluster (nsplit, 1, 1), cgs * lanes_r threads.  Dynamic smem:
-// colsum[D] and (lanes_r - 1) rows of per-lane sums.
-template <typename T>
+// colsum[D] and (lanes_r - 1) rows of per-lane sums.  SPATIAL: the history segments are
+// (1, 8, 8) blocks of frames [frames][Hg][Wg] (hv runs of wv consecutive tokens, Wg tokens
+// apart); the anchor-frame segments stay contiguous.
+template <typename T, bool SPATIAL>
 __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant__ PoolArgs a) {
   constexpr int VEC = 16 / sizeof(T);
   extern __shared__ float colsum[];
@@ -102,22 +105,33 @@ __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant_
   const char* base;
   int64_t rs;
   int nrows;
+  int run = 1 << 30;      // SPATIAL: tokens per run (wv) and rows between runs (Wg)
+  int64_t run_stride = 0;
   float* out;
   if (seg < a.n_anchors) {
     base = a.q + (int64_t)a.anchors[seg] * a.S * a.q_row_stride * a.elt;
     rs = a.q_row_stride;
     nrows = a.S;
     out = a.qbar + (int64_t)seg * a.D;
-  } else if (seg < a.n_anchors + a.M) {
-    base = a.k + (int64_t)(seg - a.n_anchors) * a.B_v * a.hist_row_stride * a.elt;
-    rs = a.hist_row_stride;
-    nrows = a.B_v;
-    out = a.kbar + (int64_t)(seg - a.n_anchors) * a.D;
   } else {
-    base = a.v + (int64_t)(seg - a.n_anchors - a.M) * a.B_v * a.hist_row_stride * a.elt;
+    const bool is_k = seg < a.n_anchors + a.M;
+    const int m = is_k ? seg - a.n_anchors : seg - a.n_anchors - a.M;
     rs = a.hist_row_stride;
-    nrows = a.B_v;
-    out = a.vbar + (int64_t)(seg - a.n_anchors - a.M) * a.D;
+    out = (is_k ? a.kbar : a.vbar) + (int64_t)m * a.D;
+    const char* src = is_k ? a.k : a.v;
+    if (SPATIAL) {
+      const int per_frame = a.nby * a.nbx;
+      const int f = m / per_frame, rem = m - f * per_frame;
+      const int by = rem / a.nbx, bx = rem - by * a.nbx;
+      const int hv = min(8, a.Hg - 8 * by), wv = min(8, a.Wg - 8 * bx);
+      base = src + (((int64_t)f * a.Hg + 8 * by) * a.Wg + 8 * bx) * rs * a.elt;
+      nrows = hv * wv;
+      run = wv;
+      run_stride = a.Wg;
+    } else {
+      base = src + (int64_t)m * a.B_v * rs * a.elt;
+      nrows = a.B_v;
+    }
   }
   const int per = (nrows + a.nsplit - 1) / a.nsplit;
   const int r0 = split * per, r1 = min(nrows, r0 + per);
@@ -131,7 +145,36 @@ __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant_
     float acc[VEC];
 #pragma unroll
     for (int k = 0; k < VEC; ++k) acc[k] = 0.f;
-    if (trl < lanes_r) {
+    if (SPATIAL && trl < lanes_r) {
+      // row r of the segment: run r / wv, token r % wv of that run
+      const char* pc = base + (int64_t)cg * VEC * a.elt;
+      auto rowp = [&](int r) {
+        const int y = r / run;
+        return pc + ((int64_t)y * run_stride + (r - y * run)) * rs * a.elt;
+      };
+      int r = r0 + trl;
+      for (; r + (kPoolUnroll - 1) * lanes_r < r1; r += kPoolUnroll * lanes_r) {
+        float x[kPoolUnroll][VEC];
+#pragma unroll
+        for (int u = 0; u < kPoolUnroll; ++u) load_vec<T>(rowp(r + u * lanes_r), x[u]);
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+          float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+          for (int u = 0; u < kPoolUnroll; u += 2) {
+            s0 += x[u][k];
+            s1 += x[u + 1][k];
+          }
+          acc[k] += s0 + s1;
+        }
+      }
+      for (; r < r1; r += lanes_r) {
+        float x0[VEC];
+        load_vec<T>(rowp(r), x0);
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) acc[k] += x0[k];
+      }
+    } else if (trl < lanes_r) {
       const char* p = base + ((int64_t)(r0 + trl) * rs + (int64_t)cg * VEC) * a.elt;
       const int64_t step = (int64_t)lanes_r * rs * a.elt;
       int r = r0 + trl;
@@ -567,10 +610,16 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   pa.D = D;
   pa.nsplit = p.nsplit;
   pa.elt = a.dtype == CAST_BF16 ? 2 : 4;
+  const HistGeom hg = hist_geom(a.hist);
+  pa.Hg = hg.Hg;
+  pa.Wg = hg.Wg;
+  pa.nby = hg.nby;
+  pa.nbx = hg.nbx;
   for (int k = 0; k < a.n_anchors; ++k) pa.anchors[k] = a.anchors[k];
 
   const size_t psm = route_pool_smem_bytes(a);
-  auto pool_fn = a.dtype == CAST_BF16 ? k_pool<__nv_bfloat16> : k_pool<float>;
+  auto pool_fn = a.dtype == CAST_BF16 ? (hg.spatial ? k_pool<__nv_bfloat16, true> : k_pool<__nv_bfloat16, false>)
+                                      : (hg.spatial ? k_pool<float, true> : k_pool<float, false>);
   if (psm > 48 * 1024 &&
       cudaFuncSetAttribute(pool_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psm) != cudaSuccess)
     return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory for pooling", psm);

@@ -22,11 +22,16 @@ _lib = C.CDLL(LIB_PATH)
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_DEVICE_TIMEOUT = 0, 1, 2, 3, 4
 F32, BF16 = 0, 1
 ROUTE_OMISSION, ROUTE_SIMILARITY = 0, 1
+HIST_BLOCKS, HIST_FRAMES = 0, 1
 GATE_PAPER, GATE_ZERO, GATE_ONE = 0, 1, 2
 MAX_FRAMES, MAX_ANCHORS = 256, 64
 
 _vp = C.c_void_p
 _i32, _i64, _f32 = C.c_int32, C.c_int64, C.c_float
+
+
+class HistLayout(C.Structure):
+    _fields_ = [("kind", _i32), ("frames", _i32), ("Hg", _i32), ("Wg", _i32)]
 
 
 class RouteArgs(C.Structure):
@@ -36,7 +41,7 @@ class RouteArgs(C.Structure):
                 ("B_v", _i32), ("gram", _vp), ("K", _i32), ("eps", _f32), ("mode", _i32),
                 ("idx", _vp), ("u", _vp), ("qbar", _vp), ("kbar", _vp), ("vbar", _vp),
                 ("k_eff", C.POINTER(_i32)), ("refine_passes", _i32), ("lambda_anc", _f32),
-                ("lambda_rec", _f32), ("refine_tol", _f32)]
+                ("lambda_rec", _f32), ("refine_tol", _f32), ("hist", HistLayout)]
 
 
 class AttnArgs(C.Structure):
@@ -45,7 +50,7 @@ class AttnArgs(C.Structure):
                 ("anchors", C.POINTER(_i32)), ("n_anchors", _i32), ("k_hist", _vp),
                 ("v_hist", _vp), ("hist_row_stride", _i64), ("M", _i32), ("B_v", _i32),
                 ("idx", _vp), ("K_eff", _i32), ("scale", _f32), ("o", _vp), ("o_dtype", _i32),
-                ("lse", _vp)]
+                ("lse", _vp), ("hist", HistLayout)]
 
 
 class ParParams(C.Structure):
@@ -70,7 +75,7 @@ class BlockArgs(C.Structure):
                 ("route_lambda_rec", _f32), ("route_refine_tol", _f32), ("scale", _f32),
                 ("r_out", _vp), ("r_dtype", _i32),
                 ("x", _vp), ("idx_out", _vp), ("channel_weight", _vp), ("par", ParParams),
-                ("w_o", _vp), ("b_o", _vp)]
+                ("w_o", _vp), ("b_o", _vp), ("hist", HistLayout)]
 
 
 class FfnArgs(C.Structure):
@@ -168,6 +173,23 @@ def _row_stride(t):
     return t.stride(1)
 
 
+def _history(k_hist, H, d):
+    """(M, B_v, row stride, HistLayout) of the history tensor: [M, B_v, H, d] blocks, or
+    [frames, Hg, Wg, H, d] frames cut into (1, 8, 8) blocks (M = frames ceil(Hg/8) ceil(Wg/8),
+    nominal B_v = 64); None means no history."""
+    lay = HistLayout()
+    if k_hist is None or k_hist.shape[0] == 0:
+        return 0, 0, H * d, lay
+    if k_hist.dim() == 5:
+        F, Hg, Wg = k_hist.shape[:3]
+        if Hg > 1 and k_hist.stride(1) != k_hist.stride(2) * Wg:
+            raise ValueError("history frames must hold consecutive token rows")
+        rs = _row_stride(k_hist.flatten(1, 2))
+        lay.kind, lay.frames, lay.Hg, lay.Wg = HIST_FRAMES, F, Hg, Wg
+        return F * (-(-Hg // 8)) * (-(-Wg // 8)), 64, rs, lay
+    return k_hist.shape[0], k_hist.shape[1], _row_stride(k_hist), lay
+
+
 def _workspace(nbytes, device):
     return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
 
@@ -196,7 +218,7 @@ REFINE_PAPER = dict(passes=2, lambda_anc=1.0, lambda_rec=1.0, tol=1e-6)   # Tab.
 def _route_args(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_OMISSION,
                 refine=None):
     N, S, H, d = q.shape
-    M = k_hist.shape[0]
+    M, B_v, rs, lay = _history(k_hist, H, d)
     a = RouteArgs()
     a.q, a.q_row_stride = _ptr(q), _row_stride(q)
     a.n_frames, a.S, a.H, a.d = N, S, H, d
@@ -205,8 +227,8 @@ def _route_args(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_O
     a.anchors = C.cast(a._anchors, C.POINTER(_i32))
     a.n_anchors = len(anchors)
     a.k_hist, a.v_hist = _ptr(k_hist), _ptr(v_hist)
-    a.hist_row_stride = _row_stride(k_hist) if M > 0 else H * d
-    a.M, a.B_v = M, k_hist.shape[1]
+    a.hist_row_stride = rs
+    a.M, a.B_v, a.hist = M, B_v if M > 0 else k_hist.shape[1], lay
     a.gram = _ptr(gram)
     a.K, a.eps, a.mode = K, eps, mode
     if refine:
@@ -225,7 +247,7 @@ def cast_route_topk(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROU
     """Returns idx [K_f, H, K_eff] int32 (and u, (qbar, kbar, vbar) when asked).  refine: None
     (independent TopK) or a dict like REFINE_PAPER (coupled refinement, Alg. routing)."""
     a = _route_args(q, anchors, k_hist, v_hist, K, gram, eps, mode, refine)
-    Kf, H, d, M = len(anchors), q.shape[2], q.shape[3], k_hist.shape[0]
+    Kf, H, d, M = len(anchors), q.shape[2], q.shape[3], a.M
     keff = min(K, M)
     dev = q.device
     idx = torch.empty((Kf, H, keff), dtype=torch.int32, device=dev)
@@ -254,7 +276,7 @@ def cast_route_topk_noalloc(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8,
     """As cast_route_topk, with the library's fixed 16 MiB device scratch instead of a
     caller workspace (for callers that cannot allocate); returns idx (and u)."""
     a = _route_args(q, anchors, k_hist, v_hist, K, gram, eps, mode)
-    Kf, H, M = len(anchors), q.shape[2], k_hist.shape[0]
+    Kf, H, M = len(anchors), q.shape[2], a.M
     idx = torch.empty((Kf, H, min(K, M)), dtype=torch.int32, device=q.device)
     u = torch.empty((Kf, H, M), dtype=torch.float32, device=q.device) if want_u else None
     a.idx, a.u = _ptr(idx), _ptr(u)
@@ -265,7 +287,7 @@ def cast_route_topk_noalloc(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8,
 # --------------------------------------------------------------------------- attention
 def _attn_args(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale=0.0):
     N, S, H, d = q.shape
-    M = k_hist.shape[0] if k_hist is not None else 0
+    M, B_v, rs, lay = _history(k_hist, H, d)
     a = AttnArgs()
     a.q, a.k_cur, a.v_cur = _ptr(q), _ptr(k_cur), _ptr(v_cur)
     a.q_row_stride, a.cur_row_stride = _row_stride(q), _row_stride(k_cur)
@@ -274,9 +296,8 @@ def _attn_args(q, k_cur, v_cur, anchors, k_hist, v_hist, idx, scale=0.0):
     a.anchors = C.cast(a._anchors, C.POINTER(_i32))
     a.n_anchors = len(anchors)
     a.k_hist, a.v_hist = _ptr(k_hist), _ptr(v_hist)
-    a.hist_row_stride = _row_stride(k_hist) if M > 0 else H * d
-    a.M = M
-    a.B_v = k_hist.shape[1] if M > 0 else 0
+    a.hist_row_stride = rs
+    a.M, a.B_v, a.hist = M, B_v, lay
     a.idx = _ptr(idx)
     a.K_eff = idx.shape[-1] if idx is not None else 0
     a.scale = scale
@@ -340,7 +361,7 @@ def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None,
                gram=None, route_eps=1e-8, route_mode=ROUTE_OMISSION, scale=0.0,
                channel_weight=None, params=None, refine=None, w_o=None, b_o=None):
     N, S, H, d = q.shape
-    M = k_hist.shape[0]
+    M, B_v, rs, lay = _history(k_hist, H, d)
     a = BlockArgs()
     a.q, a.k_cur, a.v_cur = _ptr(q), _ptr(k_cur), _ptr(v_cur)
     a.q_row_stride, a.cur_row_stride = _row_stride(q), _row_stride(k_cur)
@@ -349,8 +370,8 @@ def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None,
     a.anchors = C.cast(a._anchors, C.POINTER(_i32))
     a.n_anchors = len(anchors)
     a.k_hist, a.v_hist = _ptr(k_hist), _ptr(v_hist)
-    a.hist_row_stride = _row_stride(k_hist) if M > 0 else H * d
-    a.M, a.B_v = M, k_hist.shape[1]
+    a.hist_row_stride = rs
+    a.M, a.B_v, a.hist = M, B_v if M > 0 else k_hist.shape[1], lay
     a.gram, a.K, a.route_eps, a.route_mode, a.scale = _ptr(gram), K, route_eps, route_mode, scale
     if refine:
         a.route_refine_passes, a.route_lambda_anc = refine["passes"], refine["lambda_anc"]

@@ -94,6 +94,22 @@ def tokens_with_offsets(seed_seq, n_groups: int, rows: int, H: int, d: int,
     return x
 
 
+def frames_with_region_offsets(seed_seq, n_frames: int, Hg: int, Wg: int, H: int, d: int,
+                               offset_scale: float, region: int = 8) -> np.ndarray:
+    """[n_frames, Hg, Wg, H, d] float32 history frames: N(0,1) tokens plus one
+    N(0, offset_scale^2) d-vector per (frame, region x region patch of the token grid, head),
+    so that the means of neighbouring patches differ by O(1).  Patches at the right and
+    bottom edges are cut by the grid."""
+    s_tok, s_off = seed_seq.spawn(2)
+    x = normal(s_tok, (n_frames, Hg, Wg, H, d))
+    if offset_scale:
+        ny, nx = -(-Hg // region), -(-Wg // region)
+        off = _gen(s_off).standard_normal((n_frames, ny, nx, H, d), dtype=np.float32)
+        off = np.repeat(np.repeat(off, region, axis=1), region, axis=2)[:, :Hg, :Wg]
+        x += np.float32(offset_scale) * off
+    return x
+
+
 # --------------------------------------------------------------------------
 # residual fields for PAR
 # --------------------------------------------------------------------------

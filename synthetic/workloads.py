@@ -31,6 +31,8 @@ class BlockStepWorkload:
     band_radius: float = -1.0   # < 0: no band cut (the paper's gate on every bin)
     offset_scale: float = 1.0   # per-(frame|block, head) offsets of the tokens
     amp_drift: float = 0.0      # per-frame amplitude drift of the PAR residual fields
+    hist_frames: int = 0        # > 0: the history is this many frames of the chunk's grid,
+                                # cut into (1, 8, 8) blocks (M of them, B_v = 64 nominal)
 
     @property
     def S(self):
@@ -47,6 +49,15 @@ MG = BlockStepWorkload("mg_bf16_8f_30x52_h12d128_m16_k4", 1, 8, (30, 52), 12, 12
                        4, (0, 2, 4, 6), "bf16")
 HY = BlockStepWorkload("hy_bf16_16f_44x80_h24d128_m32_k8", 2, 16, (44, 80), 24, 128, 32, 3520,
                        8, (0, 3, 7, 12, 15), "bf16", amp_drift=0.01)
+
+
+# The paper's KV granularity (App. C Tab. config: (1, 8, 8) blocks, partial blocks masked;
+# Tab. config_cast: K = ceil(0.2 M)) on the two backbone shapes with 16 / 32 history frames:
+# 30x52 tokens = 4 x 7 blocks per frame, 44x80 = 6 x 10.
+MG64 = BlockStepWorkload("mg64_bf16_8f_30x52_h12d128_hist16f_m448_k90", 6, 8, (30, 52), 12, 128,
+                         448, 64, 90, (0, 2, 4, 6), "bf16", hist_frames=16)
+HY64 = BlockStepWorkload("hy64_bf16_16f_44x80_h24d128_hist32f_m1920_k384", 7, 16, (44, 80), 24, 128,
+                         1920, 64, 384, (0, 3, 7, 12, 15), "bf16", amp_drift=0.01, hist_frames=32)
 
 
 @dataclass(frozen=True)
@@ -105,7 +116,8 @@ def _maybe_bf16(x, dtype):
 
 def block_step_inputs(w: BlockStepWorkload, scale_rows: int | None = None):
     """Inputs of one block step: q, k_cur, v_cur [N_cur, S, H, d], k_hist, v_hist
-    [M, B_v, H, d] (float32 holding bf16 values: the attention runs in bf16),
+    [M, B_v, H, d] (or history frames [F_h, Hg, Wg, H, d] when w.hist_frames) (float32 holding
+    bf16 values: the attention runs in bf16),
     plus anchors and the mask.  All current frames carry Q (only anchor rows
     are read)."""
     ss = np.random.SeedSequence(w.seed)
@@ -114,8 +126,14 @@ def block_step_inputs(w: BlockStepWorkload, scale_rows: int | None = None):
     q = G.tokens_with_offsets(sq, w.n_cur, S, w.H, w.d, w.offset_scale)
     kc = G.tokens_with_offsets(skc, w.n_cur, S, w.H, w.d, w.offset_scale)
     vc = G.tokens_with_offsets(svc, w.n_cur, S, w.H, w.d, w.offset_scale)
-    kh = G.tokens_with_offsets(skh, w.M, w.B_v, w.H, w.d, w.offset_scale)
-    vh = G.tokens_with_offsets(svh, w.M, w.B_v, w.H, w.d, w.offset_scale)
+    if w.hist_frames:
+        # history frames [F_h, Hg, Wg, H, d]; (1, 8, 8) blocks carry their own offsets
+        Hg, Wg = w.grid
+        kh = G.frames_with_region_offsets(skh, w.hist_frames, Hg, Wg, w.H, w.d, w.offset_scale)
+        vh = G.frames_with_region_offsets(svh, w.hist_frames, Hg, Wg, w.H, w.d, w.offset_scale)
+    else:
+        kh = G.tokens_with_offsets(skh, w.M, w.B_v, w.H, w.d, w.offset_scale)
+        vh = G.tokens_with_offsets(svh, w.M, w.B_v, w.H, w.d, w.offset_scale)
     out = dict(q=q, k_cur=kc, v_cur=vc, k_hist=kh, v_hist=vh)
     for k in out:
         out[k] = G.round_bf16(out[k])

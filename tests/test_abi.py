@@ -211,3 +211,72 @@ def test_ffn_validation(lib):
     a.D, a.w1 = 64, _fake(0x20004)
     assert so.cast_ffn_step(C.byref(a), _fake(0x100000), need, None) == 1          # misaligned weight
 
+
+
+@pytest.mark.parametrize("hist,M,B_v,status", [
+    ((5, 0, 0, 0), 4, 8, 1),                 # unknown layout kind
+    ((1, 0, 16, 16), 4, 64, 1),              # no history frames
+    ((1, 1, 16, 16), 4, 64, 0),              # 1 frame of 16x16 tokens = 4 (1,8,8) blocks
+    ((1, 1, 17, 16), 4, 64, 1),              # 17 rows: 3 x 2 = 6 blocks, not 4
+    ((1, 2, 9, 20), 12, 64, 0),              # truncated edge blocks: 2 x 2 x 3
+    ((1, 1, 16, 16), 4, 8, 1),               # B_v must be the nominal 64
+])
+def test_route_history_layout_validation(lib, hist, M, B_v, status):
+    a = _route(lib, M=M, B_v=B_v)
+    a.hist.kind, a.hist.frames, a.hist.Hg, a.hist.Wg = hist
+    so = lib.library()
+    if status:
+        assert so.cast_route_topk(C.byref(a), _fake(0x100000), 1 << 30, None) == status
+        assert so.cast_last_error_detail() != b""
+    else:
+        # valid layouts pass validation: the call only fails later for the missing workspace
+        assert so.cast_route_topk(C.byref(a), None, 0, None) == 1
+        assert b"workspace" in so.cast_last_error_detail()
+
+
+def test_attention_history_layout_validation(lib):
+    a = lib.AttnArgs()
+    a.q = a.k_cur = a.v_cur = _fake()
+    a.k_hist, a.v_hist = _fake(0x20000), _fake(0x30000)
+    a.q_row_stride = a.cur_row_stride = a.hist_row_stride = 256
+    a.n_frames, a.S, a.H, a.d = 2, 16, 2, 128
+    an = (C.c_int32 * 1)(1)
+    a.anchors = C.cast(an, C.POINTER(C.c_int32))
+    a.n_anchors = 1
+    a.idx = _fake(0x40000)
+    a.M, a.B_v, a.K_eff = 6, 64, 3
+    a.o, a.o_dtype = _fake(), lib.BF16
+    a.hist.kind, a.hist.frames, a.hist.Hg, a.hist.Wg = lib.HIST_FRAMES, 1, 16, 16   # 4 blocks
+    so = lib.library()
+    assert so.cast_anchor_attention(C.byref(a), None, 1 << 30, None) == 1
+    assert b"(1,8,8)" in so.cast_last_error_detail()
+
+
+def test_struct_layouts_match_the_header(lib, tmp_path):
+    """Every ctypes argument struct has the size and field offsets that a C compiler gives
+    the header's struct (compiled with gcc on the host)."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no gcc")
+    structs = {"cast_route_args": lib.RouteArgs, "cast_attn_args": lib.AttnArgs,
+               "cast_par_params": lib.ParParams, "cast_par_args": lib.ParArgs,
+               "cast_block_args": lib.BlockArgs, "cast_ffn_args": lib.FfnArgs,
+               "cast_select_args": lib.SelectArgs, "cast_hist_layout": lib.HistLayout}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "cast.h"', "int main(void) {"]
+    for cname, py in structs.items():
+        lines.append(f'printf("{cname} sizeof %zu\\n", sizeof({cname}));')
+        for fname, _ in py._fields_:
+            lines.append(f'printf("{cname} {fname} %zu\\n", offsetof({cname}, {fname}));')
+    lines += ["return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)],
+                   check=True, capture_output=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout
+    for line in out.splitlines():
+        cname, fname, val = line.split()
+        py = structs[cname]
+        got = C.sizeof(py) if fname == "sizeof" else getattr(py, fname).offset
+        assert got == int(val), (cname, fname, got, int(val))
