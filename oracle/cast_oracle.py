@@ -298,13 +298,32 @@ def pooled_routing(q, anchors, k_hist, v_hist, proj=None, eps=1e-8) -> Routing:
     return Routing(qbar, kbar, vbar, s, pi, obar, delta, u)
 
 
-def topk_blocks(score: np.ndarray, K: int):
+def candidate_mask(candidates, M, K=0):
+    """Fixed candidate sets C_i (App. B.3): [..., M_c] distinct block indices -> boolean
+    membership [..., M].  The paper requires M_c >= K_KV; a set smaller than min(K, M), a
+    repeated index or one outside [0, M) raises ValueError."""
+    c = np.asarray(candidates, dtype=np.int64)
+    mask = np.zeros(c.shape[:-1] + (M,), dtype=bool)
+    for r in np.ndindex(c.shape[:-1]):
+        row = c[r]
+        if np.any(row < 0) or np.any(row >= M) or len(set(row.tolist())) != len(row):
+            raise ValueError("candidate indices must be distinct and inside [0, M)")
+        if len(row) < min(K, M):
+            raise ValueError("a candidate set smaller than the budget")
+        mask[r + (row,)] = True
+    return mask
+
+
+def topk_blocks(score: np.ndarray, K: int, candidates=None):
     """Per (anchor, head): the K largest scores, ties to the lower block index,
-    returned ascending.  K >= M or M == 0 keeps every block (routing bypass)."""
+    returned ascending.  K >= M or M == 0 keeps every block (routing bypass).  With
+    candidate sets ([..., M_c] block indices, App. B.3) only members are eligible."""
     M = score.shape[-1]
     keff = min(K, M)
     if M == 0:
         return np.zeros(score.shape[:-1] + (0,), dtype=np.int64)
+    if candidates is not None:
+        score = np.where(candidate_mask(candidates, M, K), score, -np.inf)
     flat = score.reshape(-1, M)
     idx = np.empty((flat.shape[0], keff), dtype=np.int64)
     for r in range(flat.shape[0]):
@@ -489,16 +508,24 @@ def _mask_from_topk(score, K):
 
 
 def coupled_routing(u, anchors, n_frames, K, passes=2, lam_anc=1.0, lam_rec=1.0, tol=1e-6,
-                    with_info=False):
+                    with_info=False, candidates=None):
     """Alg. (routing) for one head: u [n_anchors, M] omission scores.  Initialise every mask
     with TopK(u_i), then `passes` directional passes (forward, backward, ...) replacing M_i by
     TopK(G_i) when J drops by more than tol * max(J, 1e-8); stop after a pass with no change.
-    Returns idx [n_anchors, K_eff] ascending (and the objective trace with with_info)."""
+    candidates: optional fixed sets C_i ([n_anchors, M_c] block indices, App. B.3): both TopK
+    run over C_i only; blocks outside C_i stay zero and still count as omissions in J and in
+    the neighbours' gains.  Returns idx [n_anchors, K_eff] ascending (and the objective trace
+    with with_info)."""
     u = np.asarray(u, dtype=np.float64)
     J_, M = u.shape
     keff = min(K, M)
     co = routing_coefficients(anchors, n_frames)
-    x = np.stack([_mask_from_topk(u[i], keff) for i in range(J_)]) if M else np.zeros((J_, 0))
+    cand = np.ones((J_, M), dtype=bool) if candidates is None else candidate_mask(candidates, M, K)
+
+    def restrict(i, score):
+        return np.where(cand[i], score, -np.inf)
+
+    x = np.stack([_mask_from_topk(restrict(i, u[i]), keff) for i in range(J_)]) if M else np.zeros((J_, 0))
     trace = [routing_objective(u, x, co, lam_anc, lam_rec)]
     ambiguous = False
     if 0 < keff < M:
@@ -507,12 +534,12 @@ def coupled_routing(u, anchors, n_frames, K, passes=2, lam_anc=1.0, lam_rec=1.0,
             order = range(J_) if s % 2 == 1 else range(J_ - 1, -1, -1)
             for i in order:
                 G = retain_gains(i, u, x, co, lam_anc, lam_rec)
-                new = _mask_from_topk(G, keff)
+                new = _mask_from_topk(restrict(i, G), keff)
                 gain = float(np.sum(G * new) - np.sum(G * x[i]))
                 Jcur = routing_objective(u, x, co, lam_anc, lam_rec)
                 thr = tol * max(Jcur, 1e-8)
-                srt = -np.sort(-G)
-                if abs(gain - thr) <= 1e-4 * max(thr, 1e-12) or (
+                srt = -np.sort(-G[cand[i]])
+                if abs(gain - thr) <= 1e-4 * max(thr, 1e-12) or (len(srt) > keff and
                         srt[keff - 1] - srt[keff] <= 1e-4 * max(abs(srt[keff - 1]), 1e-12)):
                     ambiguous = True
                 if gain > thr:

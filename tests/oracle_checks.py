@@ -542,6 +542,68 @@ def check_coupled_routing():
 
 
 
+def _random_candidates(r, J, M, Mc):
+    return np.stack([np.sort(r.choice(M, size=Mc, replace=False)) for _ in range(J)])
+
+
+def check_candidate_topk():
+    """Fixed candidate sets (App. B.3): TopK runs over C_i only (the K-subset of C_i with the
+    largest sum, brute force), C_i = all blocks is the unrestricted TopK, and a set smaller than
+    the budget or with a repeated / out-of-range index is rejected."""
+    r = _rng(23)
+    for _ in range(20):
+        M, K, Mc = 8, 3, 5
+        u = r.standard_normal((2, M))
+        c = _random_candidates(r, 2, M, Mc)
+        got = O.topk_blocks(u, K, candidates=c)
+        for i in range(2):
+            best = max(itertools.combinations(c[i].tolist(), K), key=lambda t: sum(u[i, list(t)]))
+            assert list(got[i]) == sorted(best)
+        assert np.array_equal(O.topk_blocks(u, K, candidates=np.tile(np.arange(M), (2, 1))),
+                              O.topk_blocks(u, K))
+    for bad in ([[0, 1]], [[0, 0, 1]], [[0, 1, 9]]):
+        try:
+            O.topk_blocks(np.zeros((1, 8)), 3, candidates=np.array(bad))
+        except ValueError:
+            continue
+        raise AssertionError(f"candidate set {bad} accepted")
+
+
+def check_candidate_coupled_routing():
+    """Alg. (routing) with fixed candidate sets: every kept block lies in C_i, J never
+    increases, the result is no worse than independent TopK over the same sets, C_i = all
+    blocks reproduces the unrestricted refinement, and at a fixed point no anchor can lower J
+    (blocks outside C_i counted as omitted) with any K-subset of its own C_i (brute force)."""
+    r = _rng(24)
+    for trial in range(12):
+        anchors = sorted(r.choice(9, size=int(r.integers(2, 5)), replace=False).tolist())
+        J, M, K, Mc = len(anchors), 7, 2, 4
+        u = r.exponential(size=(J, M)) * r.uniform(0.2, 3.0, size=(1, M))
+        c = _random_candidates(r, J, M, Mc)
+        cm = O.candidate_mask(c, M)
+        co = O.routing_coefficients(anchors, 9)
+        idx, info = O.coupled_routing(u, anchors, 9, K, passes=60, with_info=True, candidates=c)
+        assert idx.shape == (J, K)
+        assert all(cm[i, idx[i]].all() for i in range(J))
+        tr = info["trace"]
+        assert all(b <= a + 1e-12 for a, b in zip(tr, tr[1:]))
+        ind = O.topk_blocks(u, K, candidates=c)
+        xi = np.zeros_like(u)
+        for i in range(J):
+            xi[i, ind[i]] = 1
+        x = info["x"]
+        J0 = O.routing_objective(u, x, co)
+        assert J0 <= O.routing_objective(u, xi, co) + 1e-12
+        for i in range(J):
+            for sub in itertools.combinations(c[i].tolist(), K):
+                y = x.copy()
+                y[i] = 0
+                y[i, list(sub)] = 1
+                assert O.routing_objective(u, y, co) >= J0 - 1e-6 * max(J0, 1e-8) - 1e-12
+        full = np.tile(np.arange(M), (J, 1))
+        assert np.array_equal(O.coupled_routing(u, anchors, 9, K, candidates=full),
+                              O.coupled_routing(u, anchors, 9, K))
+
 
 # ----------------------------------------------------------------------------------------------
 # Control-aware frame selection (Eqs. sensitivity, normalization, debt, score)

@@ -63,11 +63,13 @@ def _pooled_no_renorm(q, anchors, k, v, proj=None, eps=1e-8):
     return rt
 
 
-def _topk_high_ties(score, K):
+def _topk_high_ties(score, K, candidates=None):
     M = score.shape[-1]
     keff = min(K, M)
     if M == 0:
         return np.zeros(score.shape[:-1] + (0,), dtype=np.int64)
+    if candidates is not None:
+        score = np.where(O.candidate_mask(candidates, M, K), score, -np.inf)
     flat = score.reshape(-1, M)
     out = [np.sort(np.lexsort((-np.arange(M), -r))[:keff]) for r in flat]
     return np.array(out).reshape(score.shape[:-1] + (keff,))
@@ -180,7 +182,56 @@ def _budget_floor(M):
     return int(2 * M // 10)
 
 
+_orig_coupled = O.coupled_routing
+
+
+def _topk_candidates_ignored(score, K, candidates=None):
+    return _orig_topk(score, K)
+
+
+_orig_topk = O.topk_blocks
+
+
+def _coupled_candidates_only_at_init(u, anchors, n_frames, K, passes=2, lam_anc=1.0, lam_rec=1.0,
+                                     tol=1e-6, with_info=False, candidates=None):
+    # the candidate restriction applied to the initial TopK only, not to the best responses
+    if candidates is None:
+        return _orig_coupled(u, anchors, n_frames, K, passes, lam_anc, lam_rec, tol, with_info)
+    x0 = _orig_topk(np.asarray(u, dtype=np.float64), K, candidates=candidates)
+    lifted = np.asarray(u, dtype=np.float64).copy()
+    for i in range(lifted.shape[0]):
+        lifted[i, x0[i]] += 1e6          # forces the same initial sets
+    res = _orig_coupled(lifted, anchors, n_frames, K, passes, lam_anc, lam_rec, tol, True)
+    idx, info = res
+    info["x"] = np.zeros_like(lifted)
+    for i in range(lifted.shape[0]):
+        info["x"][i, idx[i]] = 1.0
+    return (idx, info) if with_info else idx
+
+
+def _coupled_noncandidates_retained(u, anchors, n_frames, K, passes=2, lam_anc=1.0, lam_rec=1.0,
+                                    tol=1e-6, with_info=False, candidates=None):
+    # blocks outside a neighbour's C_i treated as retained (x = 1) in the gains
+    if candidates is None:
+        return _orig_coupled(u, anchors, n_frames, K, passes, lam_anc, lam_rec, tol, with_info)
+    cm = O.candidate_mask(candidates, np.asarray(u).shape[1])
+    gains = O.retain_gains
+
+    def patched(i, uu, x, co, la=1.0, lr=1.0):
+        return gains(i, uu, np.where(cm, x, 1.0), co, la, lr)
+
+    O.retain_gains = patched
+    try:
+        return _orig_coupled(u, anchors, n_frames, K, passes, lam_anc, lam_rec, tol, with_info,
+                             candidates=candidates)
+    finally:
+        O.retain_gains = gains
+
+
 MUTATIONS = {
+    "candidates_ignored_in_topk": ("topk_blocks", _topk_candidates_ignored),
+    "candidates_only_at_init": ("coupled_routing", _coupled_candidates_only_at_init),
+    "noncandidates_retained_in_gains": ("coupled_routing", _coupled_noncandidates_retained),
     "partial_blocks_padded": ("spatial_blocks", _spatial_blocks_padded),
     "budget_floor": ("paper_budget", _budget_floor),
     "gelu_erf_form": ("gelu_tanh", _gelu_erf),
