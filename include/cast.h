@@ -124,6 +124,13 @@ typedef struct {
   int32_t refine_passes;
   float lambda_anc, lambda_rec, refine_tol;
   cast_hist_layout hist;          /* layout of k_hist/v_hist; zero = CAST_HIST_BLOCKS */
+  /* Optional fixed candidate sets C_i (App. B.3): device int32 [n_anchors, H, M_c], distinct
+     block indices per (anchor, head), K_eff <= M_c <= M.  The TopK initialisation and the
+     refinement's best responses choose within C_i only; blocks outside C_i stay unselected and
+     still count as omissions in J and in the neighbours' gains.  NULL = every block
+     (M_c = M, the paper's setting, Tab. config_cast). */
+  const int32_t* candidates;
+  int32_t M_c;
 } cast_route_args;
 
 /* Pooled mean statistics q_bar, k_bar, v_bar (mean over a frame's S tokens and over a
@@ -139,7 +146,10 @@ typedef struct {
  * an unknown hist.kind, or CAST_HIST_FRAMES with a non-positive grid, M different from its
  * block count or B_v != 64,
  * a workspace smaller than cast_route_workspace_size(), refinement with a negative weight or
- * tolerance or outside CAST_ROUTE_OMISSION; UNSUPPORTED for d not 64/128, M > 16384,
+ * tolerance or outside CAST_ROUTE_OMISSION, candidates with M_c outside K_eff..M; a candidate
+ * index outside [0, M) or repeated within a set makes the kernel record an error that
+ * cast_check_device() reports as INVALID_ARG (that set then holds fewer members and its
+ * selection is completed by the lowest-index other blocks); UNSUPPORTED for d not 64/128, M > 16384,
  * H*d > 51200 channels (pooling shared memory) or 4*(2*K_f*d + 3*K_f*M + M + 8*d) bytes of
  * per-head state above 200 KB. */
 cast_status cast_route_topk(const cast_route_args* args, void* workspace,
@@ -284,6 +294,8 @@ typedef struct {
   const void* w_o;                /* optional device bf16 [H*d, H*d], layer layout [out, in] */
   const void* b_o;                /* optional device [H*d] of r_dtype */
   cast_hist_layout hist;          /* layout of k_hist/v_hist; zero = CAST_HIST_BLOCKS */
+  const int32_t* route_candidates;   /* optional, as cast_route_args.candidates */
+  int32_t route_M_c;
 } cast_block_args;
 
 /* route_topk -> anchor_attention -> (output projection) -> par_reconstruct on one stream,
@@ -371,8 +383,9 @@ const char* cast_status_string(cast_status s);
 /* Message of the last error on the calling thread ("" if none). */
 const char* cast_last_error_detail(void);
 /* Synchronises `stream`, then reports CAST_ERR_DEVICE_TIMEOUT if a kernel on the current
- * device recorded a bounded-wait timeout (and clears the record), CAST_ERR_CUDA on a
- * pending CUDA error, CAST_OK otherwise. */
+ * device recorded a bounded-wait timeout, CAST_ERR_INVALID_ARG if one met a device-side index
+ * outside its range (a routed block in attention, a routing candidate) (both records are
+ * cleared), CAST_ERR_CUDA on a pending CUDA error, CAST_OK otherwise. */
 cast_status cast_check_device(void* stream);
 /* Library version, "major.minor.patch". */
 const char* cast_version(void);

@@ -153,6 +153,14 @@ cast_status validate_route(const cast_route_args* a) {
     if (!(a->lambda_anc >= 0.f) || !(a->lambda_rec >= 0.f) || !(a->refine_tol >= 0.f))
       return fail(CAST_ERR_INVALID_ARG, "%s: refinement weights and tolerance must be >= 0", who);
   }
+  if (a->candidates) {
+    const int keff = a->K < a->M ? a->K : a->M;
+    if (a->M_c < 1 || a->M_c < keff || a->M_c > a->M)
+      return fail(CAST_ERR_INVALID_ARG, "%s: candidate sets of M_c=%d blocks need %d <= M_c <= M=%d", who,
+                  a->M_c, keff, a->M);
+    if (reinterpret_cast<uintptr_t>(a->candidates) % 4)
+      return fail(CAST_ERR_INVALID_ARG, "%s: candidates misaligned", who);
+  }
   if (route_pool_smem_bytes(*a) > 200 * 1024)
     return fail(CAST_ERR_UNSUPPORTED, "%s: H*d = %d channels exceed the pooling kernel's shared memory",
                 who, a->H * a->d);
@@ -263,6 +271,8 @@ cast_route_args route_of_block(const cast_block_args* a, int32_t* idx) {
   r.lambda_rec = a->route_lambda_rec;
   r.refine_tol = a->route_refine_tol;
   r.hist = a->hist;
+  r.candidates = a->route_candidates;
+  r.M_c = a->route_M_c;
   r.idx = idx;
   return r;
 }
@@ -584,8 +594,10 @@ cast_status cast_check_device(void* stream) {
   if (e != cudaSuccess) return fail(CAST_ERR_CUDA, "cast_check_device: %s", cudaGetErrorString(e));
   const unsigned int wa = attention_error_word(st, true);
   const unsigned int wp = par_error_word(st, true);
+  const unsigned int wr = route_error_word(st, true);
   if (wa == 1u || wp) return fail(CAST_ERR_DEVICE_TIMEOUT, "a kernel gave up on a bounded wait");
   if (wa == 2u) return fail(CAST_ERR_INVALID_ARG, "attention: a routed block index was outside [0, M)");
+  if (wr) return fail(CAST_ERR_INVALID_ARG, "routing: a candidate index was outside [0, M) or repeated");
   return check_launch("cast_check_device");
 }
 

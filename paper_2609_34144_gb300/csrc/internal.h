@@ -62,6 +62,8 @@ size_t route_pool_smem_bytes(const cast_route_args& a);
 size_t route_head_smem_bytes(const cast_route_args& a);
 // Arguments must have been validated; ws holds at least route_plan(a).total_bytes.
 cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st);
+// Nonzero when a routing kernel met a candidate index outside [0, M) or repeated in its set.
+unsigned int route_error_word(cudaStream_t st, bool clear);
 
 // ------------------------------------------------------------------ attention
 struct AttnPlan {

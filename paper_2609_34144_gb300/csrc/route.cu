@@ -234,14 +234,17 @@ __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant_
 // ---------------------------------------------------------------------- per-head kernel
 constexpr int kHeadThreads = 256, kHeadWarps = kHeadThreads / 32;
 
+__device__ unsigned int g_route_error;
+
 struct HeadArgs {
   const float* qbar;
   const float* kbar;
   const float* vbar;
   const float* gram;
+  const int32_t* cand;   // optional [n_anchors, H, Mc] candidate sets
   int32_t* idx;
   float* u_out;
-  int H, d, M, n_anchors, K_eff, mode, passes, stage_kv;
+  int H, d, M, n_anchors, K_eff, mode, passes, stage_kv, Mc;
   float eps, lam_anc, lam_rec, tol;
   float A[CAST_MAX_ANCHORS], B[CAST_MAX_ANCHORS], C[CAST_MAX_ANCHORS];   // interval (j-1, j)
   float AL, BL, CL, AR, BR, CR;                                          // boundary sets
@@ -280,21 +283,29 @@ __device__ __forceinline__ bool in_topk(const float* key, int M, int K, int m) {
 __device__ __forceinline__ float warp_total(float v) { return warp_sum(v); }
 
 // grid (H).  Dynamic smem (floats): qb[na*d], ob[na*d], pi[na*M], key[na*M], x[na*M], G[M],
-// e[kHeadWarps*d] (Gram scratch) and, when stage_kv, kb[M*d], vb[M*d] (this head's means).
+// with candidate sets Gc[M], then e[kHeadWarps*d] (Gram scratch); with candidate sets the
+// membership bytes cm[na*M]; when stage_kv, kb[M*d], vb[M*d] (this head's means).
 __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ HeadArgs a) {
   extern __shared__ float sm[];
   const int h = blockIdx.x, na = a.n_anchors, M = a.M, d = a.d, K = a.K_eff;
   const int D = a.H * d;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool restricted = a.cand != nullptr;
   float* qb = sm;
   float* ob = qb + na * d;
   float* pi = ob + na * d;
   float* key = pi + na * M;
   float* x = key + na * M;
   float* G = x + na * M;
-  float* ew = G + M;
+  float* Gc = G + M;                         // best-response keys restricted to C_i
+  float* ew = Gc + (restricted ? M : 0);
+  uint8_t* cm = reinterpret_cast<uint8_t*>(ew + kHeadWarps * d);
   // float4 stores below: the staged means start on a 16-byte boundary
-  float* kb_s = sm + (((ew + kHeadWarps * d) - sm + 3) & ~(ptrdiff_t)3);
+  const size_t cm_bytes = restricted ? (((size_t)na * M + 15) & ~(size_t)15) : 0;
+  float* kb_s = reinterpret_cast<float*>(
+      reinterpret_cast<uint8_t*>(sm) +
+      (((reinterpret_cast<uint8_t*>(ew + kHeadWarps * d) - reinterpret_cast<uint8_t*>(sm)) + 15) & ~(ptrdiff_t)15) +
+      cm_bytes);
   float* vb_s = kb_s + (size_t)M * d;
   launch_dependents();
   grid_dependency_wait();   // the pooled means come from the preceding kernel
@@ -444,10 +455,34 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
       a.u_out[((int64_t)i * a.H + h) * M + m] = key[p];
     }
   if (K == 0) return;
+  // candidate sets C_i (App. B.3): membership bytes; the initial TopK runs on keys that are
+  // -inf outside C_i (pi is free here and holds them)
+  const float* key0 = key;
+  if (restricted) {
+    for (int p = tid; p < na * M; p += kHeadThreads) cm[p] = 0;
+    __syncthreads();
+    for (int e = tid; e < na * a.Mc; e += kHeadThreads) {
+      const int i = e / a.Mc, c = e - i * a.Mc;
+      const int m = __ldg(a.cand + ((int64_t)i * a.H + h) * a.Mc + c);
+      if (m < 0 || m >= M) atomicExch(&g_route_error, 1u);
+      else cm[i * M + m] = 1;
+    }
+    __syncthreads();
+    // a repeated index leaves its set with fewer than Mc members
+    for (int i = warp; i < na; i += kHeadWarps) {
+      int n = 0;
+      for (int m = lane; m < M; m += 32) n += cm[i * M + m];
+      n = __reduce_add_sync(0xffffffffu, n);
+      if (lane == 0 && n != a.Mc) atomicExch(&g_route_error, 1u);
+    }
+    for (int p = tid; p < na * M; p += kHeadThreads) pi[p] = cm[p] ? key[p] : -INFINITY;
+    __syncthreads();
+    key0 = pi;
+  }
   // initial masks: TopK of each anchor's key (Eq. topk)
   for (int p = tid; p < na * M; p += kHeadThreads) {
     const int i = p / M, m = p - i * M;
-    x[p] = in_topk(key + i * M, M, K, m) ? 1.f : 0.f;
+    x[p] = in_topk(key0 + i * M, M, K, m) ? 1.f : 0.f;
   }
   __syncthreads();
   if (a.passes > 0 && K < M) {
@@ -506,19 +541,22 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
               if (i == na - 2) rec += AR * ui + 2.f * CR * (1.f - x[(na - 1) * M + m]) * sq[(na - 1) * M + m];
               if (i == na - 1) rec += BR * ui + 2.f * CR * (1.f - x[(na - 2) * M + m]) * sq[(na - 1) * M + m];
             }
-            G[m] = lam_anc * ui + lam_rec * rec;
+            const float g = lam_anc * ui + lam_rec * rec;
+            G[m] = g;
+            if (restricted) Gc[m] = cm[i * M + m] ? g : -INFINITY;
           }
           __syncwarp();
-          // best response TopK(G) and its gain sum_m G_m (x_new - x_i); J is affine in x_i, so
-          // the accepted step lowers J by exactly that gain
+          // best response TopK(G) (within C_i) and its gain sum_m G_m (x_new - x_i); J is
+          // affine in x_i, so the accepted step lowers J by exactly that gain
+          const float* Gk = restricted ? Gc : G;
           float gl = 0.f;
           for (int m = lane; m < M; m += 32) {
-            const float nx = in_topk(G, M, K, m) ? 1.f : 0.f;
+            const float nx = in_topk(Gk, M, K, m) ? 1.f : 0.f;
             gl += G[m] * (nx - x[i * M + m]);
           }
           const float gain = warp_total(gl);
           if (gain > a.tol * fmaxf(J, 1e-8f)) {   // uniform across the warp
-            for (int m = lane; m < M; m += 32) x[i * M + m] = in_topk(G, M, K, m) ? 1.f : 0.f;
+            for (int m = lane; m < M; m += 32) x[i * M + m] = in_topk(Gk, M, K, m) ? 1.f : 0.f;
             J -= gain;
             changed = true;
           }
@@ -546,8 +584,10 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
 }  // namespace
 
 size_t route_head_smem_bytes(const cast_route_args& a) {
-  return ((size_t)2 * a.n_anchors * a.d + (size_t)3 * a.n_anchors * a.M + (size_t)a.M +
-          (size_t)kHeadWarps * a.d) * sizeof(float);
+  const bool restricted = a.candidates != nullptr;
+  const size_t floats = (size_t)2 * a.n_anchors * a.d + (size_t)3 * a.n_anchors * a.M + (size_t)a.M +
+                        (restricted ? (size_t)a.M : 0) + (size_t)kHeadWarps * a.d;
+  return floats * sizeof(float) + (restricted ? align_up((size_t)a.n_anchors * a.M, 16) : 0);
 }
 
 namespace {
@@ -645,6 +685,8 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   ha.kbar = kbar;
   ha.vbar = vbar;
   ha.gram = a.gram;
+  ha.cand = a.candidates;
+  ha.Mc = a.candidates ? a.M_c : a.M;
   ha.idx = a.idx;
   ha.u_out = a.u;
   ha.H = a.H;
@@ -709,6 +751,18 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   hc.numAttrs = 1;
   if (cudaLaunchKernelEx(&hc, k_head, ha) != cudaSuccess) return check_launch("routing head kernel");
   return check_launch("routing head kernel");
+}
+
+unsigned int route_error_word(cudaStream_t st, bool clear) {
+  unsigned int v = 0;
+  cudaMemcpyFromSymbolAsync(&v, g_route_error, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  cudaStreamSynchronize(st);
+  if (clear && v) {
+    const unsigned int z = 0;
+    cudaMemcpyToSymbolAsync(g_route_error, &z, sizeof(z), 0, cudaMemcpyHostToDevice, st);
+    cudaStreamSynchronize(st);
+  }
+  return v;
 }
 
 }  // namespace cast

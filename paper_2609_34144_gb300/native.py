@@ -41,7 +41,8 @@ class RouteArgs(C.Structure):
                 ("B_v", _i32), ("gram", _vp), ("K", _i32), ("eps", _f32), ("mode", _i32),
                 ("idx", _vp), ("u", _vp), ("qbar", _vp), ("kbar", _vp), ("vbar", _vp),
                 ("k_eff", C.POINTER(_i32)), ("refine_passes", _i32), ("lambda_anc", _f32),
-                ("lambda_rec", _f32), ("refine_tol", _f32), ("hist", HistLayout)]
+                ("lambda_rec", _f32), ("refine_tol", _f32), ("hist", HistLayout),
+                ("candidates", _vp), ("M_c", _i32)]
 
 
 class AttnArgs(C.Structure):
@@ -75,7 +76,8 @@ class BlockArgs(C.Structure):
                 ("route_lambda_rec", _f32), ("route_refine_tol", _f32), ("scale", _f32),
                 ("r_out", _vp), ("r_dtype", _i32),
                 ("x", _vp), ("idx_out", _vp), ("channel_weight", _vp), ("par", ParParams),
-                ("w_o", _vp), ("b_o", _vp), ("hist", HistLayout)]
+                ("w_o", _vp), ("b_o", _vp), ("hist", HistLayout), ("route_candidates", _vp),
+                ("route_M_c", _i32)]
 
 
 class FfnArgs(C.Structure):
@@ -215,8 +217,17 @@ def default_par_params():
 REFINE_PAPER = dict(passes=2, lambda_anc=1.0, lambda_rec=1.0, tol=1e-6)   # Tab. config_cast
 
 
+def _candidates(candidates):
+    """Device int32 [K_f, H, M_c] candidate sets (App. B.3) -> (pointer, M_c)."""
+    if candidates is None:
+        return None, 0
+    if candidates.dtype != torch.int32 or candidates.dim() != 3 or not candidates.is_contiguous():
+        raise ValueError("candidates must be a contiguous int32 [K_f, H, M_c] tensor")
+    return _ptr(candidates), candidates.shape[2]
+
+
 def _route_args(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_OMISSION,
-                refine=None):
+                refine=None, candidates=None):
     N, S, H, d = q.shape
     M, B_v, rs, lay = _history(k_hist, H, d)
     a = RouteArgs()
@@ -231,22 +242,25 @@ def _route_args(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_O
     a.M, a.B_v, a.hist = M, B_v if M > 0 else k_hist.shape[1], lay
     a.gram = _ptr(gram)
     a.K, a.eps, a.mode = K, eps, mode
+    a.candidates, a.M_c = _candidates(candidates)
     if refine:
         a.refine_passes, a.lambda_anc = refine["passes"], refine["lambda_anc"]
         a.lambda_rec, a.refine_tol = refine["lambda_rec"], refine["tol"]
     return a
 
 
-def route_workspace_size(q, anchors, k_hist, v_hist, K, refine=None):
-    a = _route_args(q, anchors, k_hist, v_hist, K, refine=refine)
+def route_workspace_size(q, anchors, k_hist, v_hist, K, refine=None, candidates=None):
+    a = _route_args(q, anchors, k_hist, v_hist, K, refine=refine, candidates=candidates)
     return _lib.cast_route_topk and _lib.cast_route_workspace_size(C.byref(a))
 
 
 def cast_route_topk(q, anchors, k_hist, v_hist, K, gram=None, eps=1e-8, mode=ROUTE_OMISSION,
-                    want_u=False, want_pooled=False, workspace=None, stream=None, refine=None):
+                    want_u=False, want_pooled=False, workspace=None, stream=None, refine=None,
+                    candidates=None):
     """Returns idx [K_f, H, K_eff] int32 (and u, (qbar, kbar, vbar) when asked).  refine: None
-    (independent TopK) or a dict like REFINE_PAPER (coupled refinement, Alg. routing)."""
-    a = _route_args(q, anchors, k_hist, v_hist, K, gram, eps, mode, refine)
+    (independent TopK) or a dict like REFINE_PAPER (coupled refinement, Alg. routing);
+    candidates: None (every block) or device int32 [K_f, H, M_c] fixed candidate sets."""
+    a = _route_args(q, anchors, k_hist, v_hist, K, gram, eps, mode, refine, candidates)
     Kf, H, d, M = len(anchors), q.shape[2], q.shape[3], a.M
     keff = min(K, M)
     dev = q.device
@@ -359,7 +373,7 @@ def cast_par_reconstruct(r, anchor_mask, channel_weight=None, params=None, works
 # --------------------------------------------------------------------------- block step
 def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None, idx_out=None,
                gram=None, route_eps=1e-8, route_mode=ROUTE_OMISSION, scale=0.0,
-               channel_weight=None, params=None, refine=None, w_o=None, b_o=None):
+               channel_weight=None, params=None, refine=None, w_o=None, b_o=None, candidates=None):
     N, S, H, d = q.shape
     M, B_v, rs, lay = _history(k_hist, H, d)
     a = BlockArgs()
@@ -382,6 +396,8 @@ def block_args(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=None,
     a.channel_weight = _ptr(channel_weight)
     a.par = params if params is not None else default_par_params()
     a.w_o, a.b_o = _ptr(w_o), _ptr(b_o)
+    a.route_candidates, a.route_M_c = _candidates(candidates)
+    a._keep = (candidates,)
     return a
 
 

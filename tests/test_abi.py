@@ -280,3 +280,13 @@ def test_struct_layouts_match_the_header(lib, tmp_path):
         py = structs[cname]
         got = C.sizeof(py) if fname == "sizeof" else getattr(py, fname).offset
         assert got == int(val), (cname, fname, got, int(val))
+
+
+@pytest.mark.parametrize("M_c,status", [(1, 1), (2, 0), (4, 0), (5, 1)])
+def test_route_candidate_set_size_validation(lib, M_c, status):
+    a = _route(lib)                  # M = 4, K = 2
+    a.candidates, a.M_c = _fake(0x50000), M_c
+    so = lib.library()
+    assert so.cast_route_topk(C.byref(a), None, 0, None) == 1
+    msg = so.cast_last_error_detail()
+    assert (b"M_c" in msg) == bool(status), msg

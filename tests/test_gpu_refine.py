@@ -25,22 +25,25 @@ def _mask(idx, M):
     return x
 
 
-def check_refined(idx_gpu, u, anchors, n_frames, K, refine):
-    """Compare [K_f, H, K_eff] refined indices with the oracle per head; returns
-    (#heads the refinement changed, #ambiguous heads)."""
+def check_refined(idx_gpu, u, anchors, n_frames, K, refine, candidates=None):
+    """Compare [K_f, H, K_eff] refined indices with the oracle per head (candidates: optional
+    [K_f, H, M_c] fixed sets); returns (#heads the refinement changed, #ambiguous heads)."""
     Kf, H, M = u.shape
     keff = min(K, M)
     changed = amb = 0
     for h in range(H):
         uh = u[:, h, :].astype(np.float64)
+        ch = None if candidates is None else candidates[:, h, :]
         ref, info = O.coupled_routing(uh, anchors, n_frames, K, passes=refine["passes"],
                                       lam_anc=refine["lambda_anc"], lam_rec=refine["lambda_rec"],
-                                      tol=refine["tol"], with_info=True)
+                                      tol=refine["tol"], with_info=True, candidates=ch)
         g = idx_gpu[:, h, :]
         assert g.shape == (Kf, keff)
         for i in range(Kf):
             assert np.all(np.diff(g[i]) > 0) and g[i].min() >= 0 and g[i].max() < M
-        changed += int(not np.array_equal(ref, O.topk_blocks(uh, K)))
+            if ch is not None:
+                assert set(g[i].tolist()) <= set(ch[i].tolist())
+        changed += int(not np.array_equal(ref, O.topk_blocks(uh, K, candidates=ch)))
         if not info["ambiguous"]:
             assert np.array_equal(g, ref), (h, g, ref)
         else:
