@@ -150,8 +150,9 @@ typedef struct {
  * index outside [0, M) or repeated within a set makes the kernel record an error that
  * cast_check_device() reports as INVALID_ARG (that set then holds fewer members and its
  * selection is completed by the lowest-index other blocks); UNSUPPORTED for d not 64/128, M > 16384,
- * H*d > 51200 channels (pooling shared memory) or 4*(2*K_f*d + 3*K_f*M + M + 8*d) bytes of
- * per-head state above 200 KB. */
+ * H*d > 51200 channels (pooling shared memory) or a per-head routing state above 200 KB of
+ * shared memory (about 8 K_f M bytes, 12 K_f M with refinement, plus K_f M with candidate
+ * sets, and 4 K_f d + 36 KB for the statistics). */
 cast_status cast_route_topk(const cast_route_args* args, void* workspace,
                             size_t workspace_bytes, void* stream);
 size_t cast_route_workspace_size(const cast_route_args* args);

@@ -52,7 +52,10 @@ inline HistGeom hist_geom(const cast_hist_layout& h) {
 // ------------------------------------------------------------------ routing
 struct RoutePlan {
   int n_seg;        // n_anchors + 2 M pooled segments
-  int nsplit;       // row splits per segment (CTAs of one cluster)
+  int nsplit_q;     // row splits of an anchor-frame segment (CTAs of one cluster)
+  int nsplit_kv;    // row splits of a history-block segment
+  bool wide;        // per-head statistics spread over a cluster of CTAs (large M)
+  int cl;           // CTAs per head in the wide form
   size_t pooled_bytes, total_bytes;
 };
 RoutePlan route_plan(const cast_route_args& a);

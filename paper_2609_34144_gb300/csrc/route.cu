@@ -49,6 +49,7 @@ struct PoolArgs {
   float* vbar;            // [M, D]
   int64_t q_row_stride, hist_row_stride;   // elements
   int n_anchors, M, S, B_v, D, nsplit, elt;
+  int seg_base;           // segment of blockIdx.y == 0 (anchor frames first, then K, then V blocks)
   int Hg, Wg, nby, nbx;   // CAST_HIST_FRAMES: history frame grid and its 8x8 block grid
   int anchors[CAST_MAX_ANCHORS];
 };
@@ -85,6 +86,13 @@ __device__ __forceinline__ float ld_dsmem(const float* local, uint32_t rank) {
   asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
   return v;
 }
+__device__ __forceinline__ void st_dsmem(float* local, uint32_t rank, float v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+               : "=r"(remote)
+               : "r"((uint32_t)__cvta_generic_to_shared(local)), "r"(rank));
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+}
 __device__ __forceinline__ void grid_dependency_wait() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
 }
@@ -101,7 +109,7 @@ __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant_
   constexpr int VEC = 16 / sizeof(T);
   extern __shared__ float colsum[];
   launch_dependents();
-  const int seg = blockIdx.y, split = blockIdx.x;
+  const int seg = blockIdx.y + a.seg_base, split = blockIdx.x;
   const char* base;
   int64_t rs;
   int nrows;
@@ -229,6 +237,9 @@ __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant_
     out[c] = s * inv;
   }
   cluster_sync_all();   // no CTA leaves while a peer still reads its shared memory
+  // launched as a programmatic dependent of the anchor-frame pooling: this grid completes only
+  // after that one has, so its own dependents see every mean
+  grid_dependency_wait();
 }
 
 // ---------------------------------------------------------------------- per-head kernel
@@ -581,23 +592,555 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
   }
 }
 
-}  // namespace
+// ---------------------------------------------------------------------- wide per-head kernel
+// For many history blocks (k_bar, v_bar of a head too large for one CTA's shared memory) the
+// statistics of one head are spread over a cluster of cl CTAs, each owning a contiguous range
+// of mr blocks: scores, the softmax max and sum, o_bar partial sums and the omission scores
+// are exchanged through distributed shared memory (reduced in rank order).  The rank-0 CTA
+// then gathers every anchor's scores and runs the TopK selections and the refinement passes
+// with all its threads; each TopK is an exact radix select on a 46-bit key (the score's order
+// bits, then the inverted block index, so that ties go to the lower index).
+constexpr int kWideThreads = 256, kWideWarps = kWideThreads / 32;
+constexpr int kWideMaxCl = 8, kWideGroup = 8;   // CTAs per head; anchors per o_bar pass
+constexpr int kWideRows = 8;                    // history blocks a warp loads at once
+constexpr int kRadixBins = 1024;                // 10-bit digits of the TopK radix select
 
-size_t route_head_smem_bytes(const cast_route_args& a) {
+__host__ __device__ inline uint32_t take_smem(size_t& o, size_t bytes) {
+  const size_t r = o;
+  o += (bytes + 15) & ~(size_t)15;
+  return (uint32_t)r;
+}
+
+// Byte offsets of the wide kernel's shared memory.  The o_bar partials of the warps share
+// their space with the rank-0 arrays, which are only written after the partials are reduced.
+struct WideLayout {
+  uint32_t qb, ob, obp, red, sl, pl, ew, coef, owp, u, x, sq, G, red2, hist, pre, cm;
+  size_t total;
+};
+__host__ __device__ inline WideLayout wide_layout(int na, int M, int d, int mr, bool refine,
+                                                  bool restricted) {
+  WideLayout L{};
+  size_t o = 0;
+  const size_t naf = (size_t)na * sizeof(float);
+  L.qb = take_smem(o, naf * d);
+  L.ob = take_smem(o, naf * d);
+  L.obp = take_smem(o, naf * d);
+  L.red = take_smem(o, 2 * naf);
+  L.sl = take_smem(o, naf * mr);
+  L.pl = take_smem(o, naf * mr);
+  L.ew = take_smem(o, (size_t)kWideWarps * d * sizeof(float));
+  L.coef = take_smem(o, 3 * naf);
+  const size_t region = o;
+  L.owp = (uint32_t)region;
+  const size_t owp_end = region + (size_t)kWideWarps * kWideGroup * d * sizeof(float);
+  L.u = take_smem(o, naf * M);
+  L.x = take_smem(o, naf * M);
+  L.sq = refine ? take_smem(o, naf * M) : 0;
+  L.G = take_smem(o, (size_t)M * sizeof(float));
+  L.red2 = take_smem(o, 64 * sizeof(float));
+  L.hist = take_smem(o, (size_t)2 * kRadixBins * sizeof(unsigned));
+  L.pre = take_smem(o, 4 * sizeof(unsigned long long));
+  L.cm = restricted ? take_smem(o, (size_t)na * M) : 0;
+  L.total = o > owp_end ? o : owp_end;
+  return L;
+}
+
+inline int wide_cluster(int M) {
+  const int cl = (M + 63) / 64;
+  return cl > kWideMaxCl ? kWideMaxCl : (cl < 1 ? 1 : cl);
+}
+
+// Order key of score v at block m (M <= 16384): larger key = selected first; -0 ranks as +0,
+// -inf (outside a candidate set) below every finite score.
+__device__ __forceinline__ unsigned long long order_key(float v, int m) {
+  uint32_t b = __float_as_uint(v == 0.f ? 0.f : v);
+  b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+  return ((unsigned long long)b << 14) | (unsigned long long)(16383 - m);
+}
+__device__ __forceinline__ float masked(const float* key, const uint8_t* cm, int p) {
+  return (cm && !cm[p]) ? -INFINITY : key[p];
+}
+
+// Radix select of the TopK threshold of one row key[0..M) (entries with cm[m] == 0 count as
+// -inf; 0 < K < M): returns the order key t such that exactly K keys of the row have
+// order_key >= t.  Rounds of 10-bit digits from the top of the 46-bit key; a round whose
+// chosen digit holds exactly the remaining count ends the select (its lower bits are then
+// left zero).  hist holds two 1024-bin buffers, zero on entry and zero again on return; each
+// round's buffer is cleared during the round after it.  Every thread of the CTA calls this.
+__device__ unsigned long long topk_threshold(const float* key, const uint8_t* cm, int M, int K,
+                                             unsigned* hist2, unsigned long long* sel) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  unsigned long long pre = 0ull;
+  int krem = K;
+  int round = 0;
+  for (int shift = 36;; shift = shift >= 10 ? shift - 10 : 0, ++round) {
+    const int width = shift == 0 ? 6 : 10;   // bits 45..36, 35..26, 25..16, 15..6, 5..0
+    // (the last round's 6-bit digit uses bins 0..63 of the same 1024)
+    unsigned* hist = hist2 + (round & 1) * kRadixBins;
+    if (round > 0)   // the previous round's buffer is free again (read before the last barrier)
+      for (int e = tid; e < kRadixBins; e += kWideThreads) hist2[((round - 1) & 1) * kRadixBins + e] = 0u;
+    const unsigned long long hi = ~0ull << (shift + width);
+    for (int m = tid; m < M; m += kWideThreads) {
+      const unsigned long long c = order_key(cm && !cm[m] ? -INFINITY : key[m], m);
+      if ((c & hi) == pre) atomicAdd(&hist[(int)((c >> shift) & (unsigned long long)(kRadixBins - 1))], 1u);
+    }
+    __syncthreads();
+    if (tid < 32) {
+      // the digit where the count from the top reaches krem: lane l first sums the 32 bins
+      // 1023-32l .. 992-32l (rotated so the lanes hit different banks), a warp scan picks the
+      // chunk, then the warp scans that chunk's bins
+      unsigned part = 0;
+#pragma unroll 8
+      for (int t = 0; t < 32; ++t) part += hist[kRadixBins - 1 - 32 * lane - ((t + lane) & 31)];
+      unsigned inc = part;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned w = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += w;
+      }
+      const int l = __ffs(__ballot_sync(0xffffffffu, inc >= (unsigned)krem)) - 1;
+      const unsigned carry = __shfl_sync(0xffffffffu, inc - part, l);
+      const int b = kRadixBins - 1 - 32 * l - lane;
+      const unsigned v = hist[b];
+      unsigned inc2 = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned w = __shfl_up_sync(0xffffffffu, inc2, o);
+        if (lane >= o) inc2 += w;
+      }
+      const int j = __ffs(__ballot_sync(0xffffffffu, carry + inc2 >= (unsigned)krem)) - 1;
+      if (lane == j) {
+        const unsigned before = carry + inc2 - v;
+        sel[0] = pre | ((unsigned long long)b << shift);
+        sel[1] = (unsigned long long)(krem - (int)before);
+        sel[2] = (v == (unsigned)krem - before || shift == 0) ? 1ull : 0ull;
+      }
+    }
+    __syncthreads();
+    pre = sel[0];
+    krem = (int)sel[1];
+    const bool done = sel[2] != 0ull;
+    if (done) {
+      // clear this round's buffer before leaving (the other one is already zero)
+      for (int e = tid; e < kRadixBins; e += kWideThreads) hist[e] = 0u;
+      __syncthreads();
+      return pre;
+    }
+  }
+}
+
+// Deterministic CTA-wide sum (warp sums added in warp order); every thread gets the total.
+// red2 holds two slot sets used alternately (`slot` flips between calls), so a call never
+// overwrites partials a slower thread is still adding from the previous call.
+__device__ __forceinline__ float block_sum(float v, float* red2, int& slot) {
+  v = warp_sum(v);
+  float* r = red2 + slot * kWideWarps;
+  slot ^= 1;
+  if ((threadIdx.x & 31) == 0) r[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float t = 0.f;
+#pragma unroll
+  for (int w = 0; w < kWideWarps; ++w) t += r[w];
+  return t;
+}
+
+// Sums each of v[0..7] over the 32 lanes with 9 shuffles (halving the set at each of the first
+// three steps); on return lane l holds the total of v[(l >> 2) & 7].
+__device__ __forceinline__ float warp_sum8(float (&v)[8]) {
+  const int lane = threadIdx.x & 31;
+  float w[4], y[2];
+  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float keep = b4 ? v[j + 4] : v[j], give = b4 ? v[j] : v[j + 4];
+    w[j] = keep + __shfl_xor_sync(0xffffffffu, give, 16);
+  }
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const float keep = b3 ? w[j + 2] : w[j], give = b3 ? w[j] : w[j + 2];
+    y[j] = keep + __shfl_xor_sync(0xffffffffu, give, 8);
+  }
+  float z = (b2 ? y[1] : y[0]) + __shfl_xor_sync(0xffffffffu, b2 ? y[0] : y[1], 4);
+  z += __shfl_xor_sync(0xffffffffu, z, 2);
+  z += __shfl_xor_sync(0xffffffffu, z, 1);
+  return z;
+}
+
+template <int NP>
+__device__ __forceinline__ void load_row(const float* p, float (&v)[NP]) {
+  if constexpr (NP == 4) {
+    const float4 t = __ldcg(reinterpret_cast<const float4*>(p));
+    v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+  } else {
+    const float2 t = __ldcg(reinterpret_cast<const float2*>(p));
+    v[0] = t.x; v[1] = t.y;
+  }
+}
+
+// grid (cl, H), cluster (cl, 1, 1), kWideThreads threads; lane l of a warp holds channels
+// l*NP .. l*NP+NP-1 of a head vector (HD = 32 NP).
+template <int HD>
+__global__ void __launch_bounds__(kWideThreads) k_head_wide(const __grid_constant__ HeadArgs a) {
+  constexpr int NP = HD / 32;
+  extern __shared__ __align__(16) uint8_t wsm[];
+  const int rank = blockIdx.x, cl = gridDim.x, h = blockIdx.y;
+  const int na = a.n_anchors, M = a.M, K = a.K_eff, D = a.H * HD;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool restricted = a.cand != nullptr;
+  const bool refine = a.passes > 0 && K > 0 && K < M;
+  const int mr = (M + cl - 1) / cl;
+  const int m0 = min(M, rank * mr), m1 = min(M, m0 + mr), nm = m1 - m0;
+  const WideLayout L = wide_layout(na, M, HD, mr, refine, restricted);
+  float* qb = reinterpret_cast<float*>(wsm + L.qb);
+  float* ob = reinterpret_cast<float*>(wsm + L.ob);
+  float* obp = reinterpret_cast<float*>(wsm + L.obp);
+  float* red = reinterpret_cast<float*>(wsm + L.red);
+  float* sl = reinterpret_cast<float*>(wsm + L.sl);    // [na][mr] scores s of this CTA's blocks
+  float* pl = reinterpret_cast<float*>(wsm + L.pl);    // [na][mr] pi, then the omission score u
+  float* ew = reinterpret_cast<float*>(wsm + L.ew);
+  const float* kbar = a.kbar + h * HD;
+  const float* vbar = a.vbar + h * HD;
+  launch_dependents();
+  grid_dependency_wait();   // the pooled means come from the preceding kernels
+  for (int e = tid; e < na * (HD / 4); e += kWideThreads) {
+    const int i = e / (HD / 4), c = (e - i * (HD / 4)) * 4;
+    *reinterpret_cast<float4*>(qb + i * HD + c) =
+        __ldcg(reinterpret_cast<const float4*>(a.qbar + (int64_t)i * D + h * HD + c));
+  }
+  __syncthreads();
+  // s_{i,m} = q_bar_i . k_bar_m / sqrt(d)  (Eq. pooled): a warp takes kWideRows blocks at once
+  const float scale = rsqrtf((float)HD);
+  for (int mb = m0 + warp * kWideRows; mb < m1; mb += kWideWarps * kWideRows) {
+    float kv[kWideRows][NP];
+#pragma unroll
+    for (int t = 0; t < kWideRows; ++t) {
+      if (mb + t < m1) load_row<NP>(kbar + (int64_t)(mb + t) * D + lane * NP, kv[t]);
+      else
+#pragma unroll
+        for (int k = 0; k < NP; ++k) kv[t][k] = 0.f;
+    }
+    for (int i = 0; i < na; ++i) {
+      float qv[NP], p[kWideRows];
+#pragma unroll
+      for (int k = 0; k < NP; ++k) qv[k] = qb[i * HD + lane * NP + k];
+#pragma unroll
+      for (int t = 0; t < kWideRows; ++t) {
+        p[t] = 0.f;
+#pragma unroll
+        for (int k = 0; k < NP; ++k) p[t] = fmaf(qv[k], kv[t][k], p[t]);
+      }
+      const float tot = warp_sum8(p);   // row (lane >> 2) & 7 of the batch
+      const int t = (lane >> 2) & 7;
+      if ((lane & 3) == 0 && mb + t < m1) sl[i * mr + (mb + t - m0)] = tot * scale;
+    }
+  }
+  __syncthreads();
+  // pi_i = softmax over all M blocks: cluster-wide max, then sum (both in rank order)
+  for (int i = warp; i < na; i += kWideWarps) {
+    float mx = -INFINITY;
+    for (int m = lane; m < nm; m += 32) mx = fmaxf(mx, sl[i * mr + m]);
+    mx = warp_max(mx);
+    if (lane == 0) red[i] = mx;
+  }
+  cluster_sync_all();
+  for (int i = warp; i < na; i += kWideWarps) {
+    float gm = -INFINITY;
+    for (int r = 0; r < cl; ++r) gm = fmaxf(gm, ld_dsmem(red + i, (uint32_t)r));
+    float tot = 0.f;
+    for (int m = lane; m < nm; m += 32) {
+      const float e = expf(sl[i * mr + m] - gm);
+      pl[i * mr + m] = e;
+      tot += e;
+    }
+    tot = warp_sum(tot);
+    if (lane == 0) red[na + i] = tot;
+  }
+  cluster_sync_all();
+  for (int i = warp; i < na; i += kWideWarps) {
+    float tot = 0.f;
+    for (int r = 0; r < cl; ++r) tot += ld_dsmem(red + na + i, (uint32_t)r);
+    const float inv = 1.f / tot;
+    for (int m = lane; m < nm; m += 32) pl[i * mr + m] *= inv;
+  }
+  __syncthreads();
+  // o_bar_i = sum_m pi_{i,m} v_bar_m: per-warp partials (kWideGroup anchors per pass), summed
+  // over warps in order, then over the cluster's CTAs in rank order
+  float* owp = reinterpret_cast<float*>(wsm + L.owp);
+  for (int g0 = 0; g0 < na; g0 += kWideGroup) {
+    const int ng = min(kWideGroup, na - g0);
+    float acc[kWideGroup][NP];
+#pragma unroll
+    for (int g = 0; g < kWideGroup; ++g)
+#pragma unroll
+      for (int k = 0; k < NP; ++k) acc[g][k] = 0.f;
+    for (int mb = m0 + warp * kWideRows; mb < m1; mb += kWideWarps * kWideRows) {
+      float vv[kWideRows][NP];
+#pragma unroll
+      for (int t = 0; t < kWideRows; ++t) {
+        if (mb + t < m1) load_row<NP>(vbar + (int64_t)(mb + t) * D + lane * NP, vv[t]);
+        else
+#pragma unroll
+          for (int k = 0; k < NP; ++k) vv[t][k] = 0.f;
+      }
+#pragma unroll
+      for (int g = 0; g < kWideGroup; ++g) {
+        if (g < ng) {
+#pragma unroll
+          for (int t = 0; t < kWideRows; ++t) {
+            const float w = mb + t < m1 ? pl[(g0 + g) * mr + (mb + t - m0)] : 0.f;
+#pragma unroll
+            for (int k = 0; k < NP; ++k) acc[g][k] = fmaf(w, vv[t][k], acc[g][k]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int g = 0; g < kWideGroup; ++g)
+#pragma unroll
+      for (int k = 0; k < NP; ++k) owp[(warp * kWideGroup + g) * HD + lane * NP + k] = acc[g][k];
+    __syncthreads();
+    for (int e = tid; e < ng * HD; e += kWideThreads) {
+      const int g = e / HD, c = e - g * HD;
+      float t = 0.f;
+      for (int w = 0; w < kWideWarps; ++w) t += owp[(w * kWideGroup + g) * HD + c];
+      obp[(g0 + g) * HD + c] = t;
+    }
+    __syncthreads();
+  }
+  cluster_sync_all();
+  for (int e = tid; e < na * HD; e += kWideThreads) {
+    float t = 0.f;
+    for (int r = 0; r < cl; ++r) t += ld_dsmem(obp + e, (uint32_t)r);
+    ob[e] = t;
+  }
+  __syncthreads();
+  // delta_{i,m} = pi/(1 - pi + eps) (o_bar_i - v_bar_m);  u = delta^T G delta  (Eq. omission)
+  if (a.mode == CAST_ROUTE_OMISSION && a.gram == nullptr) {
+    for (int mb = m0 + warp * kWideRows; mb < m1; mb += kWideWarps * kWideRows) {
+      float vv[kWideRows][NP];
+#pragma unroll
+      for (int t = 0; t < kWideRows; ++t) {
+        if (mb + t < m1) load_row<NP>(vbar + (int64_t)(mb + t) * D + lane * NP, vv[t]);
+        else
+#pragma unroll
+          for (int k = 0; k < NP; ++k) vv[t][k] = 0.f;
+      }
+      for (int i = 0; i < na; ++i) {
+        float ov[NP], acc[kWideRows];
+#pragma unroll
+        for (int k = 0; k < NP; ++k) ov[k] = ob[i * HD + lane * NP + k];
+#pragma unroll
+        for (int t = 0; t < kWideRows; ++t) {
+          acc[t] = 0.f;
+#pragma unroll
+          for (int k = 0; k < NP; ++k) {
+            const float df = ov[k] - vv[t][k];
+            acc[t] = fmaf(df, df, acc[t]);
+          }
+        }
+        const float tot = warp_sum8(acc);   // row (lane >> 2) & 7 of the batch
+        const int t = (lane >> 2) & 7;
+        if ((lane & 3) == 0 && mb + t < m1) {
+          const int q = i * mr + (mb + t - m0);
+          const float coef = pl[q] / (1.f - pl[q] + a.eps);
+          pl[q] = coef * coef * tot;
+        }
+      }
+    }
+  } else if (a.mode == CAST_ROUTE_OMISSION) {
+    float* e = ew + warp * HD;
+    const float* Gm = a.gram + (int64_t)h * HD * HD;
+    for (int m = m0 + warp; m < m1; m += kWideWarps) {
+      for (int i = 0; i < na; ++i) {
+        for (int c = lane; c < HD; c += 32) e[c] = ob[i * HD + c] - vbar[(int64_t)m * D + c];
+        __syncwarp();
+        float acc = 0.f;
+        for (int r = lane; r < HD; r += 32) {
+          float y = 0.f;
+          for (int c = 0; c < HD; ++c) y = fmaf(Gm[(int64_t)r * HD + c], e[c], y);
+          acc = fmaf(e[r], y, acc);
+        }
+        __syncwarp();
+        acc = warp_sum(acc);
+        if (lane == 0) {
+          const int q = i * mr + (m - m0);
+          const float coef = pl[q] / (1.f - pl[q] + a.eps);
+          pl[q] = coef * coef * acc;
+        }
+      }
+    }
+  }
+  __syncthreads();
+  // every CTA pushes its keys into rank 0's u[na][M] (that space held o_bar partials, which
+  // every CTA finished with before the last cluster barrier); the barrier below publishes them
+  const float* keyl = a.mode == CAST_ROUTE_OMISSION ? pl : sl;   // the TopK key of Eq. (topk)
+  float* u = reinterpret_cast<float*>(wsm + L.u);
+  for (int e = tid; e < na * nm; e += kWideThreads) {
+    const int i = e / nm, ml = e - i * nm;
+    const float v = keyl[i * mr + ml];
+    if (a.u_out) a.u_out[((int64_t)i * a.H + h) * M + m0 + ml] = v;
+    if (K > 0) st_dsmem(u + i * M + m0 + ml, 0u, v);
+  }
+  cluster_sync_all();
+  if (rank != 0 || K == 0) return;
+
+  float* x = reinterpret_cast<float*>(wsm + L.x);
+  float* G = reinterpret_cast<float*>(wsm + L.G);
+  float* red2 = reinterpret_cast<float*>(wsm + L.red2);
+  unsigned* hist = reinterpret_cast<unsigned*>(wsm + L.hist);
+  unsigned long long* sel = reinterpret_cast<unsigned long long*>(wsm + L.pre);
+  uint8_t* cm = restricted ? wsm + L.cm : nullptr;
+  // candidate sets C_i (App. B.3): membership bytes; keys outside C_i count as -inf
+  if (restricted) {
+    for (int p = tid; p < na * M; p += kWideThreads) cm[p] = 0;
+    __syncthreads();
+    for (int e = tid; e < na * a.Mc; e += kWideThreads) {
+      const int i = e / a.Mc, c = e - i * a.Mc;
+      const int m = __ldg(a.cand + ((int64_t)i * a.H + h) * a.Mc + c);
+      if (m < 0 || m >= M) atomicExch(&g_route_error, 1u);
+      else cm[i * M + m] = 1;
+    }
+    __syncthreads();
+    for (int i = warp; i < na; i += kWideWarps) {
+      int n = 0;
+      for (int m = lane; m < M; m += 32) n += cm[i * M + m];
+      n = __reduce_add_sync(0xffffffffu, n);
+      if (lane == 0 && n != a.Mc) atomicExch(&g_route_error, 1u);
+    }
+  }
+  for (int e = tid; e < 2 * kRadixBins; e += kWideThreads) hist[e] = 0u;
+  int slot = 0;
+  __syncthreads();
+  // initial masks: TopK of each anchor's key (Eq. topk), within C_i
+  if (K >= M) {
+    for (int p = tid; p < na * M; p += kWideThreads) x[p] = 1.f;
+  } else {
+    for (int i = 0; i < na; ++i) {
+      const uint8_t* cmi = cm ? cm + i * M : nullptr;
+      const unsigned long long t = topk_threshold(u + i * M, cmi, M, K, hist, sel);
+      for (int m = tid; m < M; m += kWideThreads)
+        x[i * M + m] = order_key(masked(u + i * M, cmi, m), m) >= t ? 1.f : 0.f;
+    }
+  }
+  __syncthreads();
+  if (refine) {
+    // Alg. (routing) with the whole CTA: sq[j][m] = sqrt(u_{j-1,m} u_{j,m}); interval
+    // coefficients A, B, C of Eq. (abc); boundary sets from the pairs (0, 1) and (na-2, na-1)
+    float* sq = reinterpret_cast<float*>(wsm + L.sq);
+    float* cA = reinterpret_cast<float*>(wsm + L.coef);
+    float* cB = cA + na;
+    float* cC = cA + 2 * na;
+    for (int p = tid; p < na * M; p += kWideThreads)
+      if (p >= M) sq[p] = sqrtf(u[p - M] * u[p]);
+    for (int j = tid; j < na; j += kWideThreads) {
+      cA[j] = a.A[j];
+      cB[j] = a.B[j];
+      cC[j] = a.C[j];
+    }
+    __syncthreads();
+    const float AL = a.AL, BL = a.BL, CL = a.CL, AR = a.AR, BR = a.BR, CR = a.CR;
+    const float lam_anc = a.lam_anc, lam_rec = a.lam_rec;
+    float Jl = 0.f;
+    for (int m = tid; m < M; m += kWideThreads) {
+      for (int i = 0; i < na; ++i) Jl += lam_anc * (1.f - x[i * M + m]) * u[i * M + m];
+      float rec = 0.f;
+      for (int j = 1; j < na; ++j) {
+        const float xp = 1.f - x[(j - 1) * M + m], xq = 1.f - x[j * M + m];
+        rec += cA[j] * xp * u[(j - 1) * M + m] + cB[j] * xq * u[j * M + m] + 2.f * cC[j] * xp * xq * sq[j * M + m];
+      }
+      if (na >= 2) {
+        const float x0 = 1.f - x[m], x1 = 1.f - x[M + m];
+        rec += AL * x0 * u[m] + BL * x1 * u[M + m] + 2.f * CL * x0 * x1 * sq[M + m];
+        const int r0 = (na - 2) * M + m, r1 = (na - 1) * M + m;
+        const float y0 = 1.f - x[r0], y1 = 1.f - x[r1];
+        rec += AR * y0 * u[r0] + BR * y1 * u[r1] + 2.f * CR * y0 * y1 * sq[r1];
+      }
+      Jl += lam_rec * rec;
+    }
+    float J = block_sum(Jl, red2, slot);
+    for (int pass = 1; pass <= a.passes; ++pass) {
+      bool changed = false;
+      for (int step = 0; step < na; ++step) {
+        const int i = (pass & 1) ? step : na - 1 - step;
+        // retain gains, Eqs. (gain) and (boundarygain)
+        for (int m = tid; m < M; m += kWideThreads) {
+          const float ui = u[i * M + m];
+          float rec = 0.f;
+          if (i >= 1) rec += cB[i] * ui + 2.f * cC[i] * (1.f - x[(i - 1) * M + m]) * sq[i * M + m];
+          if (i + 1 < na) rec += cA[i + 1] * ui + 2.f * cC[i + 1] * (1.f - x[(i + 1) * M + m]) * sq[(i + 1) * M + m];
+          if (na >= 2) {
+            if (i == 0) rec += AL * ui + 2.f * CL * (1.f - x[M + m]) * sq[M + m];
+            if (i == 1) rec += BL * ui + 2.f * CL * (1.f - x[m]) * sq[M + m];
+            if (i == na - 2) rec += AR * ui + 2.f * CR * (1.f - x[(na - 1) * M + m]) * sq[(na - 1) * M + m];
+            if (i == na - 1) rec += BR * ui + 2.f * CR * (1.f - x[(na - 2) * M + m]) * sq[(na - 1) * M + m];
+          }
+          G[m] = lam_anc * ui + lam_rec * rec;
+        }
+        __syncthreads();
+        // best response TopK(G) within C_i and its gain sum_m G_m (x_new - x_i); J is affine in
+        // x_i, so the accepted step lowers J by exactly that gain
+        const uint8_t* cmi = cm ? cm + i * M : nullptr;
+        const unsigned long long thr = topk_threshold(G, cmi, M, K, hist, sel);
+        float gl = 0.f;
+        for (int m = tid; m < M; m += kWideThreads) {
+          const float nx = order_key(masked(G, cmi, m), m) >= thr ? 1.f : 0.f;
+          gl += G[m] * (nx - x[i * M + m]);
+        }
+        const float gain = block_sum(gl, red2, slot);
+        if (gain > a.tol * fmaxf(J, 1e-8f)) {   // uniform across the CTA
+          for (int m = tid; m < M; m += kWideThreads)
+            x[i * M + m] = order_key(masked(G, cmi, m), m) >= thr ? 1.f : 0.f;
+          J -= gain;
+          changed = true;
+        }
+        __syncthreads();
+      }
+      if (!changed) break;
+    }
+  }
+  __syncthreads();
+  // ascending block indices of every anchor's mask
+  for (int i = warp; i < na; i += kWideWarps) {
+    int base = 0;
+    int32_t* out = a.idx + ((int64_t)i * a.H + h) * K;
+    for (int mb = 0; mb < M; mb += 32) {
+      const int m = mb + lane;
+      const bool on = m < M && x[i * M + m] != 0.f;
+      const unsigned bal = __ballot_sync(0xffffffffu, on);
+      if (on) out[base + __popc(bal & ((1u << lane) - 1u))] = m;
+      base += __popc(bal);
+    }
+  }
+}
+
+// shared state of the single-CTA head kernel without the staged means
+size_t head_state_bytes(const cast_route_args& a) {
   const bool restricted = a.candidates != nullptr;
   const size_t floats = (size_t)2 * a.n_anchors * a.d + (size_t)3 * a.n_anchors * a.M + (size_t)a.M +
                         (restricted ? (size_t)a.M : 0) + (size_t)kHeadWarps * a.d;
   return floats * sizeof(float) + (restricted ? align_up((size_t)a.n_anchors * a.M, 16) : 0);
 }
 
-namespace {
 constexpr size_t kHeadSmemLimit = 200 * 1024;
-// k_bar and v_bar of one head join the shared state when everything fits
+// the single-CTA head kernel holds k_bar and v_bar of its head in shared memory
 size_t head_staged_bytes(const cast_route_args& a) {
-  return align_up(route_head_smem_bytes(a), 16) + (size_t)2 * a.M * a.d * sizeof(float);
+  return align_up(head_state_bytes(a), 16) + (size_t)2 * a.M * a.d * sizeof(float);
 }
 bool head_stages_kv(const cast_route_args& a) { return head_staged_bytes(a) <= kHeadSmemLimit; }
+
+size_t wide_bytes(const cast_route_args& a) {
+  const int K_eff = a.K < a.M ? a.K : a.M;
+  const int cl = wide_cluster(a.M);
+  const int mr = (a.M + cl - 1) / cl;
+  return wide_layout(a.n_anchors, a.M, a.d, mr, a.refine_passes > 0 && K_eff > 0 && K_eff < a.M,
+                     a.candidates != nullptr).total;
+}
+
 }  // namespace
+
+size_t route_head_smem_bytes(const cast_route_args& a) {
+  return head_stages_kv(a) ? head_staged_bytes(a) : wide_bytes(a);
+}
 
 size_t route_pool_smem_bytes(const cast_route_args& a) {
   const int D = a.H * a.d;
@@ -608,17 +1151,21 @@ RoutePlan route_plan(const cast_route_args& a) {
   RoutePlan p{};
   const int D = a.H * a.d;
   p.n_seg = a.n_anchors + 2 * a.M;
-  // a cluster of up to 8 CTAs per segment, enough CTAs to cover the SMs a few times, each
-  // streaming >= 64 rows
+  // per launch (anchor frames, history blocks): a cluster of up to 8 CTAs per segment, enough
+  // CTAs to cover the SMs a few times, each streaming >= 64 rows
   int dev = 0, nsm = 148;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
   const int target = 4 * (nsm > 0 ? nsm : 148);
-  int nsplit = (target + p.n_seg - 1) / p.n_seg;
-  if (nsplit > kMaxClusterSplit) nsplit = kMaxClusterSplit;
-  const int maxrows = a.M > 0 ? (a.S > a.B_v ? a.S : a.B_v) : a.S;
-  while (nsplit > 1 && (maxrows + nsplit - 1) / nsplit < 64) --nsplit;
-  if (nsplit < 1) nsplit = 1;
-  p.nsplit = nsplit;
+  auto splits = [&](int n_seg, int rows) {
+    int ns = n_seg > 0 ? (target + n_seg - 1) / n_seg : 1;
+    if (ns > kMaxClusterSplit) ns = kMaxClusterSplit;
+    while (ns > 1 && (rows + ns - 1) / ns < 64) --ns;
+    return ns < 1 ? 1 : ns;
+  };
+  p.nsplit_q = splits(a.n_anchors, a.S);
+  p.nsplit_kv = splits(2 * a.M, a.B_v);
+  p.wide = a.M > 0 && !head_stages_kv(a);
+  p.cl = p.wide ? wide_cluster(a.M) : 1;
   p.pooled_bytes = align_up((size_t)p.n_seg * D * sizeof(float));
   p.total_bytes = p.pooled_bytes;
   return p;
@@ -648,7 +1195,6 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   pa.S = a.S;
   pa.B_v = a.B_v;
   pa.D = D;
-  pa.nsplit = p.nsplit;
   pa.elt = a.dtype == CAST_BF16 ? 2 : 4;
   const HistGeom hg = hist_geom(a.hist);
   pa.Hg = hg.Hg;
@@ -664,21 +1210,31 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
       cudaFuncSetAttribute(pool_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psm) != cudaSuccess)
     return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory for pooling", psm);
   const PoolShape ps = pool_shape(D, pa.elt);
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(p.nsplit, p.n_seg, 1);
-  cfg.blockDim = dim3(ps.cgs * ps.lanes_r, 1, 1);
-  cfg.dynamicSmemBytes = psm;
-  cfg.stream = st;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = p.nsplit;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, pool_fn, pa) != cudaSuccess) return check_launch("routing pool kernel");
-  cast_status s = check_launch("routing pool kernel");
-  if (s != CAST_OK) return s;
+  // two launches of the pooling kernel, each with its own row split: the anchor frames (few
+  // long segments), then, as a programmatic dependent that fills the remaining SMs, the
+  // history blocks (it completes only after the first, see k_pool)
+  for (int part = 0; part < 2; ++part) {
+    const int nsplit = part == 0 ? p.nsplit_q : p.nsplit_kv;
+    pa.nsplit = nsplit;
+    pa.seg_base = part == 0 ? 0 : a.n_anchors;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(nsplit, part == 0 ? a.n_anchors : 2 * a.M, 1);
+    cfg.blockDim = dim3(ps.cgs * ps.lanes_r, 1, 1);
+    cfg.dynamicSmemBytes = psm;
+    cfg.stream = st;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = nsplit;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = part == 0 ? 1 : 2;
+    if (cudaLaunchKernelEx(&cfg, pool_fn, pa) != cudaSuccess) return check_launch("routing pool kernel");
+    const cast_status s = check_launch("routing pool kernel");
+    if (s != CAST_OK) return s;
+  }
 
   HeadArgs ha{};
   ha.qbar = qbar;
@@ -734,22 +1290,27 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
            a.n_frames, ha.AR, ha.BR, ha.CR);
     }
   }
-  ha.stage_kv = head_stages_kv(a) ? 1 : 0;
-  const size_t hsm = ha.stage_kv ? head_staged_bytes(a) : route_head_smem_bytes(a);
+  ha.stage_kv = 1;
+  const size_t hsm = route_head_smem_bytes(a);
+  auto head_fn = !p.wide ? k_head : (a.d == 128 ? k_head_wide<128> : k_head_wide<64>);
   if (hsm > 48 * 1024 &&
-      cudaFuncSetAttribute(k_head, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)hsm) != cudaSuccess)
+      cudaFuncSetAttribute(head_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)hsm) != cudaSuccess)
     return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory", hsm);
   cudaLaunchConfig_t hc{};
-  hc.gridDim = dim3(a.H, 1, 1);
-  hc.blockDim = dim3(kHeadThreads, 1, 1);
+  hc.gridDim = p.wide ? dim3(p.cl, a.H, 1) : dim3(a.H, 1, 1);
+  hc.blockDim = dim3(p.wide ? kWideThreads : kHeadThreads, 1, 1);
   hc.dynamicSmemBytes = hsm;
   hc.stream = st;
-  cudaLaunchAttribute hat[1];
+  cudaLaunchAttribute hat[2];
   hat[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   hat[0].val.programmaticStreamSerializationAllowed = 1;
+  hat[1].id = cudaLaunchAttributeClusterDimension;
+  hat[1].val.clusterDim.x = p.cl;
+  hat[1].val.clusterDim.y = 1;
+  hat[1].val.clusterDim.z = 1;
   hc.attrs = hat;
-  hc.numAttrs = 1;
-  if (cudaLaunchKernelEx(&hc, k_head, ha) != cudaSuccess) return check_launch("routing head kernel");
+  hc.numAttrs = p.wide ? 2 : 1;
+  if (cudaLaunchKernelEx(&hc, head_fn, ha) != cudaSuccess) return check_launch("routing head kernel");
   return check_launch("routing head kernel");
 }
 

@@ -122,3 +122,55 @@ def stress_inputs():
     vbar = np.stack([inp["v_hist"][m].astype(np.float64).mean(axis=0) for m in range(w.M)])
     rt = O.pooled_routing(qbar[:, None], list(range(len(anchors))), kbar[:, None], vbar[:, None])
     return {"dev": dev, "anchors": anchors, "routing": rt}
+
+
+WIDE_CASES = [
+    # name, d, dtype, M, B_v, K, anchors, N, extra
+    ("refine_d128", 128, "bf16", 448, 16, 90, [0, 2, 4, 6], 8, {"refine": True}),
+    ("refine_d64_f32", 64, "f32", 1000, 6, 200, [0, 3, 7, 12, 15], 16, {"refine": True}),
+    ("topk_k1", 128, "bf16", 300, 8, 1, [1, 2], 3, {}),
+    ("keep_all", 64, "bf16", 300, 8, 300, [0, 2], 3, {}),
+    ("similarity", 128, "bf16", 300, 8, 7, [0, 1], 2, {"mode": 1}),
+    ("gram", 128, "bf16", 260, 8, 50, [0, 2], 3, {"gram": True}),
+    ("candidates", 128, "bf16", 500, 8, 100, [0, 3, 5], 6, {"refine": True, "Mc": 150}),
+]
+
+
+@pytest.mark.parametrize("case", WIDE_CASES, ids=lambda c: c[0])
+def test_route_wide(lib, case):
+    """Many history blocks: the per-head statistics spread over a cluster of CTAs and the
+    radix-select TopK / refinement (block means too large for one CTA's shared memory)."""
+    from tests.test_gpu_refine import PAPER, check_refined
+    name, d, dtype, M, Bv, K, anchors, N, extra = case
+    H, S = 2, 40
+    q, k, v = _inputs(500 + M + d, N, S, H, d, M, Bv, dtype)
+    kw = {}
+    P = None
+    if extra.get("gram"):
+        P = np.random.default_rng(6).standard_normal((H, d, d)) / np.sqrt(d)
+        kw["gram"] = torch.from_numpy(np.einsum("hod,hoe->hde", P, P).astype(np.float32)).cuda()
+    if "mode" in extra:
+        kw["mode"] = extra["mode"]
+    if extra.get("refine"):
+        kw["refine"] = PAPER
+    cand = None
+    if "Mc" in extra:
+        rng = np.random.default_rng(M)
+        cand = np.stack([[rng.permutation(M)[:extra["Mc"]] for _ in range(H)]
+                         for _ in anchors]).astype(np.int32)
+        kw["candidates"] = torch.from_numpy(cand).cuda()
+    idx, u = lib.cast_route_topk(to_dev(q, dtype), anchors, to_dev(k, dtype), to_dev(v, dtype), K,
+                                 want_u=True, **kw)
+    torch.cuda.synchronize()
+    lib.cast_check_device()
+    rt = O.pooled_routing(q, anchors, k, v, proj=P)
+    ug = to_host(u)
+    score = rt.u if extra.get("mode") != 1 else rt.s
+    np.testing.assert_allclose(ug, score, rtol=5e-4, atol=1e-6 * np.abs(score).max())
+    g = idx.cpu().numpy()
+    assert g.shape == (len(anchors), H, min(K, M))
+    if extra.get("refine"):
+        changed, amb = check_refined(g, ug, anchors, N, K, PAPER, candidates=cand)
+        assert amb < H
+    else:
+        check_idx(g, score, min(K, M))
