@@ -5,15 +5,19 @@
 //             loads.  A segment's rows are split over the CTAs of one thread-block cluster;
 //             the CTAs reduce their column sums through distributed shared memory in rank order
 //             (deterministic) and write q_bar, k_bar, v_bar in f32.  No partial sums leave the
-//             chip.
-//   K_head  : one CTA per head, every anchor at once: s, pi, o_bar, delta, u (Eq. omission,
-//             with an optional Gram matrix G = P^T P of the output projection), the TopK mask of
-//             each anchor (ties to the lower block index) and, when asked, the reconstruction-
-//             coupled best-response passes of Alg. (routing); block indices are written in
-//             ascending order.
-// The head kernel is launched as a programmatic dependent of the pooling kernel: its CTAs
-// become resident while the pooling drains and wait on the grid dependency before reading the
-// means.
+//             chip.  Two launches with their own row split: the anchor frames (few long
+//             segments), then the history blocks (with (1, 8, 8) spatial blocks of history
+//             frames, 8 runs of up to 8 tokens each).
+//   K_head  : one CTA per head, every anchor at once, with the head's k_bar and v_bar staged in
+//             shared memory: s, pi, o_bar, delta, u (Eq. omission, with an optional Gram matrix
+//             G = P^T P of the output projection), the TopK mask of each anchor (ties to the
+//             lower block index) and, when asked, the reconstruction-coupled best-response passes
+//             of Alg. (routing); block indices are written in ascending order.
+//   K_head_wide : the same for many blocks (means too large to stage): a thread-block cluster
+//             per head shares the statistics, its rank-0 CTA selects (exact radix select) and
+//             refines with all its threads.
+// Each launch is a programmatic dependent of the one before: its CTAs become resident while
+// the previous grid drains and wait on the grid dependency before reading its results.
 #include <cuda_bf16.h>
 
 #include <cfloat>
@@ -255,7 +259,7 @@ struct HeadArgs {
   const int32_t* cand;   // optional [n_anchors, H, Mc] candidate sets
   int32_t* idx;
   float* u_out;
-  int H, d, M, n_anchors, K_eff, mode, passes, stage_kv, Mc;
+  int H, d, M, n_anchors, K_eff, mode, passes, Mc;
   float eps, lam_anc, lam_rec, tol;
   float A[CAST_MAX_ANCHORS], B[CAST_MAX_ANCHORS], C[CAST_MAX_ANCHORS];   // interval (j-1, j)
   float AL, BL, CL, AR, BR, CR;                                          // boundary sets
@@ -295,7 +299,7 @@ __device__ __forceinline__ float warp_total(float v) { return warp_sum(v); }
 
 // grid (H).  Dynamic smem (floats): qb[na*d], ob[na*d], pi[na*M], key[na*M], x[na*M], G[M],
 // with candidate sets Gc[M], then e[kHeadWarps*d] (Gram scratch); with candidate sets the
-// membership bytes cm[na*M]; when stage_kv, kb[M*d], vb[M*d] (this head's means).
+// membership bytes cm[na*M]; then kb[M*d], vb[M*d] (this head's means, staged).
 __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ HeadArgs a) {
   extern __shared__ float sm[];
   const int h = blockIdx.x, na = a.n_anchors, M = a.M, d = a.d, K = a.K_eff;
@@ -320,15 +324,15 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
   float* vb_s = kb_s + (size_t)M * d;
   launch_dependents();
   grid_dependency_wait();   // the pooled means come from the preceding kernel
-  // this head's slices of q_bar (and of k_bar, v_bar when they fit), all loads in flight at once
+  // this head's slices of q_bar, k_bar and v_bar into shared memory, all loads in flight at once
   const float* kb = a.kbar + h * d;
   const float* vb = a.vbar + h * d;
-  int64_t kv_stride = D;
+  const int64_t kv_stride = d;
   {
-    // rows of d/4 float4: q_bar rows of every anchor, then k_bar and v_bar rows when staged;
+    // rows of d/4 float4: q_bar rows of every anchor, then k_bar and v_bar rows;
     // each thread issues up to 8 loads before its first store
     const int q4 = d / 4;
-    const int n_q = na * q4, n_all = n_q + (a.stage_kv ? 2 * M * q4 : 0);
+    const int n_q = na * q4, n_all = n_q + 2 * M * q4;
     for (int e0 = tid; e0 < n_all; e0 += 8 * kHeadThreads) {
       float4 v[8];
 #pragma unroll
@@ -354,11 +358,8 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
         }
       }
     }
-    if (a.stage_kv) {
-      kb = kb_s;
-      vb = vb_s;
-      kv_stride = d;
-    }
+    kb = kb_s;
+    vb = vb_s;
   }
   __syncthreads();
   const float scale = rsqrtf((float)d);
@@ -1290,7 +1291,6 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
            a.n_frames, ha.AR, ha.BR, ha.CR);
     }
   }
-  ha.stage_kv = 1;
   const size_t hsm = route_head_smem_bytes(a);
   auto head_fn = !p.wide ? k_head : (a.d == 128 ? k_head_wide<128> : k_head_wide<64>);
   if (hsm > 48 * 1024 &&
