@@ -261,7 +261,7 @@ def run_gpu(args):
             "breakdown": {
                 "route": {"ms": round(t_route, 5), "GB/s": round(route_bytes / t_route / 1e6, 1),
                           "frac_hbm": round(route_bytes / t_route / 1e6 / hbm, 4),
-                          "bytes": route_bytes, "kernels": 2},
+                          "bytes": route_bytes, "kernels": 3},
                 "attention": {"ms": round(t_attn, 5), "TFLOP/s": round(achieved, 2),
                               "frac_bf16": round(achieved / bf16, 4)},
                 "par": {"ms": round(t_par, 5), "GB/s": round(par_bytes / t_par / 1e6, 1),
