@@ -250,11 +250,13 @@ typedef struct {
  * (mirrors negated, self-conjugate bins 0), c = sum kappa|Z| / (sum kappa W + eps) over the
  * reliable non-DC bins, g = sigmoid((c - tau(nu)) / T), and
  * R_t = IRFFT2_ortho((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
- * All frames anchors: nothing to do.  cast_par_workspace_size() is 0 (workspace may be
- * NULL): the cross-channel sums stay in the shared memory of a thread-block cluster.
+ * All frames anchors: nothing to do (workspace size 0).  The workspace
+ * (cast_par_workspace_size() bytes) holds each channel chunk's partial Z, W per (tile, pair)
+ * and theta, g per bin: 120 ceil(C/128) + 80 floats per tile and anchor (each part rounded
+ * up to 256 bytes).
  * Errors: INVALID_ARG when a frame is skipped and fewer than two anchors exist, bad shapes
- * or pointers; UNSUPPORTED for tile sides outside 1..8, C not a multiple of 8, C > 4096, or
- * a cluster that cannot be made resident on this device. */
+ * or pointers, a short workspace; UNSUPPORTED for tile sides outside 1..8, C not a multiple
+ * of 8, C > 4096. */
 cast_status cast_par_reconstruct(const cast_par_args* args, void* workspace,
                                  size_t workspace_bytes, void* stream);
 size_t cast_par_workspace_size(const cast_par_args* args);

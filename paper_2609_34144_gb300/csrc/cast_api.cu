@@ -503,9 +503,36 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
   return CAST_OK;
 }
 
+namespace cast {
+namespace {
+// PAR of the FFN site: the skipped frames of r_out from its anchor rows
+cast_par_args par_of_ffn(const cast_ffn_args* a, uint8_t* mask) {
+  cast_par_args p{};
+  p.r = a->r_out;
+  p.dtype = a->r_dtype;
+  p.F = a->n_frames;
+  p.Hg = a->Hg;
+  p.Wg = a->Wg;
+  p.C = a->D;
+  for (int f = 0; f < a->n_frames && f < CAST_MAX_FRAMES; ++f) mask[f] = 0;
+  for (int k = 0; k < a->n_anchors; ++k)
+    if (a->anchors && a->anchors[k] >= 0 && a->anchors[k] < a->n_frames) mask[a->anchors[k]] = 1;
+  p.anchor_mask = mask;
+  p.channel_weight = a->channel_weight;
+  p.params = a->par;
+  return p;
+}
+}  // namespace
+}  // namespace cast
+
 size_t cast_ffn_workspace_size(const cast_ffn_args* a) {
-  if (!a || a->Hg < 1 || a->Wg < 1 || a->D_ff < 1) return 0;
-  return align_up((size_t)a->Hg * a->Wg * a->D_ff * 2) + kGemmWorkspace;
+  if (!a || a->Hg < 1 || a->Wg < 1 || a->D_ff < 1 || a->n_frames < 1 || a->n_frames > CAST_MAX_FRAMES ||
+      a->n_anchors < 1 || a->n_anchors > CAST_MAX_ANCHORS || !a->anchors)
+    return 0;
+  uint8_t mask[CAST_MAX_FRAMES];
+  const cast_par_args p = par_of_ffn(a, mask);
+  const size_t par = (p.params.tile_h >= 1 && p.params.tile_w >= 1 && p.C >= 1) ? par_plan(p).total_bytes : 0;
+  return align_up((size_t)a->Hg * a->Wg * a->D_ff * 2) + kGemmWorkspace + align_up(par);
 }
 
 cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, void* stream) {
@@ -526,18 +553,7 @@ cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, voi
       (a->b2 && !aligned16(a->b2)))
     return fail(CAST_ERR_INVALID_ARG, "%s: weights or biases NULL or misaligned", who);
   uint8_t mask[CAST_MAX_FRAMES];
-  cast_par_args p{};
-  p.r = a->r_out;
-  p.dtype = a->r_dtype;
-  p.F = a->n_frames;
-  p.Hg = a->Hg;
-  p.Wg = a->Wg;
-  p.C = a->D;
-  for (int f = 0; f < a->n_frames; ++f) mask[f] = 0;
-  for (int k = 0; k < a->n_anchors; ++k) mask[a->anchors[k]] = 1;
-  p.anchor_mask = mask;
-  p.channel_weight = a->channel_weight;
-  p.params = a->par;
+  cast_par_args p = par_of_ffn(a, mask);
   if ((s = validate_par(&p))) return s;
   const size_t need = cast_ffn_workspace_size(a);
   if (ws_bytes < need || !ws)
@@ -548,6 +564,7 @@ cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, voi
   const int S = a->Hg * a->Wg;
   char* hid = static_cast<char*>(ws);
   char* gws = hid + align_up((size_t)S * a->D_ff * 2);
+  char* pws = gws + kGemmWorkspace;
   const size_t elt = a->r_dtype == CAST_BF16 ? 2 : 4;
   for (int i = 0; i < a->n_anchors; ++i) {
     const int f = a->anchors[i];
@@ -584,7 +601,7 @@ cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, voi
     g2.ws_bytes = kGemmWorkspace;
     if ((s = gemm_rows(g2, st))) return s;
   }
-  if (par_plan(p).n_target > 0) return launch_par(p, nullptr, st);
+  if (par_plan(p).n_target > 0) return launch_par(p, pws, st);
   return CAST_OK;
 }
 

@@ -89,10 +89,9 @@ struct ParPlan {
   int tiles_y, tiles_x, n_tile;
   int n_full, n_edge;   // 8x8 tiles / truncated (or non-8x8) tiles
   int chunk;        // channels per CTA (= threads per CTA)
-  int n_chunk;      // channel groups = CTAs per cluster
-  int cl;           // CTAs per cluster
+  int n_chunk;      // channel chunks per tile
   int n_tseg_full, n_tseg_edge;   // time segments (runs of anchor pairs) per tile, per kind
-  size_t total_bytes;
+  size_t rec_bytes, trans_bytes, total_bytes;   // workspace: chunk records, theta and g
 };
 ParPlan par_plan(const cast_par_args& a);
 cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st);

@@ -1,21 +1,22 @@
 // Phase-Aware Reconstruction of skipped frames (Section 4.3, Eqs. cross, confidence, gate,
-// fcpasm; App. A.2), one fused single-pass kernel.
+// fcpasm; App. A.2) in three passes per tile kind (full 8x8 tiles / truncated edge tiles):
 //
-// A thread-block cluster owns one spectral tile position (and a run of consecutive anchor
-// pairs); its CTAs split the channels, one thread per channel.  For each anchor in time order
-// the CTA streams the anchor tile through a TMA 4-D map ([frame][row][col][channel], out-of-
-// range rows/cols/channels arrive as zeros) and forms the channel's tile spectrum in registers
-// (the previous anchor's spectrum stays in shared memory).  For every adjacent pair with
-// targets:
-//   1. each CTA reduces Z = sum_c w_c F_b conj(F_a) and W = sum_c w_c |F_b||F_a| over its
-//      channels (warp transpose reductions) into a record in its shared memory;
-//   2. after a cluster barrier every CTA sums the records of all CTAs of the cluster through
-//      distributed shared memory in rank order (deterministic, identical in every CTA) and
-//      derives eta, reliability, principal phases, the tile confidence c and the gate g;
-//   3. every target t of the pair is written straight from registers:
-//      R_t = IRFFT2((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
-// Each anchor element is read from HBM once and transformed once; each target element is
-// written once; nothing but the output goes through global memory.
+//   K_stats (tile, channel chunk): one thread per channel streams the anchors of the tile in
+//       time order through a TMA 4-D map ([frame][row][col][channel], out-of-range rows/cols/
+//       channels arrive as zeros), forms each tile spectrum in registers (the previous anchor's
+//       spectrum stays in shared memory) and, for every anchor pair with targets, reduces
+//       Z = sum_c w_c F_b conj(F_a) and W = sum_c w_c |F_b||F_a| over the chunk's channels
+//       (warp transpose reductions) into one record in the workspace.
+//   K_transport (tile, pair): sums the records of the tile's channel chunks in chunk order
+//       (deterministic) and derives eta, reliability, principal phases, the confidence c and
+//       the gate g per bin; writes theta and g.
+//   K_blend (tile, channel chunk): streams the anchors again (an L2 hit at these sizes), forms
+//       their spectra and writes every target straight from registers:
+//       R_t = IRFFT2((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
+// The CTAs of a pass never wait on each other, so the passes fill the GPU whatever the number
+// of anchor pairs; the passes are chained as programmatic dependents.  Global traffic beyond
+// the algorithmic bytes: a second read of the anchors and the records (120 floats per tile,
+// pair and chunk).
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -28,11 +29,10 @@
 namespace cast {
 namespace {
 
-constexpr int kMaxThreads = 256;   // channels per CTA (one thread each), a multiple of 32
-constexpr int kMaxCluster = 16;    // CTAs per cluster (channel groups of one tile)
+constexpr int kCC = 128;           // channels per CTA (one thread each)
 constexpr int kNB = 40;            // stored bins of an 8-wide tile: 8 x 5
 constexpr int kNV = 3 * kNB;       // (Re Z, Im Z, W) per bin, record index = 3 * bin + component
-constexpr int kRec = kNV;          // record slots per CTA (96 + 1 used for 8x8 tiles)
+constexpr int kRec = kNV;          // record slots per chunk (96 + 1 used for 8x8 tiles)
 constexpr int kCoefBatch = 4;
 
 __device__ unsigned int g_par_error;   // 1: a wait gave up
@@ -145,7 +145,10 @@ __host__ __device__ __forceinline__ constexpr int fast_value(int n) {
 struct ParKArgs {
   char* r;
   const float* wch;
-  int F, Hg, Wg, C, cl;                  // cl: CTAs per cluster (channel groups)
+  float* rec;     // workspace [tile][pair j][chunk][kRec]: each chunk's Z / W record
+  float* trans;   // workspace [tile][pair j][2][kNB]: theta and g per bin
+  int F, Hg, Wg, C, n_chunk;             // n_chunk: channel chunks of kCC channels
+  int tile_base;                         // global index of tile 0 of this launch's kind
   int th, tw, tiles_x, tiles_y, n_tile, n_tseg;
   int n_anchor;
   int anchor_frame[CAST_MAX_ANCHORS];
@@ -374,31 +377,28 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const BinIn
   }
 }
 
-__device__ __forceinline__ void cluster_sync_all() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
-                   : "memory");
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
-// Dynamic shared memory of one CTA with cc channels in a cluster of cl: the TMA stage (one
-// anchor tile, 128-byte aligned), the previous anchor's spectrum [value][thread], and the
-// records of every CTA of the cluster for two rounds [round][rank][value].
+__device__ __forceinline__ void launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Dynamic shared memory of a streaming CTA with cc channels: the TMA stage (one anchor tile,
+// 128-byte aligned) and the previous anchor's spectrum [value][thread].
 template <typename T>
 __host__ __device__ constexpr size_t stage_bytes(int cc) { return (size_t)64 * cc * sizeof(T); }
 __host__ __device__ constexpr size_t spec_bytes(int cc) { return (size_t)2 * kNB * cc * sizeof(float); }
 template <typename T>
-__host__ __device__ constexpr size_t par_dyn_smem(int cc, int cl) {
-  return stage_bytes<T>(cc) + spec_bytes(cc) + (size_t)2 * cl * kRec * sizeof(float) + 128;
+__host__ __device__ constexpr size_t par_dyn_smem(int cc) {
+  return stage_bytes<T>(cc) + spec_bytes(cc) + 128;
 }
 
-__device__ __forceinline__ void st_dsmem(float* local, uint32_t rank, float v) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
-}
-
-// grid (cl, n_tiles_of_kind * n_tseg), cluster (cl, 1, 1), CC threads = channels per CTA.
-// FULL: every tile of the grid is 8x8 (the specialised fast path); otherwise edge tiles.
-template <typename T, int CC, bool FULL>
-__global__ void __launch_bounds__(CC, FULL ? (CC == 128 ? 3 : (CC == 192 ? 2 : 1)) : 1)
+// K_stats (STATS) and K_blend (!STATS): grid (n_chunk, n_tiles_of_kind * n_tseg), CC threads,
+// one channel each.  A time segment covers the anchor pairs seg_pair0 .. seg_pair1 (it starts
+// one anchor earlier).  FULL: every tile of the launch is 8x8 (the specialised fast path).
+template <typename T, int CC, bool FULL, bool STATS>
+__global__ void __launch_bounds__(CC, FULL ? 3 : 2)
     k_par(const __grid_constant__ CUtensorMap tm, const __grid_constant__ ParKArgs a) {
   extern __shared__ uint8_t dsm_raw[];
   const uint32_t raw = smem_u32(dsm_raw);
@@ -407,20 +407,16 @@ __global__ void __launch_bounds__(CC, FULL ? (CC == 128 ? 3 : (CC == 192 ? 2 : 1
   constexpr int nwarp = CC / 32;
   const T* stage = reinterpret_cast<const T*>(dsm);          // [y][x][channel] of one anchor tile
   float* s_fprev = reinterpret_cast<float*>(dsm + stage_bytes<T>(cc));   // [value][thread]
-  float* s_recv = reinterpret_cast<float*>(dsm + stage_bytes<T>(cc) + spec_bytes(cc));
-  __shared__ float s_red[nwarp][128];
-  __shared__ float s_zw[kNV];
-  __shared__ float s_th[kNB], s_g[kNB], s_own_th[kNB];
-  __shared__ int s_own_rel[kNB];
-  __shared__ float4 s_coef[kCoefBatch][kNB];
-  __shared__ BinInfo s_bins;
+  __shared__ float s_red[STATS ? nwarp : 1][128];
+  __shared__ float4 s_coef[STATS ? 1 : kCoefBatch][kNB];
   __shared__ __align__(8) uint64_t s_full;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int rank = blockIdx.x;                        // = rank in the cluster (cluster spans x)
+  const int chunk = blockIdx.x;
   const int tile = blockIdx.y / a.n_tseg, seg = blockIdx.y - tile * a.n_tseg;
+  const int tg = a.tile_base + tile;                  // tile index in the workspace
   const int j0 = a.seg_pair0[seg] - 1, j1 = a.seg_pair1[seg];   // anchors of this segment
   const TileGeom g = tile_geom(a, tile, FULL);
-  const int c = rank * cc + tid;
+  const int c = chunk * cc + tid;
   const bool active = c < a.C;
   const float wc = active ? (a.wch ? __ldg(a.wch + c) : 1.f) : 0.f;
   // bytes one TMA box delivers: cc channels x tile_w x tile_h (must match the tensor map)
@@ -430,14 +426,13 @@ __global__ void __launch_bounds__(CC, FULL ? (CC == 128 ? 3 : (CC == 192 ? 2 : 1
     fence_barrier_init();
     tma_prefetch_desc(&tm);
     mbar_arrive_expect_tx(&s_full, box_bytes);
-    tma_load_4d(const_cast<T*>(stage), &tm, &s_full, rank * cc, g.x0, g.y0, a.anchor_frame[j0]);
+    tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * cc, g.x0, g.y0, a.anchor_frame[j0]);
   }
-  bin_info(a, g, s_bins, tid);
+  launch_dependents();
   __syncthreads();
+  // K_blend reads theta and g, written by the preceding K_transport
+  if (!STATS) grid_dependency_wait();
   bool ok = true;          // CTA-uniform; after a failed wait no more TMA is issued
-  int round = 0;           // pairs reduced so far: the receive buffer alternates per round, and
-                           // every round ends in a cluster barrier, so a buffer is rewritten
-                           // only after every CTA has passed the barrier that follows its reads
   const int64_t frame_elems = (int64_t)a.Hg * a.Wg * a.C;
   T* out = reinterpret_cast<T*>(a.r);
 
@@ -465,17 +460,15 @@ __global__ void __launch_bounds__(CC, FULL ? (CC == 128 ? 3 : (CC == 192 ? 2 : 1
       }
       if (ok && tid == 0 && j + 1 <= j1) {
         mbar_arrive_expect_tx(&s_full, box_bytes);
-        tma_load_4d(const_cast<T*>(stage), &tm, &s_full, rank * cc, g.x0, g.y0, a.anchor_frame[j + 1]);
+        tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * cc, g.x0, g.y0, a.anchor_frame[j + 1]);
       }
       if (FULL) dft::fwd2d(x, 8, 8, re, im);
       else dft::fwd2d(x, g.h, g.w, re, im);
     }
     const bool has_targets = j > j0 && a.pair_tbeg[j + 1] > a.pair_tbeg[j];
     const float* fa = s_fprev;   // spectrum of anchor j-1 (this thread's column)
-    if (has_targets) {
-      float* recv = s_recv + (size_t)(round & 1) * a.cl * kRec;   // [rank][value]
-      ++round;
-      // ---- 1. this CTA's Z = sum w F_b conj(F_a), W = sum w |F_b||F_a| (Eq. cross)
+    if (STATS && has_targets) {
+      // this chunk's Z = sum w F_b conj(F_a), W = sum w |F_b||F_a| (Eq. cross)
       if (FULL) {
         // the 96 non-redundant values in three transpose groups, W at DC by a warp sum
 #pragma unroll
@@ -519,41 +512,29 @@ __global__ void __launch_bounds__(CC, FULL ? (CC == 128 ? 3 : (CC == 192 ? 2 : 1
         }
       }
       __syncthreads();
-      // the CTA's record, pushed into slot `rank` of every CTA of the cluster
       constexpr int nrec = FULL ? 97 : kNV;
       if (tid < nrec) {
         float sum = 0.f;
 #pragma unroll
         for (int w = 0; w < nwarp; ++w) sum += s_red[w][tid];
-        for (int r = 0; r < a.cl; ++r) st_dsmem(recv + rank * kRec + tid, (uint32_t)r, sum);
+        a.rec[(((int64_t)tg * a.n_anchor + j) * a.n_chunk + chunk) * kRec + tid] = sum;
       }
-      // ---- 2. cluster-wide sums in rank order (local reads), then the tile's transport
-      cluster_sync_all();
-      if (tid < kNV) {
-        float sum = 0.f;
-        int k = tid, sign = 1;
-        if (FULL) {
-          const int src = a.fast_src[tid];
-          k = (src > 0 ? src : -src) - 1;
-          sign = src < 0 ? -1 : 1;
-        }
-        if (k >= 0)
-          for (int r = 0; r < a.cl; ++r) sum += recv[r * kRec + k];
-        s_zw[tid] = sign < 0 ? -sum : sum;
-      }
-      __syncthreads();
-      if (warp == 0) tile_transport(a, g, s_bins, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
-      __syncthreads();
-      // ---- 3. every target of the pair (Eq. fcpasm), ortho scale folded into the coefficients
+      // s_red is rewritten only after the next anchor's stage barrier
+    }
+    if (!STATS && has_targets) {
+      // every target of the pair (Eq. fcpasm), ortho scale folded into the coefficients
+      const float* th = a.trans + ((int64_t)tg * a.n_anchor + j) * 2 * kNB;
+      const float* gg = th + kNB;
       const float inv_hw = 1.f / (float)(g.h * g.w);
       for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += kCoefBatch) {
         const int nt = min(kCoefBatch, a.pair_tbeg[j + 1] - t0);
         for (int e = tid; e < nt * kNB; e += cc) {
           const int k = e / kNB, b = e % kNB;
           const float al = a.target_alpha[t0 + k];
+          const float tb = __ldcg(th + b), gb = __ldcg(gg + b);
           float sa, ca, sb, cb;
-          sincos_reduced(s_g[b] * al * s_th[b], &sa, &ca);
-          sincos_reduced(-s_g[b] * (1.f - al) * s_th[b], &sb, &cb);
+          sincos_reduced(gb * al * tb, &sa, &ca);
+          sincos_reduced(-gb * (1.f - al) * tb, &sb, &cb);
           const float fa_ = (1.f - al) * inv_hw, fb_ = al * inv_hw;
           s_coef[k][b] = make_float4(fa_ * ca, fa_ * sa, fb_ * cb, fb_ * sb);
         }
@@ -597,7 +578,44 @@ __global__ void __launch_bounds__(CC, FULL ? (CC == 128 ? 3 : (CC == 192 ? 2 : 1
       }
     }
   }
-  cluster_sync_all();   // no CTA leaves while a peer may still write its records
+}
+
+// K_transport: grid (n_tiles_of_kind, n_anchor - 1), 128 threads; block y = pair j - 1.
+template <bool FULL>
+__global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ ParKArgs a) {
+  __shared__ float s_zw[kNV];
+  __shared__ float s_th[kNB], s_g[kNB], s_own_th[kNB];
+  __shared__ int s_own_rel[kNB];
+  __shared__ BinInfo s_bins;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tile = blockIdx.x, j = blockIdx.y + 1, tg = a.tile_base + tile;
+  launch_dependents();
+  if (!(a.pair_tbeg[j + 1] > a.pair_tbeg[j])) return;   // no targets: no record
+  const TileGeom g = tile_geom(a, tile, FULL);
+  bin_info(a, g, s_bins, tid);
+  grid_dependency_wait();   // the records come from the preceding K_stats
+  if (tid < kNV) {
+    int k = tid, sign = 1;
+    if (FULL) {
+      const int src = a.fast_src[tid];
+      k = (src > 0 ? src : -src) - 1;
+      sign = src < 0 ? -1 : 1;
+    }
+    float sum = 0.f;
+    if (k >= 0) {
+      const float* r = a.rec + ((int64_t)tg * a.n_anchor + j) * a.n_chunk * kRec + k;
+      for (int ch = 0; ch < a.n_chunk; ++ch) sum += __ldcg(r + (int64_t)ch * kRec);
+    }
+    s_zw[tid] = sign < 0 ? -sum : sum;
+  }
+  __syncthreads();
+  if (warp == 0) tile_transport(a, g, s_bins, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
+  __syncthreads();
+  if (tid < kNB) {
+    float* t = a.trans + ((int64_t)tg * a.n_anchor + j) * 2 * kNB;
+    t[tid] = s_th[tid];
+    t[kNB + tid] = s_g[tid];
+  }
 }
 
 // 4-D map [F][Hg][Wg][C], box (cc channels, tw, th, 1), zero fill out of range
@@ -614,39 +632,42 @@ bool make_r_map(CUtensorMap* m, const cast_par_args& a, int cc) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <typename T, int CC, bool FULL>
-cast_status launch_kind(const CUtensorMap& tm, const ParKArgs& k, const ParPlan& p, int n_tiles,
-                        cudaStream_t st) {
-  const size_t smem = par_dyn_smem<T>(CC, p.cl);
+// One tile kind on one stream: K_stats, then K_transport and K_blend as programmatic dependents.
+template <typename T, bool FULL>
+cast_status launch_kind(const CUtensorMap& tm, const ParKArgs& k, int n_tiles, cudaStream_t st) {
+  const size_t smem = par_dyn_smem<T>(kCC);
   static bool attr_set = false;
   if (!attr_set) {
-    if (cudaFuncSetAttribute(k_par<T, CC, FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)par_dyn_smem<T>(CC, kMaxCluster)) != cudaSuccess ||
-        cudaFuncSetAttribute(k_par<T, CC, FULL>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-            cudaSuccess)
+    if (cudaFuncSetAttribute(k_par<T, kCC, FULL, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem) != cudaSuccess ||
+        cudaFuncSetAttribute(k_par<T, kCC, FULL, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem) != cudaSuccess)
       return check_launch("PAR kernel attributes");
     attr_set = true;
   }
+  cudaLaunchAttribute pdl[1];
+  pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(p.cl, n_tiles * k.n_tseg, 1);
-  cfg.blockDim = dim3(CC, 1, 1);
+  cfg.gridDim = dim3(k.n_chunk, n_tiles * k.n_tseg, 1);
+  cfg.blockDim = dim3(kCC, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = p.cl;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
+  if (cudaLaunchKernelEx(&cfg, k_par<T, kCC, FULL, true>, tm, k) != cudaSuccess)
+    return check_launch("PAR statistics kernel");
+  cudaLaunchConfig_t tc{};
+  tc.gridDim = dim3(n_tiles, k.n_anchor - 1, 1);
+  tc.blockDim = dim3(128, 1, 1);
+  tc.stream = st;
+  tc.attrs = pdl;
+  tc.numAttrs = 1;
+  if (cudaLaunchKernelEx(&tc, k_par_transport<FULL>, k) != cudaSuccess)
+    return check_launch("PAR transport kernel");
+  cfg.attrs = pdl;
   cfg.numAttrs = 1;
-  int clusters = 0;
-  if (cudaOccupancyMaxActiveClusters(&clusters, k_par<T, CC, FULL>, &cfg) != cudaSuccess || clusters < 1) {
-    cudaGetLastError();
-    return fail(CAST_ERR_UNSUPPORTED, "PAR: a cluster of %d CTAs x %d channels cannot be resident",
-                p.cl, CC);
-  }
-  if (cudaLaunchKernelEx(&cfg, k_par<T, CC, FULL>, tm, k) != cudaSuccess) return check_launch("PAR kernel");
-  return check_launch("PAR kernel");
+  if (cudaLaunchKernelEx(&cfg, k_par<T, kCC, FULL, false>, tm, k) != cudaSuccess)
+    return check_launch("PAR blend kernel");
+  return check_launch("PAR kernels");
 }
 
 // A second stream per device (and the events that fork it from and join it back into the
@@ -688,30 +709,25 @@ ParKArgs with_segments(const ParKArgs& k0, int nseg) {
   return k;
 }
 
-template <typename T, int CC>
+template <typename T>
 cast_status launch_typed(const CUtensorMap& tm, const ParKArgs& k0, const ParPlan& p, cudaStream_t st) {
-  const ParKArgs kf = with_segments(k0, p.n_tseg_full), ke = with_segments(k0, p.n_tseg_edge);
-  if (p.n_edge == 0) return launch_kind<T, CC, true>(tm, kf, p, p.n_full, st);
-  if (p.n_full == 0) return launch_kind<T, CC, false>(tm, ke, p, p.n_edge, st);
+  ParKArgs kf = with_segments(k0, p.n_tseg_full), ke = with_segments(k0, p.n_tseg_edge);
+  kf.tile_base = 0;
+  ke.tile_base = p.n_full;
+  if (p.n_edge == 0) return launch_kind<T, true>(tm, kf, p.n_full, st);
+  if (p.n_full == 0) return launch_kind<T, false>(tm, ke, p.n_edge, st);
   // full tiles on the caller's stream, edge tiles concurrently on the side stream
   ForkStream* f = nullptr;
   cast_status s = fork_stream(f);
   if (s != CAST_OK) return s;
   if (cudaEventRecord(f->fork, st) != cudaSuccess || cudaStreamWaitEvent(f->side, f->fork, 0) != cudaSuccess)
     return check_launch("PAR fork");
-  s = launch_kind<T, CC, false>(tm, ke, p, p.n_edge, f->side);
+  s = launch_kind<T, false>(tm, ke, p.n_edge, f->side);
   if (s != CAST_OK) return s;
-  s = launch_kind<T, CC, true>(tm, kf, p, p.n_full, st);
+  s = launch_kind<T, true>(tm, kf, p.n_full, st);
   if (cudaEventRecord(f->join, f->side) != cudaSuccess || cudaStreamWaitEvent(st, f->join, 0) != cudaSuccess)
     return check_launch("PAR join");
   return s;
-}
-
-template <typename T>
-cast_status launch_cc(const CUtensorMap& tm, const ParKArgs& k, const ParPlan& p, cudaStream_t st) {
-  if (p.chunk == 128) return launch_typed<T, 128>(tm, k, p, st);
-  if (p.chunk == 192) return launch_typed<T, 192>(tm, k, p, st);
-  return launch_typed<T, 256>(tm, k, p, st);
 }
 
 }  // namespace
@@ -735,26 +751,26 @@ ParPlan par_plan(const cast_par_args& a) {
     p.n_full = 0;
     p.n_edge = p.n_tile;
   }
-  // channel groups: CTAs of 128 channels, or of 192 / 256 when more than kMaxCluster CTAs of
-  // 128 would be needed; a cluster spans the groups
-  int cc = 128;
-  while (cc < kMaxThreads && (a.C + cc - 1) / cc > kMaxCluster) cc += 64;
-  const int cl = (a.C + cc - 1) / cc;
-  p.cl = cl;
-  p.chunk = cc;
-  p.n_chunk = cl;
-  // time segments: split the anchor pairs so that the clusters cover the GPU about twice
+  // channel chunks of kCC channels, one CTA each
+  p.chunk = kCC;
+  p.n_chunk = (a.C + kCC - 1) / kCC;
+  // time segments: split the anchor pairs so that the CTAs of each kind cover the SMs about
+  // three deep (each segment re-reads its first anchor)
   int dev = 0, nsm = 148;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-  const int want_clusters = 2 * (nsm > 0 ? nsm : 148) / (cl < 2 ? 2 : cl) + 1;
+  const int want_ctas = 3 * (nsm > 0 ? nsm : 148);
   auto segs = [&](int n_tiles) {
-    int nseg = n_tiles > 0 ? (want_clusters + n_tiles - 1) / n_tiles : 1;
+    const int per_seg = n_tiles * p.n_chunk;
+    int nseg = per_seg > 0 ? (want_ctas + per_seg - 1) / per_seg : 1;
     if (nseg > p.n_pair) nseg = p.n_pair;
     return nseg < 1 ? 1 : nseg;
   };
   p.n_tseg_full = segs(p.n_full);
   p.n_tseg_edge = segs(p.n_edge);
-  p.total_bytes = 0;   // no workspace: the reduction stays in the cluster's shared memory
+  // workspace: the chunk records [tile][pair][chunk][kRec] and theta, g [tile][pair][2][kNB]
+  p.rec_bytes = align_up((size_t)p.n_tile * (na > 0 ? na : 1) * p.n_chunk * kRec * sizeof(float));
+  p.trans_bytes = align_up((size_t)p.n_tile * (na > 0 ? na : 1) * 2 * kNB * sizeof(float));
+  p.total_bytes = p.n_target > 0 ? p.rec_bytes + p.trans_bytes : 0;
   return p;
 }
 
@@ -773,7 +789,9 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
   k.tiles_x = p.tiles_x;
   k.tiles_y = p.tiles_y;
   k.n_tile = p.n_tile;
-  k.cl = p.cl;
+  k.n_chunk = p.n_chunk;
+  k.rec = static_cast<float*>(ws);
+  k.trans = reinterpret_cast<float*>(static_cast<char*>(ws) + p.rec_bytes);
   int anchors[CAST_MAX_FRAMES];
   int na = 0;
   for (int f = 0; f < a.F; ++f)
@@ -828,11 +846,10 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
     }
   }
 
-  (void)ws;
   CUtensorMap tm;
   if (!make_r_map(&tm, a, p.chunk)) return fail(CAST_ERR_CUDA, "PAR: cuTensorMapEncodeTiled failed");
-  if (a.dtype == CAST_BF16) return launch_cc<__nv_bfloat16>(tm, k, p, st);
-  return launch_cc<float>(tm, k, p, st);
+  if (a.dtype == CAST_BF16) return launch_typed<__nv_bfloat16>(tm, k, p, st);
+  return launch_typed<float>(tm, k, p, st);
 }
 
 unsigned int par_error_word(cudaStream_t st, bool clear) {

@@ -135,10 +135,18 @@ def test_par_all_anchors_needs_nothing(lib):
     assert lib.library().cast_par_reconstruct(C.byref(a), None, 0, None) == 0
 
 
-def test_par_needs_no_workspace(lib):
-    # the cross-channel reduction stays in the cluster's shared memory
+def test_par_workspace_size(lib):
+    # chunk records (120 floats per 128-channel chunk) and theta, g (80 floats) per tile and anchor
+    def up(x):
+        return (x + 255) // 256 * 256
+    so = lib.library()
     for ch in (64, 512, 3072):
-        assert lib.library().cast_par_workspace_size(C.byref(_par(lib, [1, 0, 1], C=ch))) == 0
+        a = _par(lib, [1, 0, 1], C=ch)
+        tiles, na, chunks = 4, 2, -(-ch // 128)      # 16 x 16 grid of 8x8 tiles, 2 anchors
+        want = up(tiles * na * chunks * 120 * 4) + up(tiles * na * 80 * 4)
+        assert so.cast_par_workspace_size(C.byref(a)) == want
+        assert so.cast_par_reconstruct(C.byref(a), _fake(0x100000), want - 1, None) == 1
+    assert so.cast_par_workspace_size(C.byref(_par(lib, [1, 1, 1]))) == 0   # nothing to reconstruct
 
 
 def test_attention_validation(lib):
