@@ -384,14 +384,17 @@ __device__ __forceinline__ void launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-// Dynamic shared memory of a streaming CTA with cc channels: the TMA stage (one anchor tile,
-// 128-byte aligned) and the previous anchor's spectrum [value][thread].
+// Dynamic shared memory of a streaming CTA with cc channels: a ring of n_stages<T> TMA stages
+// (one anchor tile each, 128-byte aligned; two for bf16, one for f32 so that three CTAs still
+// fit an SM) and the previous anchor's spectrum [value][thread].
+template <typename T>
+__host__ __device__ constexpr int n_stages() { return sizeof(T) == 2 ? 2 : 1; }
 template <typename T>
 __host__ __device__ constexpr size_t stage_bytes(int cc) { return (size_t)64 * cc * sizeof(T); }
 __host__ __device__ constexpr size_t spec_bytes(int cc) { return (size_t)2 * kNB * cc * sizeof(float); }
 template <typename T>
 __host__ __device__ constexpr size_t par_dyn_smem(int cc) {
-  return stage_bytes<T>(cc) + spec_bytes(cc) + 128;
+  return n_stages<T>() * stage_bytes<T>(cc) + spec_bytes(cc) + 128;
 }
 
 // K_stats (STATS) and K_blend (!STATS): grid (n_chunk, n_tiles_of_kind * n_tseg), CC threads,
@@ -405,11 +408,12 @@ __global__ void __launch_bounds__(CC, FULL ? 3 : 2)
   uint8_t* dsm = dsm_raw + (((raw + 127u) & ~127u) - raw);   // TMA boxes without swizzle: 128 B
   constexpr int cc = CC;
   constexpr int nwarp = CC / 32;
-  const T* stage = reinterpret_cast<const T*>(dsm);          // [y][x][channel] of one anchor tile
-  float* s_fprev = reinterpret_cast<float*>(dsm + stage_bytes<T>(cc));   // [value][thread]
+  constexpr int kStages = n_stages<T>();
+  T* stages = reinterpret_cast<T*>(dsm);       // kStages x [y][x][channel] of one anchor tile
+  float* s_fprev = reinterpret_cast<float*>(dsm + kStages * stage_bytes<T>(cc));   // [value][thread]
   __shared__ float s_red[STATS ? nwarp : 1][128];
   __shared__ float4 s_coef[STATS ? 1 : kCoefBatch][kNB];
-  __shared__ __align__(8) uint64_t s_full;
+  __shared__ __align__(8) uint64_t s_full[kStages];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int chunk = blockIdx.x;
   const int tile = blockIdx.y / a.n_tseg, seg = blockIdx.y - tile * a.n_tseg;
@@ -422,11 +426,15 @@ __global__ void __launch_bounds__(CC, FULL ? 3 : 2)
   // bytes one TMA box delivers: cc channels x tile_w x tile_h (must match the tensor map)
   const uint32_t box_bytes = (uint32_t)(cc * a.tw * a.th * sizeof(T));
   if (tid == 0) {
-    mbar_init(&s_full, 1);
+    for (int st = 0; st < kStages; ++st) mbar_init(&s_full[st], 1);
     fence_barrier_init();
     tma_prefetch_desc(&tm);
-    mbar_arrive_expect_tx(&s_full, box_bytes);
-    tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * cc, g.x0, g.y0, a.anchor_frame[j0]);
+    // the first kStages anchors of the segment are in flight at once
+    for (int st = 0; st < kStages && j0 + st <= j1; ++st) {
+      mbar_arrive_expect_tx(&s_full[st], box_bytes);
+      tma_load_4d(stages + st * (stage_bytes<T>(cc) / sizeof(T)), &tm, &s_full[st], chunk * cc, g.x0,
+                  g.y0, a.anchor_frame[j0 + st]);
+    }
   }
   launch_dependents();
   __syncthreads();
@@ -439,7 +447,9 @@ __global__ void __launch_bounds__(CC, FULL ? 3 : 2)
   for (int j = j0; j <= j1; ++j) {
     float re[8][5], im[8][5];
     {
-      const bool got = ok && mbar_wait(&s_full, (uint32_t)(j - j0) & 1u, a.wait_ns);
+      const int it = j - j0, st = it % kStages;
+      const T* stage = stages + st * (stage_bytes<T>(cc) / sizeof(T));
+      const bool got = ok && mbar_wait(&s_full[st], (uint32_t)(it / kStages) & 1u, a.wait_ns);
       float x[8][8];
       if (FULL) {
 #pragma unroll
@@ -453,14 +463,15 @@ __global__ void __launch_bounds__(CC, FULL ? 3 : 2)
           for (int xx = 0; xx < 8; ++xx)
             x[y][xx] = (y < g.h && xx < g.w) ? to_f32(stage[(y * a.tw + xx) * cc + tid]) : 0.f;
       }
-      // the stage is free: prefetch the next anchor while this one is transformed
+      // the stage is free: the anchor kStages ahead goes into it while this one is transformed
       if (__syncthreads_or(ok && !got)) {
         if (tid == 0) atomicExch(&g_par_error, 1u);
         ok = false;
       }
-      if (ok && tid == 0 && j + 1 <= j1) {
-        mbar_arrive_expect_tx(&s_full, box_bytes);
-        tma_load_4d(const_cast<T*>(stage), &tm, &s_full, chunk * cc, g.x0, g.y0, a.anchor_frame[j + 1]);
+      if (ok && tid == 0 && j + kStages <= j1) {
+        mbar_arrive_expect_tx(&s_full[st], box_bytes);
+        tma_load_4d(const_cast<T*>(stage), &tm, &s_full[st], chunk * cc, g.x0, g.y0,
+                    a.anchor_frame[j + kStages]);
       }
       if (FULL) dft::fwd2d(x, 8, 8, re, im);
       else dft::fwd2d(x, g.h, g.w, re, im);
@@ -603,8 +614,15 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
     }
     float sum = 0.f;
     if (k >= 0) {
+      // chunk order; eight loads in flight per round
       const float* r = a.rec + ((int64_t)tg * a.n_anchor + j) * a.n_chunk * kRec + k;
-      for (int ch = 0; ch < a.n_chunk; ++ch) sum += __ldcg(r + (int64_t)ch * kRec);
+      for (int ch0 = 0; ch0 < a.n_chunk; ch0 += 8) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = ch0 + u < a.n_chunk ? __ldcg(r + (int64_t)(ch0 + u) * kRec) : 0.f;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) sum += v[u];
+      }
     }
     s_zw[tid] = sign < 0 ? -sum : sum;
   }
