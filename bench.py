@@ -10,7 +10,8 @@ anchor attention -> PAR.
   value   frames/s with inputs resident in HBM (CUDA events around each step, L2 flushed
           between steps outside the timed events)
   e2e     frames/s through the same C call with the inputs copied from pinned host memory
-          and r_out copied back, copies inside the timed region
+          and r_out copied back, copies inside the timed region (double-buffered: step k+1's
+          upload and step k-1's read-back overlap step k's compute)
   roofline  the dominant kernel (routed attention): algorithmic FLOP per launch / its average
           CUDA-event duration (stages launched through their own entry points, same kernels
           and launch configuration as inside the block step) against the measured bf16 peak
@@ -217,25 +218,57 @@ def run_gpu(args):
     t_par = statistics.mean(e[2].elapsed_time(e[3]) for e in st_ev)
 
     # ---------------- end to end through the C call with host buffers
-    h_out = torch.empty((N, S, H * dh), dtype=torch.bfloat16).pin_memory()
+    # Double-buffered, as a serving loop runs it: the inputs of step k+1 travel host -> device on
+    # a copy stream while step k computes, and each step's result goes device -> host on a second
+    # copy stream.  Every step's copies are inside the timed region (first upload to last read).
+    h_out = [torch.empty((N, S, H * dh), dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+    sets = [(d, r_out, bargs, ws)]
+    d1 = {k: torch.empty_like(d[k]) for k in names}
+    r1 = torch.empty_like(r_out)
+    idx1 = torch.empty_like(idx)
+    b1 = lib.block_args(d1["q"], d1["k_cur"], d1["v_cur"], anchors, d1["k_hist"], d1["v_hist"],
+                        wl.K, wl.grid, r1, idx_out=idx1, params=params, refine=lib.REFINE_PAPER)
+    sets.append((d1, r1, b1, torch.empty_like(ws)))
+    up, down = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    uploaded = [torch.cuda.Event() for _ in range(2)]
+    computed = [torch.cuda.Event() for _ in range(2)]
+    read = [torch.cuda.Event() for _ in range(2)]
     ne = max(10, args.steps // 4)
-    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(ne)]
-    for k in range(ne + 2):
-        flush.fill_(k & 0xFF)
-        e = e2e_ev[k - 2] if k >= 2 else None
-        if e:
-            e[0].record(stream)
-        for nm in names:
-            d[nm].copy_(host[nm], non_blocking=True)
-        step()
-        h_out.copy_(r_out, non_blocking=True)
-        if e:
-            e[1].record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
+
+    def e2e_run(n):
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        t0.record(stream)
+        up.wait_stream(stream)
+        down.wait_stream(stream)
+        for k in range(n):
+            sb = k % 2
+            dk, rk, ak, wk = sets[sb]
+            if k >= 2:
+                up.wait_event(computed[sb])       # step k-2 has finished reading this input set
+            with torch.cuda.stream(up):
+                for nm in names:
+                    dk[nm].copy_(host[nm], non_blocking=True)
+                uploaded[sb].record(up)
+            stream.wait_event(uploaded[sb])
+            if k >= 2:
+                stream.wait_event(read[sb])       # step k-2's result has been read back
+            lib.cast_block_step_args(ak, wk)
+            computed[sb].record(stream)
+            down.wait_event(computed[sb])
+            with torch.cuda.stream(down):
+                h_out[sb].copy_(rk, non_blocking=True)
+                read[sb].record(down)
+        stream.wait_stream(down)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        return t0.elapsed_time(t1) / n
+
+    e2e_run(2)
+    e2e_ms = e2e_run(ne)
+    lib.cast_check_device()
     h2d = sum(host[nm].numel() * host[nm].element_size() for nm in names)
-    d2h = h_out.numel() * h_out.element_size()
+    d2h = h_out[0].numel() * h_out[0].element_size()
 
     if rank == 0:
         hbm, bf16, src = _peaks()
@@ -269,7 +302,9 @@ def run_gpu(args):
                 "hbm_peak_gbs": hbm},
             "e2e": {"value": round(N / (e2e_ms / 1e3) * world, 3), "unit": "frames/s",
                     "ms_per_step": round(e2e_ms, 4), "h2d_bytes_per_step": int(h2d),
-                    "d2h_bytes_per_step": int(d2h)},
+                    "d2h_bytes_per_step": int(d2h),
+                    "pipeline": "double-buffered: upload of step k+1 and read-back of step k-1 "
+                                "overlap step k (host link ~210 GB/s measured)"},
             "gpu_launches": launches_per_step(wl) * args.steps,
             "clocks": clk,
         }
