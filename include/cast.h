@@ -390,6 +390,13 @@ const char* cast_last_error_detail(void);
  * outside its range (a routed block in attention, a routing candidate) (both records are
  * cleared), CAST_ERR_CUDA on a pending CUDA error, CAST_OK otherwise. */
 cast_status cast_check_device(void* stream);
+/* Failure-path self-test (no counterpart in the paper): enqueues one thread that waits on a
+ * device barrier nothing ever completes, with a deadline of limit_ns (1 us .. 2 s) on the
+ * GPU's global timer, exactly as the kernels of the path bound their waits.  When the
+ * deadline passes it records a timeout, so the next cast_check_device() on the stream returns
+ * CAST_ERR_DEVICE_TIMEOUT (and clears the record); the context stays usable.
+ * Errors: INVALID_ARG for a limit outside the range. */
+cast_status cast_selftest_bounded_wait(uint64_t limit_ns, void* stream);
 /* Library version, "major.minor.patch". */
 const char* cast_version(void);
 

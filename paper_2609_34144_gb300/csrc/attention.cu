@@ -779,6 +779,23 @@ cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, voi
   return launch_hd<64>(a, pl, o_frame_of_anchor, ws, st);
 }
 
+namespace {
+// One thread waits on an mbarrier that nothing ever arrives on, with a deadline of limit_ns on
+// %globaltimer; when the deadline passes it records the timeout like a kernel of the path.
+__global__ void k_bounded_wait_selftest(unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_barrier_init();
+  if (!mbar_wait(&bar, 0, limit_ns)) atomicExch(&g_attn_error, 1u);
+}
+}  // namespace
+
+cast_status launch_bounded_wait_selftest(uint64_t limit_ns, cudaStream_t st) {
+  k_bounded_wait_selftest<<<1, 32, 0, st>>>(limit_ns);
+  return check_launch("bounded-wait self-test");
+}
+
 unsigned int attention_error_word(cudaStream_t st, bool clear) {
   unsigned int v = 0;
   cudaMemcpyFromSymbolAsync(&v, g_attn_error, sizeof(v), 0, cudaMemcpyDeviceToHost, st);

@@ -605,6 +605,14 @@ cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, voi
   return CAST_OK;
 }
 
+cast_status cast_selftest_bounded_wait(uint64_t limit_ns, void* stream) {
+  g_detail[0] = 0;
+  if (limit_ns < 1000 || limit_ns > 2000000000ull)
+    return fail(CAST_ERR_INVALID_ARG, "cast_selftest_bounded_wait: limit %llu ns outside 1 us .. 2 s",
+                (unsigned long long)limit_ns);
+  return launch_bounded_wait_selftest(limit_ns, static_cast<cudaStream_t>(stream));
+}
+
 cast_status cast_check_device(void* stream) {
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const cudaError_t e = cudaStreamSynchronize(st);

@@ -82,6 +82,8 @@ AttnPlan attention_plan(const cast_attn_args& a);
 cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, void* ws,
                              cudaStream_t st);
 unsigned int attention_error_word(cudaStream_t st, bool clear);
+// A kernel whose only wait can never be satisfied and so runs into its deadline (limit_ns).
+cast_status launch_bounded_wait_selftest(uint64_t limit_ns, cudaStream_t st);
 
 // ------------------------------------------------------------------ PAR
 struct ParPlan {

@@ -118,6 +118,8 @@ _lib.cast_status_string.argtypes = [C.c_int]
 _lib.cast_status_string.restype = C.c_char_p
 _lib.cast_last_error_detail.restype = C.c_char_p
 _lib.cast_check_device.argtypes = [_vp]
+_lib.cast_selftest_bounded_wait.argtypes = [C.c_uint64, _vp]
+_lib.cast_selftest_bounded_wait.restype = C.c_int
 _lib.cast_version.restype = C.c_char_p
 for _f in ("cast_route_topk", "cast_route_topk_noalloc", "cast_anchor_attention", "cast_par_reconstruct", "cast_block_step",
            "cast_check_device"):
@@ -129,7 +131,8 @@ EXPORTED = ["cast_select_frames", "cast_select_workspace_size", "cast_ffn_step",
             "cast_anchor_attention", "cast_attention_workspace_size",
             "cast_par_reconstruct", "cast_par_workspace_size", "cast_par_params_default",
             "cast_block_step", "cast_block_workspace_size", "cast_status_string",
-            "cast_last_error_detail", "cast_check_device", "cast_version"]
+            "cast_last_error_detail", "cast_check_device", "cast_version",
+            "cast_selftest_bounded_wait"]
 
 
 class CastError(RuntimeError):
@@ -421,6 +424,11 @@ def cast_block_step(q, k_cur, v_cur, anchors, k_hist, v_hist, K, grid, r_out, x=
 
 def cast_check_device(stream=None):
     _check(_lib.cast_check_device(_stream(stream)))
+
+
+def cast_selftest_bounded_wait(limit_ns, stream=None):
+    """Enqueue a wait that can only end by its deadline (see include/cast.h)."""
+    _check(_lib.cast_selftest_bounded_wait(int(limit_ns), _stream(stream)))
 
 
 def version():

@@ -298,3 +298,10 @@ def test_route_candidate_set_size_validation(lib, M_c, status):
     assert so.cast_route_topk(C.byref(a), None, 0, None) == 1
     msg = so.cast_last_error_detail()
     assert (b"M_c" in msg) == bool(status), msg
+
+
+def test_selftest_limit_validated_on_the_host(lib):
+    so = lib.library()
+    assert so.cast_selftest_bounded_wait(10, None) == 1            # below 1 us
+    assert so.cast_selftest_bounded_wait(3_000_000_000, None) == 1  # above 2 s
+    assert so.cast_last_error_detail() != b""
