@@ -562,13 +562,15 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
           // affine in x_i, so the accepted step lowers J by exactly that gain
           const float* Gk = restricted ? Gc : G;
           float gl = 0.f;
-          for (int m = lane; m < M; m += 32) {
-            const float nx = in_topk(Gk, M, K, m) ? 1.f : 0.f;
-            gl += G[m] * (nx - x[i * M + m]);
+          uint32_t sel = 0u;   // this lane's memberships (bit r: block lane + 32 r; M <= 1024 here)
+          for (int m = lane, r = 0; m < M; m += 32, ++r) {
+            const bool in = in_topk(Gk, M, K, m);
+            sel |= (uint32_t)in << r;
+            gl += G[m] * ((in ? 1.f : 0.f) - x[i * M + m]);
           }
           const float gain = warp_total(gl);
           if (gain > a.tol * fmaxf(J, 1e-8f)) {   // uniform across the warp
-            for (int m = lane; m < M; m += 32) x[i * M + m] = in_topk(Gk, M, K, m) ? 1.f : 0.f;
+            for (int m = lane, r = 0; m < M; m += 32, ++r) x[i * M + m] = ((sel >> r) & 1u) ? 1.f : 0.f;
             J -= gain;
             changed = true;
           }
@@ -1127,7 +1129,7 @@ constexpr size_t kHeadSmemLimit = 200 * 1024;
 size_t head_staged_bytes(const cast_route_args& a) {
   return align_up(head_state_bytes(a), 16) + (size_t)2 * a.M * a.d * sizeof(float);
 }
-bool head_stages_kv(const cast_route_args& a) { return head_staged_bytes(a) <= kHeadSmemLimit; }
+bool head_stages_kv(const cast_route_args& a) { return a.M <= 1024 && head_staged_bytes(a) <= kHeadSmemLimit; }
 
 size_t wide_bytes(const cast_route_args& a) {
   const int K_eff = a.K < a.M ? a.K : a.M;
