@@ -302,9 +302,9 @@ typedef struct {
 } cast_block_args;
 
 /* route_topk -> anchor_attention -> (output projection) -> par_reconstruct on one stream,
- * then the optional residual update x += r_out.  The projection is a plain GEMM run through
- * cuBLASLt with the caller's workspace.  Errors: those of the steps; INVALID_ARG for a
- * misaligned w_o / b_o. */
+ * then the optional residual update x += r_out.  The projection of every anchor's rows is
+ * one tcgen05 GEMM launch (bias epilogue) on the caller's stream.  Errors: those of the steps;
+ * INVALID_ARG for a misaligned w_o / b_o. */
 cast_status cast_block_step(const cast_block_args* args, void* workspace,
                             size_t workspace_bytes, void* stream);
 size_t cast_block_workspace_size(const cast_block_args* args);
@@ -332,9 +332,11 @@ typedef struct {
 
 /* For every anchor frame a: r_out[a] = GELU(x[a] W1^T + b1) W2^T + b2 (GELU in its tanh
  * form, the hidden activations rounded to bf16 between the two GEMMs), then
- * par_reconstruct(r_out) over the skipped frames.  The two GEMMs are plain GEMMs run through
- * cuBLASLt with the caller's workspace.  Errors: INVALID_ARG for bad shapes, strides or
- * pointers, anchors as in cast_block_step, a short workspace; those of par_reconstruct. */
+ * par_reconstruct(r_out) over the skipped frames.  Each GEMM is one tcgen05 launch over the
+ * rows of every anchor (bias, and GELU, in its epilogue); the workspace holds the hidden
+ * activations [n_anchors, S, D_ff] bf16 and PAR's records.  Errors: INVALID_ARG for bad
+ * shapes, strides or pointers, anchors as in cast_block_step, a short workspace; those of
+ * par_reconstruct. */
 cast_status cast_ffn_step(const cast_ffn_args* args, void* workspace, size_t workspace_bytes,
                           void* stream);
 size_t cast_ffn_workspace_size(const cast_ffn_args* args);

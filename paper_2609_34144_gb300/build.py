@@ -46,9 +46,7 @@ def build(verbose_ptxas: bool = False, quiet: bool = True) -> str:
                 print(log, file=sys.stderr)
     objs = [o for (o, _) in results]
     tmp = LIB + ".tmp"
-    cuda_lib = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "lib64")
-    cmd = [nvcc(), *ARCH, "-shared", "-o", tmp, *objs, "-L", cuda_lib, "-lcublasLt",
-           "-Xlinker", "-rpath=" + cuda_lib, "-lrt", "-lpthread", "-ldl"]
+    cmd = [nvcc(), *ARCH, "-shared", "-o", tmp, *objs, "-lrt", "-lpthread", "-ldl"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")

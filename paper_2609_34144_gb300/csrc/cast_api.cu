@@ -321,8 +321,8 @@ BlockPlan block_plan(const cast_block_args* a) {
   uint8_t mask[CAST_MAX_FRAMES];
   cast_par_args p = par_of_block(a, mask);
   b.par_bytes = par_plan(p).total_bytes;
-  // with W_O: the attention output [n_anchors, S, H*d] bf16, then the GEMM scratch
-  b.proj_bytes = a->w_o ? align_up((size_t)a->n_anchors * a->Hg * a->Wg * a->H * a->d * 2) + kGemmWorkspace : 0;
+  // with W_O: the attention output [n_anchors, S, H*d] bf16
+  b.proj_bytes = a->w_o ? align_up((size_t)a->n_anchors * a->Hg * a->Wg * a->H * a->d * 2) : 0;
   b.total = b.route_bytes + b.idx_bytes + b.attn_bytes + b.par_bytes + b.proj_bytes;
   return b;
 }
@@ -473,25 +473,29 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
     t.o = proj;
     t.o_dtype = CAST_BF16;
     if ((s = launch_attention(t, 0, w + bp.route_bytes + bp.idx_bytes, st))) return s;
-    const size_t elt = a->r_dtype == CAST_BF16 ? 2 : 4;
+    (void)o_bytes;
+    AnchorGemm g{};
+    g.a = proj;
+    g.lda = D;
+    g.a_frame_stride = (int64_t)S * D;
+    g.a_frames = a->n_anchors;
+    g.w = a->w_o;
+    g.ldw = D;
+    g.bias = a->b_o;
+    g.bias_dtype = a->r_dtype;
+    g.c = a->r_out;
+    g.ldc = D;
+    g.c_dtype = a->r_dtype;
+    g.S = S;
+    g.N = D;
+    g.K = D;
+    g.n_anchors = a->n_anchors;
     for (int i = 0; i < a->n_anchors; ++i) {
-      GemmRows g{};
-      g.a = proj + (size_t)i * S * D * 2;
-      g.lda = D;
-      g.w = a->w_o;
-      g.ldw = D;
-      g.bias = a->b_o;
-      g.c = static_cast<char*>(a->r_out) + (size_t)a->anchors[i] * S * D * elt;
-      g.ldc = D;
-      g.c_dtype = a->r_dtype;
-      g.M = S;
-      g.N = D;
-      g.K = D;
-      g.gelu = false;
-      g.ws = proj + o_bytes;
-      g.ws_bytes = kGemmWorkspace;
-      if ((s = gemm_rows(g, st))) return s;
+      g.a_frame[i] = i;
+      g.c_frame[i] = a->anchors[i];
     }
+    g.gelu = false;
+    if ((s = gemm_anchor_rows(g, st))) return s;
   }
   if (par_plan(p).n_target > 0) {
     if ((s = launch_par(p, w + bp.route_bytes + bp.idx_bytes + bp.attn_bytes, st))) return s;
@@ -532,7 +536,7 @@ size_t cast_ffn_workspace_size(const cast_ffn_args* a) {
   uint8_t mask[CAST_MAX_FRAMES];
   const cast_par_args p = par_of_ffn(a, mask);
   const size_t par = (p.params.tile_h >= 1 && p.params.tile_w >= 1 && p.C >= 1) ? par_plan(p).total_bytes : 0;
-  return align_up((size_t)a->Hg * a->Wg * a->D_ff * 2) + kGemmWorkspace + align_up(par);
+  return align_up((size_t)a->n_anchors * a->Hg * a->Wg * a->D_ff * 2) + align_up(par);
 }
 
 cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, void* stream) {
@@ -562,45 +566,51 @@ cast_status cast_ffn_step(const cast_ffn_args* a, void* ws, size_t ws_bytes, voi
     return fail(CAST_ERR_INVALID_ARG, "%s: workspace not 256-byte aligned", who);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const int S = a->Hg * a->Wg;
+  // hidden activations of every anchor [n_anchors, S, D_ff] bf16, then the PAR workspace
   char* hid = static_cast<char*>(ws);
-  char* gws = hid + align_up((size_t)S * a->D_ff * 2);
-  char* pws = gws + kGemmWorkspace;
-  const size_t elt = a->r_dtype == CAST_BF16 ? 2 : 4;
+  char* pws = hid + align_up((size_t)a->n_anchors * S * a->D_ff * 2);
+  AnchorGemm g1{};
+  g1.a = a->x;
+  g1.lda = a->x_row_stride;
+  g1.a_frame_stride = (int64_t)S * a->x_row_stride;
+  g1.a_frames = a->n_frames;
+  g1.w = a->w1;
+  g1.ldw = a->D;
+  g1.bias = a->b1;
+  g1.bias_dtype = CAST_BF16;
+  g1.c = hid;
+  g1.ldc = a->D_ff;
+  g1.c_dtype = CAST_BF16;
+  g1.S = S;
+  g1.N = a->D_ff;
+  g1.K = a->D;
+  g1.n_anchors = a->n_anchors;
+  g1.gelu = true;
+  AnchorGemm g2{};
+  g2.a = hid;
+  g2.lda = a->D_ff;
+  g2.a_frame_stride = (int64_t)S * a->D_ff;
+  g2.a_frames = a->n_anchors;
+  g2.w = a->w2;
+  g2.ldw = a->D_ff;
+  g2.bias = a->b2;
+  g2.bias_dtype = a->r_dtype;
+  g2.c = a->r_out;
+  g2.ldc = a->D;
+  g2.c_dtype = a->r_dtype;
+  g2.S = S;
+  g2.N = a->D;
+  g2.K = a->D_ff;
+  g2.n_anchors = a->n_anchors;
+  g2.gelu = false;
   for (int i = 0; i < a->n_anchors; ++i) {
-    const int f = a->anchors[i];
-    GemmRows g1{};
-    g1.a = static_cast<const char*>(a->x) + (size_t)f * S * a->x_row_stride * 2;
-    g1.lda = a->x_row_stride;
-    g1.w = a->w1;
-    g1.ldw = a->D;
-    g1.bias = a->b1;
-    g1.c = hid;
-    g1.ldc = a->D_ff;
-    g1.c_dtype = CAST_BF16;
-    g1.M = S;
-    g1.N = a->D_ff;
-    g1.K = a->D;
-    g1.gelu = true;
-    g1.ws = gws;
-    g1.ws_bytes = kGemmWorkspace;
-    if ((s = gemm_rows(g1, st))) return s;
-    GemmRows g2{};
-    g2.a = hid;
-    g2.lda = a->D_ff;
-    g2.w = a->w2;
-    g2.ldw = a->D_ff;
-    g2.bias = a->b2;
-    g2.c = static_cast<char*>(a->r_out) + (size_t)f * S * a->D * elt;
-    g2.ldc = a->D;
-    g2.c_dtype = a->r_dtype;
-    g2.M = S;
-    g2.N = a->D;
-    g2.K = a->D_ff;
-    g2.gelu = false;
-    g2.ws = gws;
-    g2.ws_bytes = kGemmWorkspace;
-    if ((s = gemm_rows(g2, st))) return s;
+    g1.a_frame[i] = a->anchors[i];
+    g1.c_frame[i] = i;
+    g2.a_frame[i] = i;
+    g2.c_frame[i] = a->anchors[i];
   }
+  if ((s = gemm_anchor_rows(g1, st))) return s;
+  if ((s = gemm_anchor_rows(g2, st))) return s;
   if (par_plan(p).n_target > 0) return launch_par(p, pws, st);
   return CAST_OK;
 }
@@ -620,7 +630,8 @@ cast_status cast_check_device(void* stream) {
   const unsigned int wa = attention_error_word(st, true);
   const unsigned int wp = par_error_word(st, true);
   const unsigned int wr = route_error_word(st, true);
-  if (wa == 1u || wp) return fail(CAST_ERR_DEVICE_TIMEOUT, "a kernel gave up on a bounded wait");
+  const unsigned int wd = dense_error_word(st, true);
+  if (wa == 1u || wp || wd) return fail(CAST_ERR_DEVICE_TIMEOUT, "a kernel gave up on a bounded wait");
   if (wa == 2u) return fail(CAST_ERR_INVALID_ARG, "attention: a routed block index was outside [0, M)");
   if (wr) return fail(CAST_ERR_INVALID_ARG, "routing: a candidate index was outside [0, M) or repeated");
   return check_launch("cast_check_device");

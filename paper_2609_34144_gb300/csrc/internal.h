@@ -100,24 +100,27 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st);
 unsigned int par_error_word(cudaStream_t st, bool clear);
 
 // ------------------------------------------------------------------ dense projections
-constexpr size_t kGemmWorkspace = (size_t)32 << 20;   // cuBLASLt scratch per GEMM call
-// Row-major C[M, N] = act(A[M, K] W[N, K]^T + bias[N]), A and W bf16 (16-byte aligned rows),
-// C and bias of c_dtype; act = GELU (cuBLASLt epilogue) when gelu.
-struct GemmRows {
+// C[anchor i, row r, :] = act(A[a_frame[i], r, :] W[N, K]^T + bias[N]) for r < S: A, W bf16
+// (16-byte aligned rows, lda / ldw multiples of 8), row r of anchor i of A at
+// a + (a_frame[i] * a_frame_stride + r * lda), of C at c + (c_frame[i] * S + r) * ldc; C and
+// bias of their dtypes; act = GELU (tanh form) when gelu.  One tcgen05 kernel per call.
+struct AnchorGemm {
   const void* a;
-  int64_t lda;
+  int64_t lda, a_frame_stride;
+  int a_frames;                  // frames the A tensor holds (its tensor map depth)
   const void* w;
   int64_t ldw;
   const void* bias;
+  int bias_dtype;
   void* c;
   int64_t ldc;
   int c_dtype;
-  int M, N, K;
+  int S, N, K, n_anchors;
+  int a_frame[CAST_MAX_ANCHORS], c_frame[CAST_MAX_ANCHORS];
   bool gelu;
-  void* ws;
-  size_t ws_bytes;
 };
-cast_status gemm_rows(const GemmRows& g, cudaStream_t st);
+cast_status gemm_anchor_rows(const AnchorGemm& g, cudaStream_t st);
+unsigned int dense_error_word(cudaStream_t st, bool clear);
 
 // ------------------------------------------------------------------ residual update
 cast_status launch_residual_add(void* x, const void* r, int dtype, size_t n, cudaStream_t st);

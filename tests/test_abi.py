@@ -212,7 +212,9 @@ def test_ffn_validation(lib):
     a.par = lib.default_par_params()
     so = lib.library()
     need = so.cast_ffn_workspace_size(C.byref(a))
-    assert need > 32 << 20
+    # hidden activations [2 anchors, 16 rows, 256] bf16, then PAR's records and theta / g of the
+    # single (4x4) tile: 2 anchors x 1 chunk x 120 floats and 2 x 80 floats, each 256-B aligned
+    assert need == 2 * 16 * 256 * 2 + 1024 + 768
     assert so.cast_ffn_step(C.byref(a), _fake(0x100000), need - 1, None) == 1      # short workspace
     a.D = 60
     assert so.cast_ffn_step(C.byref(a), _fake(0x100000), need, None) == 1          # D not a multiple of 8
