@@ -498,12 +498,12 @@ def _captured_traffic():
 # ------------------------------------------------------------------------------ CPU oracle
 def launches_per_step(wl):
     """Library kernels one block step launches: pooling (anchor frames, history blocks) and
-    the per-head routing kernel, attention, and PAR (one kernel for full 8x8 tiles, one for
-    truncated edge tiles when the grid has both)."""
+    the per-head routing kernel, attention, and PAR (statistics, transport and blend passes
+    for the full 8x8 tiles and for the truncated edge tiles when the grid has both)."""
     hg, wg = wl.grid
     full = (hg // 8) * (wg // 8) > 0
     edge = hg % 8 != 0 or wg % 8 != 0
-    return 3 + 1 + (int(full) + int(edge))
+    return 3 + 1 + 3 * (int(full) + int(edge))
 
 
 def _oracle_sample(wl, inp, R, heads, row_stride, tiles):
