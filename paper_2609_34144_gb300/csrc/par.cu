@@ -401,7 +401,7 @@ __host__ __device__ constexpr size_t par_dyn_smem(int cc) {
 // one channel each.  A time segment covers the anchor pairs seg_pair0 .. seg_pair1 (it starts
 // one anchor earlier).  FULL: every tile of the launch is 8x8 (the specialised fast path).
 template <typename T, int CC, bool FULL, bool STATS>
-__global__ void __launch_bounds__(CC, FULL ? 3 : 2)
+__global__ void __launch_bounds__(CC, 3)
     k_par(const __grid_constant__ CUtensorMap tm, const __grid_constant__ ParKArgs a) {
   extern __shared__ uint8_t dsm_raw[];
   const uint32_t raw = smem_u32(dsm_raw);
