@@ -32,6 +32,9 @@
 // part that arrives last merges them (exp2-weighted by the row maxima).
 // Every wait is bounded; on a timeout the CTA records an error word, drains its UMMAs and
 // frees TMEM before leaving.
+// Inside the block step the kernel is a programmatic dependent of the routing kernel: its CTAs
+// start on the current-chunk tiles while routing finishes, and each thread that reads the
+// routed block indices waits on the grid dependency just before its first history tile.
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -112,6 +115,15 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 // Whole-CTA barrier reached from the code of different roles (non-aligned form, barrier 1).
 __device__ __forceinline__ void end_barrier() {
   asm volatile("barrier.sync 1, %0;" ::"n"(kThreads) : "memory");
+}
+
+// Waits (once per thread) until the grid this one depends on has completed and its writes
+// (the routed block indices) are visible; a no-op for an ordinary launch.
+__device__ __forceinline__ void wait_routing(bool& waited) {
+  if (!waited) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    waited = true;
+  }
 }
 
 __device__ __forceinline__ bool aborted(const Bars* b) {
@@ -272,7 +284,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int b = 0; b < HD / 64; ++b)
           tma_load_3d(sQ + t * C::Q_BYTES + b * BM * 128, &tm_q, &bars->q_full, h * HD + b * 64,
                       row0 + t * BM, a.q_frame[i]);
+      bool waited = false;
       for (int j = 0; j < n_tiles; ++j) {
+        if (k0 + j >= a.n_cur_tiles) wait_routing(waited);
         const TileCoord c = tile_coord(a, i, h, k0 + j);
         const int s = j % kStages;
         if (aborted(bars) || !mbar_wait(&bars->k_empty[s], ((uint32_t)(j / kStages) & 1u) ^ 1u, lim)) {
@@ -300,7 +314,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (lane == 1) {
       tma_prefetch_desc(&tm_vc);
       tma_prefetch_desc(&tm_vh);
+      bool waited = false;
       for (int j = 0; j < n_tiles; ++j) {
+        if (k0 + j >= a.n_cur_tiles) wait_routing(waited);
         const TileCoord c = tile_coord(a, i, h, k0 + j);
         const int s = j % kStages;
         if (aborted(bars) || !mbar_wait(&bars->v_empty[s], ((uint32_t)(j / kStages) & 1u) ^ 1u, lim)) {
@@ -411,11 +427,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t colS = t * BN, colO = 256 + t * 128;
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
+    bool waited = false;
     for (int j = 0; j < n_tiles; ++j) {
       const int jg = k0 + j;   // global K/V tile
       // spatial history tile: the routed block indices are fetched before the wait
       int sm0 = -1, sm1 = -1;
       if (a.spatial && jg >= a.n_cur_tiles) {
+        wait_routing(waited);
         const int jj = jg - a.n_cur_tiles;
         sm0 = routed_block(a, i, h, 2 * jj);
         sm1 = 2 * jj + 1 < a.K_eff ? routed_block(a, i, h, 2 * jj + 1) : -1;
@@ -651,7 +669,7 @@ bool make_map_frames(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
 
 template <int HD>
 cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_of_anchor, void* ws,
-                      cudaStream_t st) {
+                      cudaStream_t st, bool after_route) {
   using C = Cfg<HD>;
   const int D = a.H * HD;
   CUtensorMap mq, mkc, mvc, mkh, mvh;
@@ -723,10 +741,23 @@ cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_o
       return check_launch("attention smem attribute");
     attr_set = true;
   }
-  if (pl.n_tail > 0 &&
+  // after routing the caller has reset the tail counters before the routing launches, so that
+  // this launch follows the routing kernel directly (programmatic dependent launch)
+  if (!after_route && pl.n_tail > 0 &&
       cudaMemsetAsync(k.counters, 0, (size_t)pl.n_tail * sizeof(unsigned), st) != cudaSuccess)
     return check_launch("attention counter reset");
-  k_attn<HD><<<pl.grid, kThreads, C::SMEM, st>>>(mq, mkc, mvc, mkh, mvh, k);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(pl.grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = after_route ? 1 : 0;
+  if (cudaLaunchKernelEx(&cfg, k_attn<HD>, mq, mkc, mvc, mkh, mvh, k) != cudaSuccess)
+    return check_launch("attention kernel");
   return check_launch("attention kernel");
 }
 
@@ -773,10 +804,20 @@ AttnPlan attention_plan(const cast_attn_args& a) {
 }
 
 cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, void* ws,
-                             cudaStream_t st) {
+                             cudaStream_t st, bool after_route) {
   const AttnPlan pl = attention_plan(a);
-  if (a.d == 128) return launch_hd<128>(a, pl, o_frame_of_anchor, ws, st);
-  return launch_hd<64>(a, pl, o_frame_of_anchor, ws, st);
+  if (a.d == 128) return launch_hd<128>(a, pl, o_frame_of_anchor, ws, st, after_route);
+  return launch_hd<64>(a, pl, o_frame_of_anchor, ws, st, after_route);
+}
+
+cast_status attention_reset_counters(const cast_attn_args& a, void* ws, cudaStream_t st) {
+  const AttnPlan pl = attention_plan(a);
+  if (pl.n_tail == 0) return CAST_OK;
+  char* w = static_cast<char*>(ws);
+  if (cudaMemsetAsync(w + pl.part_o_bytes + pl.part_ml_bytes, 0, (size_t)pl.n_tail * sizeof(unsigned),
+                      st) != cudaSuccess)
+    return check_launch("attention counter reset");
+  return CAST_OK;
 }
 
 namespace {

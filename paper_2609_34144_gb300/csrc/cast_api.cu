@@ -460,11 +460,15 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
   if (reinterpret_cast<uintptr_t>(ws) % kWsAlign)
     return fail(CAST_ERR_INVALID_ARG, "%s: workspace not 256-byte aligned", who);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (a->M > 0 && a->K > 0) {
+  const bool routed = a->M > 0 && a->K > 0;
+  char* aws = w + bp.route_bytes + bp.idx_bytes;
+  if (routed) {
+    // the attention follows the routing kernel directly: its tail counters are reset first
+    if ((s = attention_reset_counters(t, aws, st))) return s;
     if ((s = launch_route(r, w, st))) return s;
   }
   if (!a->w_o) {
-    if ((s = launch_attention(t, 1, w + bp.route_bytes + bp.idx_bytes, st))) return s;
+    if ((s = launch_attention(t, 1, aws, st, routed))) return s;
   } else {
     // attention output of the anchors into the workspace, then r_out[a] = O_a W_O^T + b_O
     char* proj = w + bp.route_bytes + bp.idx_bytes + bp.attn_bytes + bp.par_bytes;
@@ -472,7 +476,7 @@ cast_status cast_block_step(const cast_block_args* a, void* ws, size_t ws_bytes,
     const size_t o_bytes = align_up((size_t)a->n_anchors * S * D * 2);
     t.o = proj;
     t.o_dtype = CAST_BF16;
-    if ((s = launch_attention(t, 0, w + bp.route_bytes + bp.idx_bytes, st))) return s;
+    if ((s = launch_attention(t, 0, aws, st, routed))) return s;
     (void)o_bytes;
     AnchorGemm g{};
     g.a = proj;

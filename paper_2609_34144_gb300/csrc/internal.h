@@ -79,8 +79,12 @@ AttnPlan attention_plan(const cast_attn_args& a);
 // o_frame_of_anchor: 0 -> output frame i for anchor i (o is [n_anchors, S, H*d]);
 //                    1 -> output frame anchors[i] (o is [n_frames, S, H*d], block step).
 // ws holds attention_plan(a).total_bytes (may be null when that is 0).
+// after_route: launched right behind the routing kernels as a programmatic dependent (history
+// tiles wait on the grid dependency); the caller has run attention_reset_counters() on the
+// stream before routing.
 cast_status launch_attention(const cast_attn_args& a, int o_frame_of_anchor, void* ws,
-                             cudaStream_t st);
+                             cudaStream_t st, bool after_route = false);
+cast_status attention_reset_counters(const cast_attn_args& a, void* ws, cudaStream_t st);
 unsigned int attention_error_word(cudaStream_t st, bool clear);
 // A kernel whose only wait can never be satisfied and so runs into its deadline (limit_ns).
 cast_status launch_bounded_wait_selftest(uint64_t limit_ns, cudaStream_t st);
