@@ -319,7 +319,7 @@ def run_gpu(args):
 
 # ------------------------------------------------------------------------------ scale points
 SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy", "select_mg", "ffn_mg",
-                "route_mg64", "attn_mg64", "attn_hy64", "block_mg64")
+                "route_mg64", "attn_mg64", "attn_hy64", "block_mg64", "block_hy", "block_hy64")
 
 
 def _block_tokens(wl):
@@ -397,8 +397,18 @@ def _scale_setup(name, lib, torch, dev):
                          device=dev)
         return (lambda: lib.cast_ffn_step(x, an, w1, b1, w2, b2, wl.grid, r, workspace=ws),
                 4.0 * len(an) * S * D * Dff, "FLOP")
-    if name in ("route_mg64", "attn_mg64", "attn_hy64", "block_mg64"):
-        wl = W.HY64 if name == "attn_hy64" else W.MG64
+    if name == "block_hy":
+        wl = W.HY
+        N, S, H, d = wl.n_cur, wl.S, wl.H, wl.d
+        q, kc, vc = rnd(N, S, H, d), rnd(N, S, H, d), rnd(N, S, H, d)
+        kh, vh = rnd(wl.M, wl.B_v, H, d), rnd(wl.M, wl.B_v, H, d)
+        r = torch.zeros((N, S, H * d), dtype=torch.bfloat16, device=dev)
+        a = lib.block_args(q, kc, vc, list(wl.anchors), kh, vh, wl.K, wl.grid, r,
+                           params=lib.par_params(band_radius=wl.band_radius), refine=lib.REFINE_PAPER)
+        ws = torch.empty(lib.block_workspace_size(a), dtype=torch.uint8, device=dev)
+        return (lambda: lib.cast_block_step_args(a, ws), N, "frames")
+    if name in ("route_mg64", "attn_mg64", "attn_hy64", "block_mg64", "block_hy64"):
+        wl = W.HY64 if name in ("attn_hy64", "block_hy64") else W.MG64
         N, S, H, d = wl.n_cur, wl.S, wl.H, wl.d
         an = list(wl.anchors)
         Kf = len(an)
@@ -409,7 +419,7 @@ def _scale_setup(name, lib, torch, dev):
             ws = torch.empty(lib.route_workspace_size(q, an, kh, vh, wl.K), dtype=torch.uint8, device=dev)
             return (lambda: lib.cast_route_topk(q, an, kh, vh, wl.K, workspace=ws),
                     (Kf * S + 2 * wl.hist_frames * S) * H * d * 2, "B")
-        if name == "block_mg64":
+        if name in ("block_mg64", "block_hy64"):
             r = torch.zeros((N, S, H * d), dtype=torch.bfloat16, device=dev)
             a = lib.block_args(q, kc, vc, an, kh, vh, wl.K, wl.grid, r, refine=lib.REFINE_PAPER)
             ws = torch.empty(lib.block_workspace_size(a), dtype=torch.uint8, device=dev)
