@@ -110,6 +110,22 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------ GPU arm
+def reduce_max_ms(total_ms, world, device):
+    """The job's time is the slowest rank's: max over ranks (all-reduce; identity on one rank)."""
+    if world <= 1:
+        return total_ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([total_ms], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_value(world, frames_per_rank, steps, max_ms):
+    """Frames of all ranks (each runs its own chunk: weak scaling) per second of the slowest."""
+    return world * frames_per_rank * steps / (max_ms / 1e3)
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -173,12 +189,8 @@ def run_gpu(args):
         dist.barrier()
     lib.cast_check_device()
     ms = [a.elapsed_time(b) for a, b in ev]
-    total_ms = sum(ms)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    value = world * N * args.steps / (total_ms / 1e3)
+    total_ms = reduce_max_ms(sum(ms), world, dev)
+    value = whole_job_value(world, N, args.steps, total_ms)
 
     # ---------------- per-stage breakdown (same kernels through the stage entry points)
     o_att = torch.empty((len(anchors), S, H * dh), dtype=torch.bfloat16, device=dev)
