@@ -78,6 +78,9 @@ FFN_CASES = [
     # F, grid, D, D_ff, anchors, r dtype
     (6, (11, 13), 64, 256, (1, 3), "f32"),
     (7, (9, 16), 128, 512, (0, 2, 5), "bf16"),
+    # K not a multiple of the 64-wide k-slice, N not a multiple of the 32-column epilogue chunk
+    # nor of the 256-column tile, 17 x 9 = 153 rows (a ragged second row tile), three anchors
+    (5, (17, 9), 72, 200, (0, 2, 4), "f32"),
 ]
 
 
