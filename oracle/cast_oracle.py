@@ -22,6 +22,11 @@ Readings of points where the paper is silent (each listed in the design doc):
   * optional band cut: bins with rho = sqrt((ky_s*8/h)^2 + (kx*8/w)^2) > band
     radius get g = 0 (plain interpolation); band < 0 is the paper's gate;
   * optional per-channel weights w_c >= 0 multiply both pooled sums of Eq. (cross).
+
+Parity unpinned: the full paper gate of PAR on data that is not a translation.  The
+paper prints no worked example for it; the pins fix its pieces (the transform, the
+confidence bounds and closed forms, the gate's limits g = 0 / g = 1, exact translations
+and Prop. 1), and beyond them the oracle is the definition itself.
 """
 from __future__ import annotations
 

@@ -1,6 +1,7 @@
 // Small 1-D and 2-D DFTs of tile sides 1..8 held entirely in registers (one channel per
-// thread).  Length 8 uses written-out radix-2 transforms; lengths 1..7 (edge tiles) use
-// the defining sum with compile-time twiddles.  Unnormalised: the caller folds the
+// thread).  Lengths 8 and 4 use written-out radix-2 transforms and complex length 6 two
+// length-3 transforms; the other lengths (edge tiles) use the defining sum with compile-time
+// twiddles, zero twiddles left out.  Unnormalised: the caller folds the
 // orthonormal 1/sqrt(h w) factors (Section 4.3, App. A.2) into its coefficients.
 //
 // Register layout of a tile spectrum: re[ky][kx], im[ky][kx] with ky < 8, kx < 5 (the
@@ -103,12 +104,22 @@ __host__ __device__ __forceinline__ void rfwd(const float* x, float* re, float* 
     float ar = 0.f, ai = 0.f;
 #pragma unroll
     for (int n = 0; n < N; ++n) {
-      ar += x[n] * tw_cos(N, (k * n) % N);
-      ai -= x[n] * tw_sin(N, (k * n) % N);
+      const float c = tw_cos(N, (k * n) % N), s = tw_sin(N, (k * n) % N);
+      // zero twiddles skipped at compile time (x * 0 is not foldable under IEEE rules)
+      if (c != 0.f) ar += x[n] * c;
+      if (s != 0.f) ai -= x[n] * s;
     }
     re[k] = ar;
     im[k] = ai;
   }
+}
+
+template <>
+__host__ __device__ __forceinline__ void rfwd<4>(const float* x, float* re, float* im) {
+  const float s02 = x[0] + x[2], s13 = x[1] + x[3];
+  re[0] = s02 + s13;      im[0] = 0.f;
+  re[1] = x[0] - x[2];    im[1] = x[3] - x[1];
+  re[2] = s02 - s13;      im[2] = 0.f;
 }
 
 template <>
@@ -134,10 +145,22 @@ __host__ __device__ __forceinline__ void rinv(const float* re, const float* im, 
     float acc = re[0];
     if (N % 2 == 0) acc += (n % 2 ? -re[N / 2] : re[N / 2]);
 #pragma unroll
-    for (int k = 1; k <= (N - 1) / 2; ++k)
-      acc += 2.f * (re[k] * tw_cos(N, (k * n) % N) - im[k] * tw_sin(N, (k * n) % N));
+    for (int k = 1; k <= (N - 1) / 2; ++k) {
+      const float c = 2.f * tw_cos(N, (k * n) % N), s = 2.f * tw_sin(N, (k * n) % N);
+      if (c != 0.f) acc += re[k] * c;
+      if (s != 0.f) acc -= im[k] * s;
+    }
     x[n] = acc;
   }
+}
+
+template <>
+__host__ __device__ __forceinline__ void rinv<4>(const float* re, const float* im, float* x) {
+  const float e = re[0] + re[2], o = re[0] - re[2];
+  x[0] = e + 2.f * re[1];
+  x[2] = e - 2.f * re[1];
+  x[1] = o - 2.f * im[1];
+  x[3] = o + 2.f * im[1];
 }
 
 template <>
@@ -172,8 +195,14 @@ __host__ __device__ __forceinline__ void ccol(float (&re)[8][5], float (&im)[8][
 #pragma unroll
     for (int n = 0; n < N; ++n) {
       const float c = tw_cos(N, (k * n) % N), s = SIGN * tw_sin(N, (k * n) % N);
-      ar += xr[n] * c - xi[n] * s;
-      ai += xi[n] * c + xr[n] * s;
+      if (c != 0.f) {
+        ar += xr[n] * c;
+        ai += xi[n] * c;
+      }
+      if (s != 0.f) {
+        ar -= xi[n] * s;
+        ai += xr[n] * s;
+      }
     }
     re[k][KX] = ar;
     im[k][KX] = ai;
@@ -213,9 +242,50 @@ __host__ __device__ __forceinline__ void ccol8(float (&re)[8][5], float (&im)[8]
   }
 }
 
+template <int SIGN, int KX>
+__host__ __device__ __forceinline__ void ccol4(float (&re)[8][5], float (&im)[8][5]) {
+  fft4<SIGN>(re[0][KX], im[0][KX], re[1][KX], im[1][KX], re[2][KX], im[2][KX], re[3][KX], im[3][KX]);
+}
+
+// Length 3: A0 = a + b + c, A1,2 = a - (b + c) / 2 +- SIGN i (sqrt 3 / 2)(b - c).
+template <int SIGN>
+__host__ __device__ __forceinline__ void dft3(float& ar, float& ai, float& br, float& bi, float& cr,
+                                              float& ci) {
+  constexpr float kHalfSqrt3 = 8.660254038e-01f;
+  const float tr = br + cr, ti = bi + ci, ur = br - cr, ui = bi - ci;
+  const float mr = ar - 0.5f * tr, mi = ai - 0.5f * ti;
+  // SIGN i (sqrt 3 / 2) u
+  const float vr = -SIGN * kHalfSqrt3 * ui, vi = SIGN * kHalfSqrt3 * ur;
+  ar = ar + tr;  ai = ai + ti;
+  br = mr + vr;  bi = mi + vi;
+  cr = mr - vr;  ci = mi - vi;
+}
+
+// Length 6 by decimation in time: two length-3 transforms of the even and odd samples,
+// X[k] = E[k] + w^k O[k], X[k + 3] = E[k] - w^k O[k], w = exp(SIGN 2 pi i / 6).
+template <int SIGN, int KX>
+__host__ __device__ __forceinline__ void ccol6(float (&re)[8][5], float (&im)[8][5]) {
+  constexpr float kHalfSqrt3 = 8.660254038e-01f;
+  float e0r = re[0][KX], e0i = im[0][KX], e1r = re[2][KX], e1i = im[2][KX], e2r = re[4][KX], e2i = im[4][KX];
+  float o0r = re[1][KX], o0i = im[1][KX], o1r = re[3][KX], o1i = im[3][KX], o2r = re[5][KX], o2i = im[5][KX];
+  dft3<SIGN>(e0r, e0i, e1r, e1i, e2r, e2i);
+  dft3<SIGN>(o0r, o0i, o1r, o1i, o2r, o2i);
+  // w = 1/2 + SIGN i sqrt3/2, w^2 = -1/2 + SIGN i sqrt3/2
+  const float w1r = 0.5f * o1r - SIGN * kHalfSqrt3 * o1i, w1i = 0.5f * o1i + SIGN * kHalfSqrt3 * o1r;
+  const float w2r = -0.5f * o2r - SIGN * kHalfSqrt3 * o2i, w2i = -0.5f * o2i + SIGN * kHalfSqrt3 * o2r;
+  re[0][KX] = e0r + o0r;  im[0][KX] = e0i + o0i;
+  re[3][KX] = e0r - o0r;  im[3][KX] = e0i - o0i;
+  re[1][KX] = e1r + w1r;  im[1][KX] = e1i + w1i;
+  re[4][KX] = e1r - w1r;  im[4][KX] = e1i - w1i;
+  re[2][KX] = e2r + w2r;  im[2][KX] = e2i + w2i;
+  re[5][KX] = e2r - w2r;  im[5][KX] = e2i - w2i;
+}
+
 template <int N, int SIGN, int KX>
 __host__ __device__ __forceinline__ void col(float (&re)[8][5], float (&im)[8][5]) {
   if constexpr (N == 8) ccol8<SIGN, KX>(re, im);
+  else if constexpr (N == 6) ccol6<SIGN, KX>(re, im);
+  else if constexpr (N == 4) ccol4<SIGN, KX>(re, im);
   else ccol<N, SIGN, KX>(re, im);
 }
 

@@ -50,11 +50,15 @@ CASES = [
     (5, 9, 9, 128, (2, 4), "f32", {"tile": (4, 6)}),
     (9, 8, 8, 136, (0, 8), "f32", {}),
     (9, 8, 8, 136, (0, 8), "bf16", {"band_radius": 4.0}),
-    # one tile and three anchor pairs (one time segment per pair); 1096 channels: a cluster of
-    # 9 CTAs whose last CTA is partly empty
+    # one tile and three anchor pairs (one time segment per pair); 1096 channels: 9 channel
+    # chunks of 128, the last one partly empty
     (8, 8, 8, 1096, (0, 2, 5, 7), "f32", {}),
-    # the channel maximum: 16 CTAs of 256 channels
+    # 4096 channels: 32 chunks
     (5, 16, 24, 4096, (0, 4), "bf16", {}),
+    # edge tiles of sides 7 and 2 (15 = 8 + 7 rows, 10 = 8 + 2 columns)
+    (5, 15, 10, 72, (0, 3), "f32", {}),
+    # edge tiles of sides 6 and 4 (the Matrix-Game remainders), frame 0 extrapolated
+    (5, 14, 12, 48, (1, 4), "bf16", {}),
 ]
 
 
