@@ -289,6 +289,45 @@ __host__ __device__ __forceinline__ void col(float (&re)[8][5], float (&im)[8][5
   else ccol<N, SIGN, KX>(re, im);
 }
 
+// A column whose row transforms are real: kx = 0, and kx = w/2 for even w (the only width
+// with a fifth stored column is w = 8, whose column 4 is its Nyquist column).  Forward
+// (SIGN = -1) it holds a real signal: a real transform gives ky = 0..N/2 and the mirrors
+// N - ky follow by conjugation.  Inverse (SIGN = +1) it holds the Hermitian spectrum of a
+// real signal (the conjugate-symmetric blend of App. A.2): the real inverse reads
+// ky = 0..N/2 only and the imaginary parts of the result are zero.
+template <int N, int SIGN, int KX>
+__host__ __device__ __forceinline__ void rcol(float (&re)[8][5], float (&im)[8][5]) {
+  if constexpr (SIGN < 0) {
+    float x[N], r[N / 2 + 1], i[N / 2 + 1];
+#pragma unroll
+    for (int n = 0; n < N; ++n) x[n] = re[n][KX];
+    rfwd<N>(x, r, i);
+#pragma unroll
+    for (int k = 0; k <= N / 2; ++k) {
+      re[k][KX] = r[k];
+      im[k][KX] = i[k];
+    }
+#pragma unroll
+    for (int k = 1; k <= (N - 1) / 2; ++k) {
+      re[N - k][KX] = r[k];
+      im[N - k][KX] = -i[k];
+    }
+  } else {
+    float r[N / 2 + 1], i[N / 2 + 1], x[N];
+#pragma unroll
+    for (int k = 0; k <= N / 2; ++k) {
+      r[k] = re[k][KX];
+      i[k] = im[k][KX];
+    }
+    rinv<N>(r, i, x);
+#pragma unroll
+    for (int n = 0; n < N; ++n) {
+      re[n][KX] = x[n];
+      im[n][KX] = 0.f;
+    }
+  }
+}
+
 // -------------------------------------------------------------- 2-D, tile h x w
 template <int W>
 __host__ __device__ __forceinline__ void rows_fwd(const float (&x)[8][8], int h, float (&re)[8][5],
@@ -300,11 +339,11 @@ __host__ __device__ __forceinline__ void rows_fwd(const float (&x)[8][8], int h,
 template <int H, int SIGN>
 __host__ __device__ __forceinline__ void cols(int w, float (&re)[8][5], float (&im)[8][5]) {
   const int nkx = w / 2;
-  col<H, SIGN, 0>(re, im);
+  rcol<H, SIGN, 0>(re, im);
   if (nkx >= 1) col<H, SIGN, 1>(re, im);
   if (nkx >= 2) col<H, SIGN, 2>(re, im);
   if (nkx >= 3) col<H, SIGN, 3>(re, im);
-  if (nkx >= 4) col<H, SIGN, 4>(re, im);
+  if (nkx >= 4) rcol<H, SIGN, 4>(re, im);
 }
 template <int W>
 __host__ __device__ __forceinline__ void rows_inv(const float (&re)[8][5], const float (&im)[8][5],
