@@ -42,8 +42,9 @@ def test_candidate_topk(lib, Mc_extra):
 
 
 @pytest.mark.parametrize("Mc", [8, 13])
-def test_candidate_refinement(lib, Mc):
-    N, S, H, d, M, Bv, K = 16, 40, 6, 128, 40, 24, 8
+@pytest.mark.parametrize("M", [40, 24])
+def test_candidate_refinement(lib, Mc, M):
+    N, S, H, d, Bv, K = 16, 40, 6, 128, 24, 8
     anchors = [0, 3, 7, 12, 15]
     q, k, v = _inputs(72, N, S, H, d, M, Bv, "bf16")
     c = _sets(Mc, len(anchors), H, M, Mc)

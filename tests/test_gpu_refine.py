@@ -68,6 +68,22 @@ def test_refine_small(lib, dtype, d):
     assert amb < H
 
 
+@pytest.mark.parametrize("M,anchors", [(32, [0, 2, 4, 6, 8, 10, 12, 15]),
+                                       (20, [0, 1, 3, 5, 6, 8, 10, 11, 13, 15]),
+                                       (7, [2, 9])])
+def test_refine_small_histories(lib, M, anchors):
+    """Short histories (one warp's width of blocks and fewer) with many anchors (8 and 10:
+    every interior interval and both boundary sets) and with two anchors (both boundary sets
+    on the one pair)."""
+    N, S, H, d, Bv, K = 16, 24, 4, 64, 16, 3
+    q, k, v = _inputs(110 + M, N, S, H, d, M, Bv, "f32")
+    idx, u = lib.cast_route_topk(to_dev(q, "f32"), anchors, to_dev(k, "f32"), to_dev(v, "f32"),
+                                 K, want_u=True, refine=PAPER)
+    torch.cuda.synchronize()
+    changed, amb = check_refined(idx.cpu().numpy(), to_host(u), anchors, N, K, PAPER)
+    assert amb < H
+
+
 @pytest.mark.parametrize("passes", [1, 2, 5])
 def test_refine_passes_and_weights(lib, passes):
     N, S, H, d, M, Bv, K = 12, 30, 4, 128, 24, 16, 5
