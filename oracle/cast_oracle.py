@@ -9,7 +9,7 @@ defining double sum (as products with the DFT matrices), the softmax is
 explicit, TopK is a full sort.  Inputs are the exact values the GPU receives
 (bf16-rounded where the GPU reads bf16).
 
-Readings of points where the paper is silent (each listed in the design doc):
+Readings of points where the paper is silent, ambiguous or garbled:
   * pooled statistics are arithmetic means over tokens (Eq. pooled);
   * eps in Eq. (omission) is 1e-8 (the paper's stated epsilon of App. A.2);
   * TopK ties go to the lower block index; the selected set is returned ascending;
