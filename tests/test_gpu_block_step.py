@@ -87,3 +87,27 @@ def test_block_step_full_size(lib, wl):
     ntile = len(O.tiles_of(wl.grid[0], wl.grid[1], 8, 8))
     tiles = sorted({0, ntile - 1, int(rng.integers(0, ntile)), int(rng.integers(0, ntile))})
     _check(wl, inp, out, rows=rows, tiles=tiles)
+
+
+DEGENERATE = [
+    # every frame an anchor: PAR has nothing to reconstruct, every row is attention output
+    W.BlockStepWorkload("all_anchors_f32_3f_12x10_h2d64_m3_k2", 11, 3, (12, 10), 2, 64, 3, 40, 2,
+                        (0, 1, 2), "f32"),
+    # budget above the history: every block routed (TopK bypassed), bf16 residual
+    W.BlockStepWorkload("bypass_bf16_5f_9x13_h2d128_m3_k7", 12, 5, (9, 13), 2, 128, 3, 70, 7,
+                        (0, 4), "bf16"),
+    # one anchor pair in the middle: frames on both sides extrapolated (alpha < 0 and > 1),
+    # tiles of sides 8, 3 and 1
+    W.BlockStepWorkload("extrap_f32_6f_11x9_h1d64_m5_k2", 13, 6, (11, 9), 1, 64, 5, 33, 2,
+                        (2, 3), "f32"),
+]
+
+
+@pytest.mark.parametrize("wl", DEGENERATE, ids=lambda w: w.name)
+def test_block_step_degenerate(lib, wl):
+    inp = W.block_step_inputs(wl)
+    out = _run_block(lib, wl, inp)
+    if wl.K >= wl.M:
+        assert np.array_equal(out["idx"], np.tile(np.arange(wl.M, dtype=np.int32),
+                                                  (len(wl.anchors), wl.H, 1)))
+    _check(wl, inp, out)
