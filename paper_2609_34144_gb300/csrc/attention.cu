@@ -727,20 +727,29 @@ cast_status launch_hd(const cast_attn_args& a, const AttnPlan& pl, int o_frame_o
     k.q_frame[j] = a.anchors[j];
     k.o_frame[j] = o_frame_of_anchor ? a.anchors[j] : j;
   }
-  static bool attr_set = false;
-  if (!attr_set) {
+  static std::atomic<uint64_t> attr_done{0};
+  cast_status setup_status = CAST_OK;
+  const bool set_up = once_per_device(attr_done, [&] {
     // the register hand-over in the kernel assumes exactly kLaunchRegs per thread at launch
     cudaFuncAttributes fa{};
-    if (cudaFuncGetAttributes(&fa, k_attn<HD>) != cudaSuccess)
-      return check_launch("attention kernel attributes");
-    if (fa.numRegs != kLaunchRegs)
-      return fail(CAST_ERR_UNSUPPORTED, "attention kernel built with %d registers per thread, expected %d",
-                  fa.numRegs, kLaunchRegs);
+    if (cudaFuncGetAttributes(&fa, k_attn<HD>) != cudaSuccess) {
+      setup_status = check_launch("attention kernel attributes");
+      return false;
+    }
+    if (fa.numRegs != kLaunchRegs) {
+      setup_status = fail(CAST_ERR_UNSUPPORTED,
+                          "attention kernel built with %d registers per thread, expected %d",
+                          fa.numRegs, kLaunchRegs);
+      return false;
+    }
     if (cudaFuncSetAttribute(k_attn<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
-        cudaSuccess)
-      return check_launch("attention smem attribute");
-    attr_set = true;
-  }
+        cudaSuccess) {
+      setup_status = check_launch("attention smem attribute");
+      return false;
+    }
+    return true;
+  });
+  if (!set_up) return setup_status != CAST_OK ? setup_status : check_launch("attention setup");
   // after routing the caller has reset the tail counters before the routing launches, so that
   // this launch follows the routing kernel directly (programmatic dependent launch)
   if (!after_route && pl.n_tail > 0 &&

@@ -368,12 +368,12 @@ cast_status gemm_anchor_rows(const AnchorGemm& g, cudaStream_t st) {
     k.a_frame[j] = g.a_frame[j];
     k.c_frame[j] = g.c_frame[j];
   }
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(k_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem) != cudaSuccess)
-      return check_launch("dense GEMM smem attribute");
-    attr_set = true;
-  }
+  static std::atomic<uint64_t> attr_done{0};
+  if (!once_per_device(attr_done, [] {
+        return cudaFuncSetAttribute(k_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem) ==
+               cudaSuccess;
+      }))
+    return check_launch("dense GEMM smem attribute");
   int dev = 0, nsm = 148;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
   const int clusters = k.total_pairs < nsm / 2 ? k.total_pairs : nsm / 2;

@@ -3,6 +3,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 
@@ -24,6 +25,20 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 EncodeTiledFn tensor_map_encoder();
+
+// Runs setup() for the current device unless it already succeeded there: kernel attributes
+// (the dynamic shared-memory limit) belong to one device's context, so a process that drives
+// several devices sets them once per device.  Concurrent first calls may both run setup().
+template <class F>
+bool once_per_device(std::atomic<uint64_t>& done, F&& setup) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return setup();
+  const uint64_t bit = 1ull << dev;
+  if (done.load(std::memory_order_acquire) & bit) return true;
+  if (!setup()) return false;
+  done.fetch_or(bit, std::memory_order_acq_rel);
+  return true;
+}
 
 constexpr size_t kWsAlign = 256;
 inline size_t align_up(size_t x, size_t a = kWsAlign) { return (x + a - 1) / a * a; }

@@ -654,15 +654,14 @@ bool make_r_map(CUtensorMap* m, const cast_par_args& a, int cc) {
 template <typename T, bool FULL>
 cast_status launch_kind(const CUtensorMap& tm, const ParKArgs& k, int n_tiles, cudaStream_t st) {
   const size_t smem = par_dyn_smem<T>(kCC);
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(k_par<T, kCC, FULL, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem) != cudaSuccess ||
-        cudaFuncSetAttribute(k_par<T, kCC, FULL, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem) != cudaSuccess)
-      return check_launch("PAR kernel attributes");
-    attr_set = true;
-  }
+  static std::atomic<uint64_t> attr_done{0};
+  if (!once_per_device(attr_done, [smem] {
+        return cudaFuncSetAttribute(k_par<T, kCC, FULL, true>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess &&
+               cudaFuncSetAttribute(k_par<T, kCC, FULL, false>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess;
+      }))
+    return check_launch("PAR kernel attributes");
   cudaLaunchAttribute pdl[1];
   pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
