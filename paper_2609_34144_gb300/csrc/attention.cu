@@ -349,28 +349,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, HD, false, true);
       const uint32_t q_addr = smem_u32(sQ), k_addr = smem_u32(sK), v_addr = smem_u32(sV);
       const int nq = has_q1 ? 2 : 1;
+      // Descriptors of the first k-slice of each operand; a k-slice, query tile or stage
+      // further on adds its byte offset / 16 to the 14-bit start-address field (the whole
+      // shared-memory window is below 256 KB, so the field never carries).  This keeps the
+      // single issuing thread at a few instructions per UMMA.
+      static_assert(C::SMEM + 1024 <= 256 * 1024, "descriptor start-address field would carry");
+      static_assert(BM == BN, "Q and K tiles share their k-slice offsets");
+      const uint64_t dq = sdesc_sw128(q_addr, 16, 1024);
+      const uint64_t dk = sdesc_sw128(k_addr, 16, 1024);
+      const uint64_t dv = sdesc_sw128(v_addr, BN * 128, 1024);
       // S_t = Q_t K_j^T into the S_t columns (t * 128)
       auto qk = [&](int t, int j) {
-        const int s = j % kStages;
+        const uint64_t aq = dq + (uint64_t)((t * C::Q_BYTES) >> 4);
+        const uint64_t bk = dk + (uint64_t)(((j % kStages) * C::KV_BYTES) >> 4);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(q_addr + t * C::Q_BYTES + (kk >> 2) * (BM * 128) + (kk & 3) * 32,
-                                          16, 1024);
-          const uint64_t bd = sdesc_sw128(k_addr + s * C::KV_BYTES + (kk >> 2) * (BN * 128) + (kk & 3) * 32,
-                                          16, 1024);
-          umma_bf16_ss(tmem + t * BN, ad, bd, idesc_qk, kk > 0 ? 1u : 0u);
+          const uint64_t off = (uint64_t)(((kk >> 2) * (BM * 128) + (kk & 3) * 32) >> 4);
+          umma_bf16_ss(tmem + t * BN, aq + off, bk + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
         umma_commit(&bars->s_full[t]);
       };
       // O_t += P_t V_j, P_t read from TMEM over the S_t columns
       auto pv = [&](int t, int j) {
-        const int s = j % kStages;
+        const uint64_t bv = dv + (uint64_t)(((j % kStages) * C::KV_BYTES) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(v_addr + s * C::KV_BYTES + kk * 16 * 128, BN * 128, 1024);
-          umma_bf16_ts(tmem + 256 + t * 128, tmem + t * BN + kk * 8, bd, idesc_pv,
-                       (j > 0 || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < BN / 16; ++kk)
+          umma_bf16_ts(tmem + 256 + t * 128, tmem + t * BN + kk * 8,
+                       bv + (uint64_t)((kk * 16 * 128) >> 4), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
       };
       bool ok = mbar_wait(&bars->q_full, 0, lim) && mbar_wait(&bars->k_full[0], 0, lim);
       tc_fence_after();
