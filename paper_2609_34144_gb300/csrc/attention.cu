@@ -387,16 +387,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = j % kStages;
         const uint32_t ph = (uint32_t)j & 1u;
         const bool more = j + 1 < n_tiles;
+        // K_{j+1} is awaited with V_j, while P_0 is still being formed, so that S_0 of tile
+        // j+1 follows PV_0 of tile j without a wait (its load was released two tiles ago)
         if (aborted(bars) || !mbar_wait(&bars->v_full[s], (uint32_t)(j / kStages) & 1u, lim) ||
+            (more && !mbar_wait(&bars->k_full[(j + 1) % kStages], (uint32_t)((j + 1) / kStages) & 1u, lim)) ||
             !mbar_wait(&bars->p_full[0], ph, lim)) { ok = false; break; }
         tc_fence_after();
         pv(0, j);
-        if (more) {
-          const int s1 = (j + 1) % kStages;
-          if (!mbar_wait(&bars->k_full[s1], (uint32_t)((j + 1) / kStages) & 1u, lim)) { ok = false; break; }
-          tc_fence_after();
-          qk(0, j + 1);
-        }
+        if (more) qk(0, j + 1);
         if (nq == 2) {
           if (aborted(bars) || !mbar_wait(&bars->p_full[1], ph, lim)) { ok = false; break; }
           tc_fence_after();
