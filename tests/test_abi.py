@@ -307,3 +307,50 @@ def test_selftest_limit_validated_on_the_host(lib):
     assert so.cast_selftest_bounded_wait(10, None) == 1            # below 1 us
     assert so.cast_selftest_bounded_wait(3_000_000_000, None) == 1  # above 2 s
     assert so.cast_last_error_detail() != b""
+
+
+def _block(lib, **kw):
+    a = lib.BlockArgs()
+    a.q, a.k_cur, a.v_cur = _fake(), _fake(0x20000), _fake(0x30000)
+    a.q_row_stride = a.cur_row_stride = 256
+    a.n_frames, a.Hg, a.Wg, a.H, a.d = 4, 4, 4, 2, 128
+    anchors = kw.pop("anchors", [0, 3])
+    a._an = (C.c_int32 * len(anchors))(*anchors)
+    a.anchors = C.cast(a._an, C.POINTER(C.c_int32))
+    a.n_anchors = len(anchors)
+    a.k_hist, a.v_hist = _fake(0x40000), _fake(0x50000)
+    a.hist_row_stride = 256
+    a.M, a.B_v, a.K, a.route_eps = 4, 8, 2, 1e-8
+    a.r_out, a.r_dtype = _fake(0x60000), lib.BF16
+    a.par = lib.default_par_params()
+    for k, v in kw.items():
+        if k.startswith("p_"):
+            setattr(a.par, k[2:], v)
+        else:
+            setattr(a, k, v)
+    return a
+
+
+@pytest.mark.parametrize("bad,status", [
+    ({"anchors": [3, 0]}, 1),                 # anchors must ascend
+    ({"anchors": [1]}, 1),                    # skipped frames need two anchors (Eq. block)
+    ({"d": 96}, 2),                           # head dim outside {64, 128}
+    ({"K": -1}, 1),
+    ({"r_dtype": 7}, 1),
+    ({"r_out": None}, 1),
+    ({"route_refine_passes": -1}, 1),
+    ({"p_T": 0.0}, 1),                        # PAR gate temperature
+    ({"w_o": _fake(0x70008)}, 1),             # misaligned output projection
+])
+def test_block_step_validation(lib, bad, status):
+    """Validation runs on the host before any launch, so these need no GPU."""
+    a = _block(lib, **bad)
+    assert lib.library().cast_block_step(C.byref(a), _fake(0x100000), 1 << 30, None) == status
+    assert lib.library().cast_last_error_detail() != b""
+
+
+def test_block_step_short_workspace_is_rejected(lib):
+    a = _block(lib)
+    need = lib.library().cast_block_workspace_size(C.byref(a))
+    assert need > 0
+    assert lib.library().cast_block_step(C.byref(a), _fake(0x100000), need - 1, None) == 1
