@@ -2,8 +2,9 @@
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
-Workload: the Matrix-Game-3.0-shaped bf16 block step (8 current latent frames of 30x52 tokens,
-12 heads x 128, 16 history blocks of 1560 tokens, K = 4, anchors every second frame).
+Workload: the HY-World-1.5-shaped bf16 block step, the largest block-step configuration (16
+current latent frames of 44x80 tokens, 24 heads x 128, 32 history blocks of 3520 tokens, K = 8,
+anchors {0, 3, 7, 12, 15}), on its seeded synthetic inputs.
 A step is cast_block_step: routing (pooled scores, TopK, then the reconstruction-coupled
 refinement with the paper's L_s = 2 passes and (lambda_anc, lambda_rec) = (1, 1)) -> routed
 anchor attention -> PAR.
@@ -15,7 +16,8 @@ anchor attention -> PAR.
   roofline  the dominant kernel (routed attention): algorithmic FLOP per launch / its average
           CUDA-event duration (stages launched through their own entry points, same kernels
           and launch configuration as inside the block step) against the measured bf16 peak
-  cpu_baseline  the CPU oracle timed on a bounded sample of the same workload
+  cpu_baseline  the CPU oracle timed on a bounded sample of the same workload (the same sample
+          and scaling model as `--impl reference`)
 Under torchrun each rank runs its own block step (independent chunks, no collective): weak
 scaling, value = frames of all ranks / max over ranks of the timed region.
 """
@@ -39,7 +41,7 @@ from synthetic import generators as G  # noqa: E402
 from synthetic import workloads as W  # noqa: E402
 
 METRIC = "block-step frames/s; routed-attn TFLOP/s & PAR GB/s as % of GB300 peak"
-WL = W.MG
+WL = W.HY
 
 
 def _peaks():
@@ -107,6 +109,16 @@ class ClockSampler:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
                 "reasons": sorted(reasons)}
+
+
+def bench_config(wl, world):
+    """The workload description both arms print."""
+    return {"workload": wl.name, "frames_per_step": wl.n_cur, "grid": list(wl.grid),
+            "heads": wl.H, "head_dim": wl.d, "history_blocks": wl.M, "block_tokens": wl.B_v,
+            "K": wl.K, "anchors": list(wl.anchors), "global_batch": world,
+            "routing": "coupled refinement, 2 passes, lambda (1, 1), tol 1e-6",
+            "l2": "flushed (256 MiB write) between timed steps, outside the events",
+            "parallelism": f"replicas x{world} (independent chunks, no collective)"}
 
 
 # ------------------------------------------------------------------------------ GPU arm
@@ -292,12 +304,7 @@ def run_gpu(args):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": wl.name, "frames_per_step": N, "grid": list(wl.grid),
-                       "heads": H, "head_dim": dh, "history_blocks": wl.M, "block_tokens": wl.B_v,
-                       "K": wl.K, "anchors": anchors, "global_batch": world,
-                       "routing": "coupled refinement, 2 passes, lambda (1, 1), tol 1e-6",
-                       "l2": "flushed (256 MiB write) between timed steps, outside the events",
-                       "parallelism": f"replicas x{world} (independent chunks, no collective)"},
+            "config": bench_config(wl, world),
             "roofline": {"bound": "tensor", "kernel": "k_attn<128> (routed anchor attention)",
                          "achieved": round(achieved, 2), "peak": bf16, "unit": "TFLOP/s",
                          "frac": round(achieved / bf16, 4), "peak_source": f"{src} bf16 burst",
@@ -323,15 +330,21 @@ def run_gpu(args):
         if not args.no_scale_points:
             line["scale_points"] = scale_points(lib, torch, dev, flush)
         if not args.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_baseline(wl)
+            line["cpu_baseline"] = cpu_baseline(wl, inp)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
 
 
 # ------------------------------------------------------------------------------ scale points
-SCALE_POINTS = ("par_sweep_f32", "par_sweep_bf16", "route_stress", "attn_hy", "select_mg", "ffn_mg",
-                "route_mg64", "attn_mg64", "attn_hy64", "block_mg64", "block_hy", "block_hy64")
+SCALE_POINTS = ("block_mg", "route_mg", "attn_mg", "par_mg",
+                "par_sweep_f32_s2", "par_sweep_f32_s3", "par_sweep_f32_s4",
+                "par_sweep_bf16_s2", "par_sweep_bf16_s3", "par_sweep_bf16_s4",
+                "route_stress_k4", "route_stress_k8", "route_stress_k16", "route_stress_k32",
+                "route_stress_k8_refine", "route_stress_k32_refine",
+                "attn_stress_k4", "attn_stress_k8", "attn_stress_k16", "attn_stress_k32",
+                "select_mg", "ffn_mg", "route_mg64", "attn_mg64", "attn_hy64", "block_mg64",
+                "block_hy64")
 
 
 def _block_tokens(wl):
@@ -353,38 +366,80 @@ def _scale_setup(name, lib, torch, dev):
 
     if name.startswith("par_sweep"):
         w = W.PAR_SWEEP
-        dt = torch.float32 if name.endswith("f32") else torch.bfloat16
+        dt = torch.float32 if "_f32_" in name else torch.bfloat16
         r = rnd(w.F, w.grid[0], w.grid[1], w.C, dtype=dt)
         wc = torch.rand(w.C, generator=g, device=dev)
-        mask = W.anchor_mask(w.F, w.anchors(2))
+        mask = W.anchor_mask(w.F, w.anchors(int(name.rsplit("_s", 1)[1])))
         p = lib.par_params(band_radius=w.band_radius)
         ws = torch.empty(lib.par_workspace_size(r, mask, p), dtype=torch.uint8, device=dev)
         return (lambda: lib.cast_par_reconstruct(r, mask, wc, p, workspace=ws),
                 r.numel() * r.element_size(), "B")
-    if name == "route_stress":
+    if name.startswith("route_stress"):
         s = W.STRESS
+        K = int(name.split("_k")[1].split("_")[0])
+        refine = lib.REFINE_PAPER if name.endswith("_refine") else None
         q = rnd(s.n_cur, s.S, s.H, s.d)
         kh, vh = rnd(s.M, s.B_v, s.H, s.d), rnd(s.M, s.B_v, s.H, s.d)
         an = list(range(s.n_cur))
-        ws = torch.empty(lib.route_workspace_size(q, an, kh, vh, 8), dtype=torch.uint8, device=dev)
-        return (lambda: lib.cast_route_topk(q, an, kh, vh, 8, workspace=ws),
+        ws = torch.empty(lib.route_workspace_size(q, an, kh, vh, K, refine=refine), dtype=torch.uint8,
+                         device=dev)
+        return (lambda: lib.cast_route_topk(q, an, kh, vh, K, workspace=ws, refine=refine),
                 (s.n_cur * s.S + 2 * s.M * s.B_v) * s.H * s.d * 2, "B")
-    if name == "attn_hy":
-        wl = W.HY
-        N, S = wl.n_cur, wl.S
-        q, kc, vc = rnd(N, S, wl.H, wl.d), rnd(N, S, wl.H, wl.d), rnd(N, S, wl.H, wl.d)
-        kh, vh = rnd(wl.M, wl.B_v, wl.H, wl.d), rnd(wl.M, wl.B_v, wl.H, wl.d)
-        Kf = len(wl.anchors)
-        perm = torch.stack([torch.randperm(wl.M, generator=torch.Generator().manual_seed(k))[:wl.K]
-                            for k in range(Kf * wl.H)]).view(Kf, wl.H, wl.K)
-        idx = perm.int().to(dev)
-        o = torch.empty((Kf, S, wl.H * wl.d), dtype=torch.bfloat16, device=dev)
-        flop = 4.0 * Kf * S * (N * S + wl.K * wl.B_v) * wl.d * wl.H
-        aws = torch.empty(max(lib.attention_workspace_size(q, kc, vc, list(wl.anchors), kh, vh, idx), 256),
+    if name.startswith("attn_stress"):
+        s = W.STRESS
+        K = int(name.split("_k")[1])
+        N, S = s.n_cur, s.S
+        q, kc, vc = rnd(N, S, s.H, s.d), rnd(N, S, s.H, s.d), rnd(N, S, s.H, s.d)
+        kh, vh = rnd(s.M, s.B_v, s.H, s.d), rnd(s.M, s.B_v, s.H, s.d)
+        an = list(range(N))
+        idx = lib.cast_route_topk(q, an, kh, vh, K)   # the kernel's own routing of these inputs
+        o = torch.empty((N, S, s.H * s.d), dtype=torch.bfloat16, device=dev)
+        flop = 4.0 * N * S * (N * S + K * s.B_v) * s.d * s.H
+        aws = torch.empty(max(lib.attention_workspace_size(q, kc, vc, an, kh, vh, idx), 256),
                           dtype=torch.uint8, device=dev)
-        return (lambda: lib.cast_anchor_attention(q, kc, vc, list(wl.anchors), kh, vh, idx, out=o,
-                                                  workspace=aws),
+        return (lambda: lib.cast_anchor_attention(q, kc, vc, an, kh, vh, idx, out=o, workspace=aws),
                 flop, "FLOP")
+    if name in ("block_mg", "route_mg", "attn_mg", "par_mg"):
+        # the Matrix-Game-shaped chunk on its seeded inputs
+        wl = W.MG
+        inp = W.block_step_inputs(wl)
+        t = {k: torch.from_numpy(G.bf16_bits(inp[k]).view(np.int16)).to(dev).view(torch.bfloat16)
+             for k in ("q", "k_cur", "v_cur", "k_hist", "v_hist")}
+        N, S, H, d = inp["q"].shape
+        an = list(wl.anchors)
+        attn_flop, route_bytes, par_bytes = algorithmic_work(wl)
+        if name == "block_mg":
+            r = torch.zeros((N, S, H * d), dtype=torch.bfloat16, device=dev)
+            a = lib.block_args(t["q"], t["k_cur"], t["v_cur"], an, t["k_hist"], t["v_hist"], wl.K,
+                               wl.grid, r, params=lib.par_params(band_radius=wl.band_radius),
+                               refine=lib.REFINE_PAPER)
+            ws = torch.empty(lib.block_workspace_size(a), dtype=torch.uint8, device=dev)
+            return (lambda: lib.cast_block_step_args(a, ws), N, "frames")
+        if name == "route_mg":
+            ws = torch.empty(lib.route_workspace_size(t["q"], an, t["k_hist"], t["v_hist"], wl.K,
+                                                      refine=lib.REFINE_PAPER),
+                             dtype=torch.uint8, device=dev)
+            return (lambda: lib.cast_route_topk(t["q"], an, t["k_hist"], t["v_hist"], wl.K, workspace=ws,
+                                                refine=lib.REFINE_PAPER), route_bytes, "B")
+        if name == "attn_mg":
+            idx = lib.cast_route_topk(t["q"], an, t["k_hist"], t["v_hist"], wl.K, refine=lib.REFINE_PAPER)
+            o = torch.empty((len(an), S, H * d), dtype=torch.bfloat16, device=dev)
+            aws = torch.empty(max(lib.attention_workspace_size(t["q"], t["k_cur"], t["v_cur"], an,
+                                                               t["k_hist"], t["v_hist"], idx), 256),
+                              dtype=torch.uint8, device=dev)
+            return (lambda: lib.cast_anchor_attention(t["q"], t["k_cur"], t["v_cur"], an, t["k_hist"],
+                                                      t["v_hist"], idx, out=o, workspace=aws),
+                    attn_flop, "FLOP")
+        # par_mg: PAR of the chunk's attention output (the block step's residual site)
+        idx = lib.cast_route_topk(t["q"], an, t["k_hist"], t["v_hist"], wl.K, refine=lib.REFINE_PAPER)
+        r = torch.zeros((N, S, H * d), dtype=torch.bfloat16, device=dev)
+        o = lib.cast_anchor_attention(t["q"], t["k_cur"], t["v_cur"], an, t["k_hist"], t["v_hist"], idx)
+        r[an] = o
+        rp = r.view(N, wl.grid[0], wl.grid[1], H * d)
+        mask = W.anchor_mask(N, an)
+        p = lib.par_params(band_radius=wl.band_radius)
+        ws = torch.empty(max(lib.par_workspace_size(rp, mask, p), 256), dtype=torch.uint8, device=dev)
+        return (lambda: lib.cast_par_reconstruct(rp, mask, None, p, workspace=ws), par_bytes, "B")
     if name == "select_mg":
         w = W.SELECT_MG
         S = w.grid[0] * w.grid[1]
@@ -409,16 +464,6 @@ def _scale_setup(name, lib, torch, dev):
                          device=dev)
         return (lambda: lib.cast_ffn_step(x, an, w1, b1, w2, b2, wl.grid, r, workspace=ws),
                 4.0 * len(an) * S * D * Dff, "FLOP")
-    if name == "block_hy":
-        wl = W.HY
-        N, S, H, d = wl.n_cur, wl.S, wl.H, wl.d
-        q, kc, vc = rnd(N, S, H, d), rnd(N, S, H, d), rnd(N, S, H, d)
-        kh, vh = rnd(wl.M, wl.B_v, H, d), rnd(wl.M, wl.B_v, H, d)
-        r = torch.zeros((N, S, H * d), dtype=torch.bfloat16, device=dev)
-        a = lib.block_args(q, kc, vc, list(wl.anchors), kh, vh, wl.K, wl.grid, r,
-                           params=lib.par_params(band_radius=wl.band_radius), refine=lib.REFINE_PAPER)
-        ws = torch.empty(lib.block_workspace_size(a), dtype=torch.uint8, device=dev)
-        return (lambda: lib.cast_block_step_args(a, ws), N, "frames")
     if name in ("route_mg64", "attn_mg64", "attn_hy64", "block_mg64", "block_hy64"):
         wl = W.HY64 if name in ("attn_hy64", "block_hy64") else W.MG64
         N, S, H, d = wl.n_cur, wl.S, wl.H, wl.d
@@ -500,11 +545,11 @@ def run_profile(name):
 
 
 def _captured_traffic():
-    """DRAM bytes per attention launch from the committed ncu summary, or None when the
-    kernel sources changed since that capture (hash of attention.cu + ptx.cuh)."""
+    """DRAM bytes per attention launch at the bench workload from the committed ncu summary, or
+    None when the kernel sources changed since that capture (hash of attention.cu + ptx.cuh)."""
     import hashlib
     import re
-    prof = os.path.join(ROOT, "profiles", "k_attn_mg_block_step.md")
+    prof = os.path.join(ROOT, "profiles", "k_attn_hy_block_step.md")
     if not os.path.exists(prof):
         return None
     m = re.search(r"dram_bytes_per_launch=(\d+) source_sha256_16=([0-9a-f]+)", open(prof).read())
@@ -528,35 +573,46 @@ def launches_per_step(wl):
     return 3 + 1 + 3 * (int(full) + int(edge))
 
 
-def _oracle_sample(wl, inp, R, heads, row_stride, tiles):
-    """One bounded sample of the block step in the CPU oracle: routing and attention on the
-    first `heads` heads (attention on every `row_stride`-th query row), PAR on the first
-    `tiles` tiles (pooled over every channel).  Returns (seconds for the whole workload
-    scaled from the sample, description of the sample)."""
+# One bounded sample of the block step, the same for the `cpu_baseline` leg and for `--impl
+# reference`: routing (pooled scores, omission, TopK and the 2-pass refinement) on the first
+# `route_heads` heads with every token and block; routed attention on the first `attn_heads`
+# heads for `attn_rows` evenly spaced query rows of every anchor; PAR on `par_tiles` tiles
+# spread over the grid (pooled over every channel).
+SAMPLE_PLAN = {"route_heads": 4, "attn_heads": 1, "attn_rows": 128, "par_tiles": 3}
+
+
+def _oracle_sample(wl, inp, R, plan=SAMPLE_PLAN):
+    """Runs the sample in the CPU oracle.  Returns (estimated seconds of the whole block step,
+    measured seconds of the sample, description).  Scaling model: each stage's sample time
+    times the stage's share of the full work (routing heads H / route_heads; attention
+    (H / attn_heads) * (S / attn_rows); PAR n_tiles / par_tiles)."""
     import oracle.cast_oracle as O
     anchors = list(wl.anchors)
-    hs = slice(0, heads)
+    hr, ha = slice(0, plan["route_heads"]), slice(0, plan["attn_heads"])
     t0 = time.perf_counter()
-    rt = O.pooled_routing(inp["q"][:, :, hs], anchors, inp["k_hist"][:, :, hs],
-                          inp["v_hist"][:, :, hs])
+    rt = O.pooled_routing(inp["q"][:, :, hr], anchors, inp["k_hist"][:, :, hr],
+                          inp["v_hist"][:, :, hr])
     idx = np.stack([O.coupled_routing(rt.u[:, h], anchors, wl.n_cur, wl.K)
                     for h in range(rt.u.shape[1])], axis=1)
     t1 = time.perf_counter()
-    rows = np.arange(0, wl.S, row_stride)
-    O.routed_attention(inp["q"][:, :, hs], inp["k_cur"][:, :, hs], inp["v_cur"][:, :, hs],
-                       inp["k_hist"][:, :, hs], inp["v_hist"][:, :, hs], anchors, idx, rows=rows)
+    rows = np.linspace(0, wl.S - 1, plan["attn_rows"]).astype(np.int64)
+    O.routed_attention(inp["q"][:, :, ha], inp["k_cur"][:, :, ha], inp["v_cur"][:, :, ha],
+                       inp["k_hist"][:, :, ha], inp["v_hist"][:, :, ha], anchors,
+                       idx[:, :plan["attn_heads"]], rows=rows)
     t2 = time.perf_counter()
     n_tiles = len(O.tiles_of(wl.grid[0], wl.grid[1], 8, 8))
+    tiles = sorted({int(v) for v in np.linspace(0, n_tiles - 1, plan["par_tiles"])})
     O.par_reconstruct(R, W.anchor_mask(wl.n_cur, anchors), None,
-                      O.ParParams(band_radius=wl.band_radius), tiles=range(tiles))
+                      O.ParParams(band_radius=wl.band_radius), tiles=tiles)
     t3 = time.perf_counter()
-    hf = wl.H / heads
-    est = (t1 - t0) * hf + (t2 - t1) * hf * (wl.S / len(rows)) + (t3 - t2) * (n_tiles / tiles)
-    desc = (f"routing with 2-pass refinement on {heads}/{wl.H} heads (all tokens, all blocks), "
-            f"attention on those heads "
-            f"for {len(rows)}/{wl.S} query rows of every anchor, PAR on {tiles}/{n_tiles} tiles; "
-            f"each stage scaled to the full workload by its share of the work")
-    return est, desc
+    est = ((t1 - t0) * wl.H / plan["route_heads"]
+           + (t2 - t1) * (wl.H / plan["attn_heads"]) * (wl.S / len(rows))
+           + (t3 - t2) * (n_tiles / len(tiles)))
+    desc = (f"routing with 2-pass refinement on {plan['route_heads']}/{wl.H} heads (all tokens, all "
+            f"blocks); attention on {plan['attn_heads']}/{wl.H} heads for {len(rows)}/{wl.S} query "
+            f"rows of every anchor; PAR on {len(tiles)}/{n_tiles} tiles (all channels); whole-step "
+            f"time = sum of each stage's sample time x its share of the full work")
+    return est, t3 - t0, desc
 
 
 def _par_input(wl):
@@ -564,17 +620,18 @@ def _par_input(wl):
         (wl.n_cur, wl.grid[0], wl.grid[1], wl.H * wl.d)).astype(np.float32)
 
 
-def cpu_baseline(wl):
-    inp = W.block_step_inputs(wl)
+def cpu_baseline(wl, inp):
     R = _par_input(wl)
     cores = len(os.sched_getaffinity(0))
-    n_tiles = (wl.grid[0] + 7) // 8 * ((wl.grid[1] + 7) // 8)
-    est, desc = _oracle_sample(wl, inp, R, heads=wl.H, row_stride=16, tiles=n_tiles)
+    est, took, desc = _oracle_sample(wl, inp, R)
     return {"value": round(wl.n_cur / est, 6), "unit": "frames/s", "cores": cores, "kind": "oracle",
-            "sample": desc, "est_seconds_per_step": round(est, 3)}
+            "sample": desc, "est_seconds_per_step": round(est, 3), "sample_seconds": round(took, 3)}
 
 
 def run_reference(args):
+    """The reference arm: the CPU oracle as it stands, one bounded sample per step (the
+    sample and scaling model of `cpu_baseline`).  value = frames of the whole workload per
+    second of estimated full-step time; ms_per_step is the measured time of one sample."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
@@ -583,17 +640,20 @@ def run_reference(args):
     R = _par_input(wl)
     cores = len(os.sched_getaffinity(0))
     for _ in range(args.warmup):
-        _oracle_sample(wl, inp, R, heads=1, row_stride=wl.S // 8, tiles=1)
-    total, desc = 0.0, ""
+        _oracle_sample(wl, inp, R)
+    est_total, took_total, desc = 0.0, 0.0, ""
     for _ in range(args.steps):
-        est, desc = _oracle_sample(wl, inp, R, heads=1, row_stride=wl.S // 8, tiles=1)
-        total += est
-    value = wl.n_cur * args.steps / total
+        est, took, desc = _oracle_sample(wl, inp, R)
+        est_total += est
+        took_total += took
+    value = wl.n_cur * args.steps / est_total
+    world = int(os.environ.get("WORLD_SIZE", "1"))
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "frames/s",
-            "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 2),
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(took_total / args.steps * 1e3, 2),
+            "est_full_step_ms": round(est_total / args.steps * 1e3, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": wl.name},
+            "data": "synthetic", "config": bench_config(wl, 1),
             "cpu_baseline": {"value": round(value, 6), "unit": "frames/s", "cores": cores,
                              "kind": "oracle", "sample": desc},
             "e2e": {"value": round(value, 6), "unit": "frames/s", "h2d_bytes_per_step": 0,

@@ -166,7 +166,9 @@ size_t cast_route_workspace_size(const cast_route_args* args);
  *   - Problems needing more than 16 MiB of scratch (cast_route_workspace_size() > 16 MiB)
  *     are rejected with CAST_ERR_UNSUPPORTED and a message; nothing is launched.
  *   - The first call on a device looks up the array's device address with that device
- *     current (no allocation); make that first call before any stream capture.
+ *     current (no allocation); make that first call before any stream capture.  The address
+ *     is kept for the life of the process: do not call this entry point on a device after a
+ *     cudaDeviceReset() (or any other teardown of its primary context) in the same process.
  *   - All calls share the one array and the kernels fully overwrite what they read, so no
  *     clearing is needed between calls; calls whose work overlaps on the GPU (concurrent
  *     streams, or several host threads) race on it and must be serialised by the caller.

@@ -7,12 +7,11 @@
 // bf16 A and W (K contiguous), f32 accumulation in TMEM, bias (+ GELU, tanh form) in the
 // epilogue, C in bf16 or f32.  Tiles of 128 rows x 256 columns; a tile never spans anchors
 // (rows past S read as zero through the 3-D tensor map [frame][row][k] and are not written).
-// The two CTAs of a cluster take the two row tiles of one 256-row pair with the same W tile:
-// each loads its own A k-slice and half of the W k-slice, multicast into both CTAs, so a W
-// byte leaves L2 once per pair; each CTA's UMMA issuer releases a stage in both CTAs.
+// Persistent CTAs, one per SM, each loading its own A and W k-slices (no clusters): CTAs that
+// run at the same time take neighbouring column tiles of one row tile, so the A tile and the
+// W matrix (a few MB) are served from L2.
 // Warp roles (384 threads, one CTA per SM, 193 KB shared memory, 512 TMEM columns):
-//   warp 0      TMA producer: A (128 x 64) and half of W (128 x 64, multicast to the pair)
-//               k-slices into a 4-stage ring
+//   warp 0      TMA producer: A (128 x 64) and W (256 x 64) k-slices into a 4-stage ring
 //   warp 1      TMEM owner and single-thread UMMA issuer (kind::f16, M = 128, N = 256, K = 16),
 //               accumulating each tile in one of two 256-column TMEM buffers
 //   warps 4..11 epilogue: one output row per thread and half of the tile's columns per warp
@@ -40,7 +39,7 @@ constexpr int kGSmem = kGStages * kStageBytes + 256 + 1024;   // ring + barriers
 
 struct GemmKArgs {
   int S, N, K, n_anchors, m_tiles, n_tiles, n_k;
-  int m_pairs, total_pairs;   // 256-row pairs of row tiles per anchor; pair tiles in all
+  int total_tiles;   // n_anchors * m_tiles * n_tiles
   const void* bias;
   void* c;
   int64_t ldc;
@@ -78,42 +77,14 @@ __device__ __forceinline__ float gelu_tanh(float x) {
   return 0.5f * x * (1.f + t);
 }
 
-// Pair tile p -> (anchor i, row tile mt of this cluster rank, column tile nt); a rank-1 row
-// tile past the anchor's rows reads zeros and writes nothing.
-__device__ __forceinline__ void tile_of(const GemmKArgs& a, int p, int rank, int& i, int& mt, int& nt) {
-  const int per_anchor = a.m_pairs * a.n_tiles;
-  i = p / per_anchor;
-  const int rem = p - i * per_anchor;
-  const int mp = rem / a.n_tiles;
-  nt = rem - mp * a.n_tiles;
-  mt = 2 * mp + rank;
-}
-
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ void cluster_barrier() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
-                   : "memory");
-}
-// 2-D tile load delivered to the same shared-memory offset (and mbarrier) of every CTA in mask
-__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* m, uint64_t* bar,
-                                               int32_t x, int32_t y, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
-      : "memory");
-}
-// Arrive on `bar` in every CTA of mask once this thread's issued UMMAs have completed
-__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-          smem_u32(bar)),
-      "h"(mask)
-      : "memory");
+// Tile t -> (anchor i, row tile mt, column tile nt), column tiles innermost; a row tile past
+// the anchor's rows reads zeros and writes nothing.
+__device__ __forceinline__ void tile_of(const GemmKArgs& a, int t, int& i, int& mt, int& nt) {
+  const int per_anchor = a.m_tiles * a.n_tiles;
+  i = t / per_anchor;
+  const int rem = t - i * per_anchor;
+  mt = rem / a.n_tiles;
+  nt = rem - mt * a.n_tiles;
 }
 
 __global__ void __launch_bounds__(kGThreads, 1)
@@ -125,11 +96,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
   GBars* bars = reinterpret_cast<GBars*>(smem + kGStages * kStageBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint64_t lim = a.wait_ns;
-  const int rank = (int)cluster_rank(), pair = blockIdx.x >> 1, n_pairs_grid = gridDim.x >> 1;
+  const int first = blockIdx.x, stride = gridDim.x;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kGStages; ++s) {
       mbar_init(&bars->full[s], 1);
-      mbar_init(&bars->empty[s], 2);   // released by the UMMA issuers of both CTAs
+      mbar_init(&bars->empty[s], 1);   // released by the UMMA issuer
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars->acc_full[b], 1);
@@ -144,8 +115,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
     tmem_relinquish();
     tc_fence_before();
   }
-  // both CTAs' barriers exist before either multicasts into the other
-  cluster_barrier();
+  __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
 
@@ -156,22 +126,21 @@ __global__ void __launch_bounds__(kGThreads, 1)
       tma_prefetch_desc(&tm_w);
       int it = 0;
       bool ok = true;
-      for (int p = pair; ok && p < a.total_pairs; p += n_pairs_grid) {
+      for (int t = first; ok && t < a.total_tiles; t += stride) {
         int i, mt, nt;
-        tile_of(a, p, rank, i, mt, nt);
+        tile_of(a, t, i, mt, nt);
         for (int ks = 0; ks < a.n_k; ++ks, ++it) {
           const int s = it % kGStages;
-          // both CTAs have consumed this stage (the peer's W half lands in it too)
+          // the UMMAs that read this stage have completed
           if (g_aborted(bars) || !mbar_wait(&bars->empty[s], ((uint32_t)(it / kGStages) & 1u) ^ 1u, lim)) {
             g_set_abort(bars);
             ok = false;
             break;
           }
           uint8_t* st = smem + s * kStageBytes;
-          mbar_arrive_expect_tx(&bars->full[s], kStageBytes);   // own A + both W halves
+          mbar_arrive_expect_tx(&bars->full[s], kStageBytes);   // A + W k-slices
           tma_load_3d(st, &tm_a, &bars->full[s], ks * GBK, mt * GBM, a.a_frame[i]);
-          tma_load_2d_mc(st + kABytes + rank * (GBN / 2) * 128, &tm_w, &bars->full[s], ks * GBK,
-                         nt * GBN + rank * (GBN / 2), (uint16_t)0x3);
+          tma_load_2d(st + kABytes, &tm_w, &bars->full[s], ks * GBK, nt * GBN);
         }
       }
     }
@@ -182,7 +151,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
       const uint32_t base = smem_u32(smem);
       int it = 0, lt = 0;
       bool ok = true;
-      for (int p = pair; ok && p < a.total_pairs; p += n_pairs_grid, ++lt) {
+      for (int t = first; ok && t < a.total_tiles; t += stride, ++lt) {
         const int buf = lt & 1;
         if (g_aborted(bars) || !mbar_wait(&bars->acc_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, lim)) {
           ok = false;
@@ -201,7 +170,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
           for (int kk = 0; kk < GBK / 16; ++kk)
             umma_bf16_ss(tmem + buf * GBN, sdesc_sw128(sa + kk * 32, 16, 1024),
                          sdesc_sw128(sb + kk * 32, 16, 1024), idesc, (ks > 0 || kk > 0) ? 1u : 0u);
-          umma_commit_mc(&bars->empty[s], (uint16_t)0x3);   // free in both CTAs once read
+          umma_commit(&bars->empty[s]);   // the stage is free once these UMMAs have read it
         }
         if (!ok) break;
         umma_commit(&bars->acc_full[buf]);
@@ -216,7 +185,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
     const int q4 = warp & 3, half = (warp - 4) >> 2;
     const int row = q4 * 32 + lane;
     int lt = 0;
-    for (int p = pair; p < a.total_pairs; p += n_pairs_grid, ++lt) {
+    for (int t = first; t < a.total_tiles; t += stride, ++lt) {
       const int buf = lt & 1;
       const bool w = !g_aborted(bars) && mbar_wait(&bars->acc_full[buf], (uint32_t)(lt >> 1) & 1u, lim);
       if (!__all_sync(0xffffffffu, w)) {
@@ -225,7 +194,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
       }
       tc_fence_after();
       int i, mt, nt;
-      tile_of(a, p, rank, i, mt, nt);
+      tile_of(a, t, i, mt, nt);
       const int r = mt * GBM + row;
       const bool live = r < a.S;
       const uint32_t tl = tmem + buf * GBN + ((uint32_t)(q4 * 32) << 16);
@@ -320,7 +289,6 @@ __global__ void __launch_bounds__(kGThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
-  cluster_barrier();   // no CTA leaves while its peer may still arrive on its barriers
 }
 
 // bf16 [depth][rows][inner] (rank 2 when depth == 0), box 64 x box_rows (x 1), 128-B swizzle
@@ -345,7 +313,7 @@ cast_status gemm_anchor_rows(const AnchorGemm& g, cudaStream_t st) {
   CUtensorMap ma, mw;
   if (!make_gemm_map(&ma, g.a, (uint64_t)g.K, (uint64_t)g.S, (uint64_t)g.lda * 2, (uint64_t)g.a_frames,
                      (uint64_t)g.a_frame_stride * 2, GBM) ||
-      !make_gemm_map(&mw, g.w, (uint64_t)g.K, (uint64_t)g.N, (uint64_t)g.ldw * 2, 0, 0, GBN / 2))
+      !make_gemm_map(&mw, g.w, (uint64_t)g.K, (uint64_t)g.N, (uint64_t)g.ldw * 2, 0, 0, GBN))
     return fail(CAST_ERR_CUDA, "dense: cuTensorMapEncodeTiled failed");
   GemmKArgs k{};
   k.S = g.S;
@@ -355,8 +323,7 @@ cast_status gemm_anchor_rows(const AnchorGemm& g, cudaStream_t st) {
   k.m_tiles = (g.S + GBM - 1) / GBM;
   k.n_tiles = (g.N + GBN - 1) / GBN;
   k.n_k = (g.K + GBK - 1) / GBK;
-  k.m_pairs = (k.m_tiles + 1) / 2;
-  k.total_pairs = g.n_anchors * k.m_pairs * k.n_tiles;
+  k.total_tiles = g.n_anchors * k.m_tiles * k.n_tiles;
   k.bias = g.bias;
   k.c = g.c;
   k.ldc = g.ldc;
@@ -376,19 +343,13 @@ cast_status gemm_anchor_rows(const AnchorGemm& g, cudaStream_t st) {
     return check_launch("dense GEMM smem attribute");
   int dev = 0, nsm = 148;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-  const int clusters = k.total_pairs < nsm / 2 ? k.total_pairs : nsm / 2;
+  const int grid = k.total_tiles < nsm ? k.total_tiles : nsm;
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(2 * (clusters > 0 ? clusters : 1), 1, 1);
+  cfg.gridDim = dim3(grid > 0 ? grid : 1, 1, 1);
   cfg.blockDim = dim3(kGThreads, 1, 1);
   cfg.dynamicSmemBytes = kGSmem;
   cfg.stream = st;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = 2;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 0;
   if (cudaLaunchKernelEx(&cfg, k_gemm, ma, mw, k) != cudaSuccess) return check_launch("dense GEMM kernel");
   return check_launch("dense GEMM kernel");
 }

@@ -23,7 +23,9 @@ static __device__ __align__(256) unsigned char g_route_scratch[kNoAllocScratchBy
 std::mutex g_setup_mu;
 void* g_scratch_ptr[kMaxDevices] = {};
 
-// Device address of g_route_scratch on the current device, looked up once per device.
+// Device address of g_route_scratch on the current device, looked up once per device and kept
+// for the life of the process (a context torn down by cudaDeviceReset would invalidate it; the
+// header tells callers not to use this entry point after a reset).
 cast_status scratch_for_current_device(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);

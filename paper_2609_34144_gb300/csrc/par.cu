@@ -237,28 +237,6 @@ __device__ __forceinline__ float sqrt_approx(float x) {
   return y;
 }
 
-// atan2(y, x) in (-pi, pi]: octant reduction to a = min(|x|,|y|) / max(|x|,|y|) in [0, 1] and an
-// odd degree-15 polynomial for atan(a) whose coefficients were fitted (weighted least squares
-// at Chebyshev nodes) for this kernel; |error| < 2e-7 rad in f32.
-__device__ __forceinline__ float atan2_fast(float y, float x) {
-  const float ax = fabsf(x), ay = fabsf(y);
-  const float mx = fmaxf(ax, ay), mn = fminf(ax, ay);
-  const float a = mx > 0.f ? mn * rcp_approx(mx) : 0.f;
-  const float a2 = a * a;
-  float p = -4.054564983e-03f;
-  p = fmaf(p, a2, 2.186295576e-02f);
-  p = fmaf(p, a2, -5.591233447e-02f);
-  p = fmaf(p, a2, 9.642198682e-02f);
-  p = fmaf(p, a2, -1.390863061e-01f);
-  p = fmaf(p, a2, 1.994656622e-01f);
-  p = fmaf(p, a2, -3.332985938e-01f);
-  p = fmaf(p, a2, 9.999993443e-01f);
-  float r = p * a;
-  if (ay > ax) r = 1.57079632679489662f - r;
-  if (x < 0.f) r = 3.14159265358979324f - r;
-  return signbit(y) ? -r : r;
-}
-
 // sin and cos of x = 2 pi k + r with |r| <= pi (Cody-Waite split of 2 pi into two parts),
 // then the hardware approximations on the reduced argument.
 __device__ __forceinline__ void sincos_reduced(float x, float* s, float* c) {
@@ -320,7 +298,7 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const BinIn
     Zi[s] = v ? zw[3 * b + 1] * inv_hw : 0.f;
     Wv[s] = v ? zw[3 * b + 2] * inv_hw : 0.f;
     Za[s] = sqrt_approx(Zr[s] * Zr[s] + Zi[s] * Zi[s]);
-    t[s] = atan2_fast(Zi[s], Zr[s]);
+    t[s] = atan2f(Zi[s], Zr[s]);
     if (t[s] <= -3.14159265358979f) t[s] = 3.14159265358979f;   // principal branch (-pi, pi]
     if (v) wmax = fmaxf(wmax, Wv[s]);
   }

@@ -12,7 +12,7 @@ from tests.test_gpu_route import check_idx
 pytestmark = pytest.mark.gpu
 
 
-def _run_block(lib, wl, inp, with_x=False):
+def _run_block(lib, wl, inp, with_x=False, refine=None):
     dk = (lambda x: to_dev(x, "bf16"))
     N, S, H, d = inp["q"].shape
     rdt = torch.float32 if wl.dtype == "f32" else torch.bfloat16
@@ -26,7 +26,7 @@ def _run_block(lib, wl, inp, with_x=False):
     params = lib.par_params(band_radius=wl.band_radius)
     lib.cast_block_step(dk(inp["q"]), dk(inp["k_cur"]), dk(inp["v_cur"]), list(wl.anchors),
                         dk(inp["k_hist"]), dk(inp["v_hist"]), wl.K, wl.grid, r_out, x=x,
-                        idx_out=idx, params=params)
+                        idx_out=idx, params=params, refine=refine)
     torch.cuda.synchronize()
     lib.cast_check_device()
     out = {"r": to_host(r_out), "idx": idx.cpu().numpy()}
@@ -35,13 +35,14 @@ def _run_block(lib, wl, inp, with_x=False):
     return out
 
 
-def _check(wl, inp, out, rows=None, tiles=None):
+def _check(wl, inp, out, rows=None, tiles=None, routing=True):
     anchors = list(wl.anchors)
     Kf = len(anchors)
     N, S, H, d = inp["q"].shape
     # routing
-    rt = O.pooled_routing(inp["q"], anchors, inp["k_hist"], inp["v_hist"])
-    check_idx(out["idx"], rt.u, min(wl.K, wl.M))
+    if routing:
+        rt = O.pooled_routing(inp["q"], anchors, inp["k_hist"], inp["v_hist"])
+        check_idx(out["idx"], rt.u, min(wl.K, wl.M))
     # attention, fed the GPU's routed blocks
     ref = O.routed_attention(inp["q"], inp["k_cur"], inp["v_cur"], inp["k_hist"], inp["v_hist"],
                              anchors, out["idx"], rows=rows)
@@ -111,3 +112,30 @@ def test_block_step_degenerate(lib, wl):
         assert np.array_equal(out["idx"], np.tile(np.arange(wl.M, dtype=np.int32),
                                                   (len(wl.anchors), wl.H, 1)))
     _check(wl, inp, out)
+
+
+def test_block_step_refined_mg_full_size(lib):
+    """The bench configuration: the Matrix-Game-shaped block step with the paper's two
+    refinement passes (Alg. routing).  The omission scores are compared with the oracle's,
+    the refined block sets with Alg. routing run by the oracle on those scores, and the
+    attention rows and PAR outputs with the oracle fed the GPU's routed blocks / anchor rows
+    (sampled rows on both sides of query-tile boundaries; every tile shape of the grid)."""
+    from tests.test_gpu_par_configs import edge_kind_sample
+    from tests.test_gpu_refine import PAPER, check_refined
+    wl = W.MG
+    inp = W.block_step_inputs(wl)
+    out = _run_block(lib, wl, inp, refine=PAPER)
+    anchors = list(wl.anchors)
+    dk = (lambda x: to_dev(x, "bf16"))
+    _, u = lib.cast_route_topk(dk(inp["q"]), anchors, dk(inp["k_hist"]), dk(inp["v_hist"]), wl.K,
+                               want_u=True, refine=PAPER)
+    torch.cuda.synchronize()
+    ug = to_host(u)
+    rt = O.pooled_routing(inp["q"], anchors, inp["k_hist"], inp["v_hist"])
+    np.testing.assert_allclose(ug, rt.u, rtol=1e-3, atol=1e-6 * rt.u.max())
+    changed, amb = check_refined(out["idx"], ug, anchors, wl.n_cur, wl.K, PAPER)
+    assert amb < wl.H
+    rng = np.random.default_rng(wl.seed + 1)
+    rows = np.unique(np.concatenate([[0, 127, 128, 1535, 1536, wl.S - 1], rng.integers(0, wl.S, 4)]))
+    tiles = edge_kind_sample(wl.grid[0], wl.grid[1], extra=(int(rng.integers(0, 28)),))
+    _check(wl, inp, out, rows=rows, tiles=tiles, routing=False)

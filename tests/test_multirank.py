@@ -51,7 +51,7 @@ def test_single_rank_is_identity():
 
 
 def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
-    monkeypatch.setattr(bench, "_oracle_sample", lambda *a, **k: (2.0, "stub sample"))
+    monkeypatch.setattr(bench, "_oracle_sample", lambda *a, **k: (2.0, 0.5, "stub sample"))
     monkeypatch.setattr(bench, "_par_input", lambda wl: None)
     monkeypatch.setattr(bench.W, "block_step_inputs", lambda wl: {})
     args = type("A", (), {"steps": 2, "warmup": 3})()

@@ -29,9 +29,9 @@ def _inputs(seed, N=3, S=300, H=4, d=128, M=12, Bv=200):
     return to_dev(q, "bf16"), to_dev(k, "bf16"), to_dev(v, "bf16")
 
 
-def _call_noalloc(lib, q, anchors, k, v, K):
+def _call_noalloc(lib, q, anchors, k, v, K, refine=None):
     """Direct C-ABI call of cast_route_topk_noalloc (no workspace argument)."""
-    a = lib._route_args(q, anchors, k, v, K)
+    a = lib._route_args(q, anchors, k, v, K, refine=refine)
     Kf, H, M = len(anchors), q.shape[2], k.shape[0]
     idx = torch.full((Kf, H, min(K, M)), -1, dtype=torch.int32, device="cuda")
     u = torch.full((Kf, H, M), float("nan"), dtype=torch.float32, device="cuda")
@@ -49,6 +49,25 @@ def test_noalloc_matches_workspace_entry_point_twice(lib):
         ref_idx, ref_u = lib.cast_route_topk(q, anchors, k, v, K, want_u=True)
         idx, u = _call_noalloc(lib, q, anchors, k, v, K)
         torch.cuda.synchronize()
+        np.testing.assert_allclose(to_host(u), to_host(ref_u), rtol=2e-4, atol=1e-7)
+        assert np.array_equal(idx.cpu().numpy(), ref_idx.cpu().numpy()), f"call {call}"
+
+
+def test_noalloc_wide_path_with_refinement(lib):
+    """Many history blocks (the per-head statistics spread over a cluster of CTAs, radix-select
+    TopK) with the paper's two refinement passes: the shared scratch is left holding another
+    problem's means by the call before, and each result must still equal the workspace entry
+    point's."""
+    anchors, K, M = [0, 2, 4, 6], 90, 448
+    for call, seed in enumerate((41, 42)):
+        q, k, v = _inputs(seed, N=8, S=40, H=2, d=128, M=M, Bv=16)
+        # a different problem through the fixed scratch first
+        q0, k0, v0 = _inputs(seed + 100)
+        _call_noalloc(lib, q0, [0, 1], k0, v0, 5, refine=lib.REFINE_PAPER)
+        ref_idx, ref_u = lib.cast_route_topk(q, anchors, k, v, K, want_u=True, refine=lib.REFINE_PAPER)
+        idx, u = _call_noalloc(lib, q, anchors, k, v, K, refine=lib.REFINE_PAPER)
+        torch.cuda.synchronize()
+        lib.cast_check_device()
         np.testing.assert_allclose(to_host(u), to_host(ref_u), rtol=2e-4, atol=1e-7)
         assert np.array_equal(idx.cpu().numpy(), ref_idx.cpu().numpy()), f"call {call}"
 
