@@ -254,8 +254,9 @@ typedef struct {
  * R_t = IRFFT2_ortho((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
  * All frames anchors: nothing to do (workspace size 0).  The workspace
  * (cast_par_workspace_size() bytes) holds each channel chunk's partial Z, W per (tile, pair)
- * and theta, g per bin: 120 ceil(C/128) + 80 floats per tile and anchor (each part rounded
- * up to 256 bytes).
+ * and theta, g per bin: 120 ceil(C/128) + 80 floats per tile and anchor, and for bf16
+ * residuals each target's blend matrix (32 KB per tile and skipped frame) for the tensor-core
+ * blend (each part rounded up to 256 bytes).
  * Errors: INVALID_ARG when a frame is skipped and fewer than two anchors exist, bad shapes
  * or pointers, a short workspace; UNSUPPORTED for tile sides outside 1..8, C not a multiple
  * of 8, C > 4096. */

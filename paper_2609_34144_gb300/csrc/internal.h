@@ -112,7 +112,8 @@ struct ParPlan {
   int chunk;        // channels per CTA (= threads per CTA)
   int n_chunk;      // channel chunks per tile
   int n_tseg_full, n_tseg_edge;   // time segments (runs of anchor pairs) per tile, per kind
-  size_t rec_bytes, trans_bytes, total_bytes;   // workspace: chunk records, theta and g
+  size_t rec_bytes, trans_bytes, img_bytes, total_bytes;   // workspace: chunk records, theta and g,
+                                                          // blend matrices (bf16)
 };
 ParPlan par_plan(const cast_par_args& a);
 cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st);

@@ -13,6 +13,13 @@
 //   K_blend (tile, channel chunk): streams the anchors again (an L2 hit at these sizes), forms
 //       their spectra and writes every target straight from registers:
 //       R_t = IRFFT2((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
+//       This is the f32 blend.  For bf16 residuals the blend runs on the tensor cores instead
+//       (K_blend_tc below): on one tile, Eq. (fcpasm) is exactly two circular convolutions,
+//         R_t = h_a (*) R_a + h_b (*) R_b,  h = IDFT2 of the Hermitian-extended phasors
+//         phi_a = (1-alpha) e^{i g alpha theta}, phi_b = alpha e^{-i g (1-alpha) theta},
+//       so K_transport also writes each target's 64 x 128 matrix [H_a | H_b] (two bf16 pieces,
+//       laid out as a swizzled UMMA operand) and one UMMA chain per pair of targets computes
+//       [H_t1 ; H_t2] [X_a ; X_b] for 128 channels (M = 128 output rows, K = 128 tokens).
 // The CTAs of a pass never wait on each other, so the passes fill the GPU whatever the number
 // of anchor pairs; the passes are chained as programmatic dependents.  Global traffic beyond
 // the algorithmic bytes: a second read of the anchors and the records (120 floats per tile,
@@ -147,6 +154,8 @@ struct ParKArgs {
   const float* wch;
   float* rec;     // workspace [tile][pair j][chunk][kRec]: each chunk's Z / W record
   float* trans;   // workspace [tile][pair j][2][kNB]: theta and g per bin
+  char* img;      // workspace [tile][target][kImgBytes]: blend matrices (bf16 runs), or null
+  int n_target;
   int F, Hg, Wg, C, n_chunk;             // n_chunk: channel chunks of kCC channels
   int tile_base;                         // global index of tile 0 of this launch's kind
   int th, tw, tiles_x, tiles_y, n_tile, n_tseg;
@@ -352,6 +361,100 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const BinIn
     if (bi.cut[b]) gv = 0.f;   // outside the band
     th[b] = any ? thv[s] : 0.f;
     gate[b] = gv;
+  }
+}
+
+// ------------------------------------------------------------------ blend matrices
+constexpr int kImgTerm = 64 * 128 * 2;   // one bf16 piece of one target's [64][128] matrix, 16 KB
+constexpr int kImgBytes = 2 * kImgTerm;  // both pieces (hi, lo): 32 KB per (tile, target)
+
+// The blend matrices of every target t of one (tile, pair), written as UMMA operand images
+// (K-major, 128-byte swizzle, K-blocks of 64 tokens 8 KB apart, two bf16 pieces kImgTerm apart):
+// row m = output token 8 yo + xo, column 64 side + 8 yi + xi = input token of anchor a (side 0)
+// or b (side 1); entry h_side((yo - yi) mod h, (xo - xi) mod w) with
+// h_side(d) = (1 / (h w)) sum over stored bins of kappa' Re(phi_side e^{2 pi i (ky dy / h + kx dx / w)}),
+// kappa' = 1 on the kx = 0 and Nyquist columns (every ky stored), 2 elsewhere;
+// phi_a = (1 - alpha) e^{i g alpha theta}, phi_b = alpha e^{-i g (1 - alpha) theta}.  128 threads.
+__device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const BinInfo& bi,
+                                   const float* th, const float* gate, int tg, int j, int tid) {
+  __shared__ float2 s_cs[64];
+  __shared__ unsigned char s_ym[8][8], s_xm[5][8];
+  __shared__ float4 s_phi[kNB];
+  __shared__ float s_h[2][64];
+  const int h = g.h, w = g.w, n = h * w;
+  if (tid < 64) {
+    if (tid < n) {
+      float sv, cv;
+      sincospif(2.f * (float)tid / (float)n, &sv, &cv);
+      s_cs[tid] = make_float2(cv, sv);
+    }
+    s_ym[tid >> 3][tid & 7] = (unsigned char)(((tid >> 3) * (tid & 7)) % h);
+  } else if (tid < 64 + 40) {
+    const int e = tid - 64;
+    s_xm[e >> 3][e & 7] = (unsigned char)(((e >> 3) * (e & 7)) % w);
+  }
+  const float inv_n = 1.f / (float)n;
+  const int side = tid >> 6, d = tid & 63, dy0 = d >> 3, dx0 = d & 7;
+  for (int t = a.pair_tbeg[j]; t < a.pair_tbeg[j + 1]; ++t) {
+    const float al = a.target_alpha[t];
+    if (tid < kNB) {
+      const int b = tid, kx = b % 5;
+      float4 ph = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (bi.valid[b]) {
+        const bool edge = kx == 0 || ((w % 2 == 0) && kx == w / 2);
+        const float kap = (edge ? 1.f : 2.f) * inv_n;
+        float sa, ca, sb, cb;
+        const float gt = gate[b] * th[b];
+        sincosf(gt * al, &sa, &ca);
+        sincosf(-gt * (1.f - al), &sb, &cb);
+        ph = make_float4(kap * (1.f - al) * ca, kap * (1.f - al) * sa, kap * al * cb, kap * al * sb);
+      }
+      s_phi[b] = ph;
+    }
+    __syncthreads();
+    {
+      float acc = 0.f;
+      if (dy0 < h && dx0 < w) {
+        for (int b = 0; b < kNB; ++b) {
+          const int ky = b / 5, kx = b % 5;
+          if (ky >= h || kx > w / 2) continue;
+          int p = (int)s_ym[ky][dy0] * w + (int)s_xm[kx][dx0] * h;
+          if (p >= n) p -= n;
+          const float2 e = s_cs[p];
+          const float4 ph = s_phi[b];
+          const float pr = side ? ph.z : ph.x, pi = side ? ph.w : ph.y;
+          acc = fmaf(pr, e.x, fmaf(-pi, e.y, acc));
+        }
+      }
+      s_h[side][d] = acc;
+    }
+    __syncthreads();
+    // thread = (output token m, side): one 64-entry row segment, eight 16-byte chunks per piece
+    uint8_t* img = reinterpret_cast<uint8_t*>(a.img) + ((int64_t)tg * a.n_target + t) * kImgBytes;
+    const int m = tid & 63, yo = m >> 3, xo = m & 7;
+    const bool row_ok = yo < h && xo < w;
+#pragma unroll
+    for (int yi = 0; yi < 8; ++yi) {
+      float v[8];
+      const int dy = yo - yi + (yo < yi ? h : 0);
+#pragma unroll
+      for (int xi = 0; xi < 8; ++xi) {
+        const int dx = xo - xi + (xo < xi ? w : 0);
+        v[xi] = (row_ok && yi < h && xi < w) ? s_h[side][dy * 8 + dx] : 0.f;
+      }
+      uint32_t hi[4], lo[4];
+#pragma unroll
+      for (int u = 0; u < 8; u += 2) {
+        const __nv_bfloat162 b1 = __floats2bfloat162_rn(v[u], v[u + 1]);
+        const __nv_bfloat162 b2 = __floats2bfloat162_rn(v[u] - __low2float(b1), v[u + 1] - __high2float(b1));
+        hi[u / 2] = *reinterpret_cast<const uint32_t*>(&b1);
+        lo[u / 2] = *reinterpret_cast<const uint32_t*>(&b2);
+      }
+      const int off = side * 8192 + m * 128 + ((yi ^ (m & 7)) << 4);
+      *reinterpret_cast<uint4*>(img + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+      *reinterpret_cast<uint4*>(img + kImgTerm + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    }
+    __syncthreads();   // s_phi and s_h are rewritten for the next target
   }
 }
 
@@ -612,6 +715,248 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
     t[tid] = s_th[tid];
     t[kNB + tid] = s_g[tid];
   }
+  if (a.img) build_blend_images(a, g, s_bins, s_th, s_g, tg, j, tid);
+}
+
+// ------------------------------------------------------------------ K_blend_tc (bf16)
+// Persistent, one CTA per SM over the (tile, 128-channel chunk) items of one tile kind, 224
+// threads: warp 0 streams the anchors of each item ([8 x 8 tokens][channels] through a
+// 128-byte-swizzled TMA box, the MN-major UMMA operand) through three stages; warp 6 streams
+// the blend matrices K_transport wrote, two targets of one pair stacked per group (rows 0-63
+// target 1, 64-127 target 2 of the M = 128 operand), two groups in flight;
+// warp 1 issues one UMMA chain per group (2 pieces x 8 K-steps, M = 128, N = 128) into one of
+// two TMEM buffers; warps 2-5 (one TMEM lane quadrant each: a target slot and 32 output tokens)
+// convert the result to bf16 into a swizzled staging tile that one thread stores with TMA.
+constexpr int kTbNC = 128;                      // channels per item
+constexpr int kTbStages = 3;
+constexpr int kTbPlane = 64 * kTbNC * 2;        // one anchor tile, 16 KB
+constexpr int kTbPiece = 128 * 128 * 2;         // one bf16 piece of a group's [128][128] operand, 32 KB
+constexpr int kTbGroup = 2 * kTbPiece;          // both pieces, 64 KB
+constexpr int kTbOut = 2 * kTbPlane;            // two targets' output tiles, 32 KB
+constexpr int kTbThreads = 224;
+constexpr int kTbSmem = kTbStages * kTbPlane + 2 * kTbGroup + kTbOut + 1024;
+
+template <bool FULL>
+__global__ void __launch_bounds__(kTbThreads, 1)
+    k_par_blend_tc(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtensorMap tm_out,
+                   const __grid_constant__ ParKArgs a, int n_tiles) {
+  extern __shared__ uint8_t dsm_raw[];
+  const uint32_t raw_addr = smem_u32(dsm_raw);
+  uint8_t* dsm = dsm_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);   // 128-byte swizzle atoms
+  uint8_t* s_stage = dsm;
+  uint8_t* s_img = dsm + kTbStages * kTbPlane;
+  uint8_t* s_out = s_img + 2 * kTbGroup;
+  __shared__ __align__(8) uint64_t b_full[kTbStages], b_empty[kTbStages], b_ifull[2], b_iempty[2],
+      b_tfull[2], b_tempty[2];
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int n_anc = a.n_anchor;
+  const int nck = (a.C + kTbNC - 1) / kTbNC;   // 128-channel chunks per tile
+  const int n_items = nck * n_tiles;           // item = tile * nck + chunk, CTAs stride the items
+  const uint64_t lim = a.wait_ns;
+  auto wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+    if (s_abort) return false;
+    if (mbar_wait(bar, parity, lim)) return true;
+    s_abort = 1;
+    atomicExch(&g_par_error, 1u);
+    return false;
+  };
+  if (tid == 0) {
+    for (int s = 0; s < kTbStages; ++s) {
+      mbar_init(&b_full[s], 1);
+      mbar_init(&b_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&b_ifull[b], 1);
+      mbar_init(&b_iempty[b], 1);
+      mbar_init(&b_tfull[b], 1);
+      mbar_init(&b_tempty[b], 4);
+    }
+    fence_barrier_init();
+    s_abort = 0;
+  }
+  if (warp == 1) {
+    tmem_alloc(&s_tmem, 2 * kTbNC);
+    tmem_relinquish();
+  }
+  launch_dependents();
+  // the blend images come from the preceding K_transport (and the anchors from kernels before)
+  grid_dependency_wait();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  constexpr uint32_t kAnchorBytes = (uint32_t)kTbPlane;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- anchor producer
+    // anchor load L (counted over the CTA's items) goes into stage L % kTbStages once anchor
+    // L - kTbStages has been released by the UMMA issuer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm);
+      int L = 0;
+      for (int item = blockIdx.x; item < n_items && !s_abort; item += gridDim.x) {
+        const int tile = item / nck, c0 = (item - tile * nck) * kTbNC;
+        const TileGeom g = tile_geom(a, tile, FULL);
+        for (int i = 0; i < n_anc; ++i, ++L) {
+          const int s = L % kTbStages;
+          if (L >= kTbStages && !wait(&b_empty[s], (uint32_t)((L / kTbStages) - 1) & 1u)) break;
+          mbar_arrive_expect_tx(&b_full[s], kAnchorBytes);
+          tma_load_4d(s_stage + s * kTbPlane, &tm, &b_full[s], c0, g.x0, g.y0, a.anchor_frame[i]);
+          tma_load_4d(s_stage + s * kTbPlane + 8192, &tm, &b_full[s], c0 + 64, g.x0, g.y0, a.anchor_frame[i]);
+        }
+      }
+      if (s_abort)   // the copies still in flight land before the shared memory is released
+        for (int l = L > kTbStages ? L - kTbStages : 0; l < L; ++l)
+          mbar_wait(&b_full[l % kTbStages], (uint32_t)(l / kTbStages) & 1u, lim);
+    }
+  } else if (warp == 6) {
+    // ---------------------------------------------------------------- image producer
+    if (lane == 0) {
+      int n = 0;
+      for (int item = blockIdx.x; item < n_items && !s_abort; item += gridDim.x) {
+        const int tg = a.tile_base + item / nck;
+        for (int j = 1; j < n_anc && !s_abort; ++j)
+          for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += 2, ++n) {
+            const int ib = n & 1, nt = min(2, a.pair_tbeg[j + 1] - t0);
+            if (n >= 2 && !wait(&b_iempty[ib], (uint32_t)((n >> 1) - 1) & 1u)) break;
+            mbar_arrive_expect_tx(&b_ifull[ib], (uint32_t)(nt * kImgBytes));
+            uint8_t* dst = s_img + ib * kTbGroup;
+            for (int ts = 0; ts < nt; ++ts) {
+              const char* src = a.img + ((int64_t)tg * a.n_target + t0 + ts) * kImgBytes;
+              // piece p, K-block kb of the target -> rows 64 ts .. 64 ts + 63 of the stacked operand
+              for (int p = 0; p < 2; ++p)
+                for (int kb = 0; kb < 2; ++kb)
+                  bulk_load(dst + p * kTbPiece + kb * 16384 + ts * 8192, src + p * kImgTerm + kb * 8192, 8192u,
+                            &b_ifull[ib]);
+            }
+          }
+      }
+      if (s_abort)   // let the images in flight land (at most the last two groups)
+        for (int l = n > 2 ? n - 2 : 0; l < n; ++l) mbar_wait(&b_ifull[l & 1], (uint32_t)(l >> 1) & 1u, lim);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- UMMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, kTbNC, false, true);
+      int n = 0, L = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; ok && item < n_items; item += gridDim.x, L += n_anc) {
+        if (!wait(&b_full[L % kTbStages], (uint32_t)(L / kTbStages) & 1u)) break;
+        for (int j = 1; ok && j < n_anc; ++j) {
+          const int La = L + j - 1, Lb = L + j;
+          if (!wait(&b_full[Lb % kTbStages], (uint32_t)(Lb / kTbStages) & 1u)) { ok = false; break; }
+          const uint32_t xa = smem_u32(s_stage + (La % kTbStages) * kTbPlane);
+          const uint32_t xb = smem_u32(s_stage + (Lb % kTbStages) * kTbPlane);
+          for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += 2, ++n) {
+            const int ib = n & 1;
+            if (!wait(&b_ifull[ib], (uint32_t)(n >> 1) & 1u) ||
+                (n >= 2 && !wait(&b_tempty[ib], (uint32_t)((n >> 1) - 1) & 1u))) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t im = smem_u32(s_img + ib * kTbGroup), d = tmem + (uint32_t)(ib * kTbNC);
+#pragma unroll
+            for (int p = 0; p < 2; ++p)
+#pragma unroll
+              for (int kk = 0; kk < 8; ++kk)
+                umma_bf16_ss(d, sdesc_sw128(im + p * kTbPiece + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                             sdesc_sw128((kk < 4 ? xa : xb) + (kk & 3) * 2048, 8192, 1024), idesc,
+                             (p | kk) ? 1u : 0u);
+            umma_commit(&b_iempty[ib]);
+            umma_commit(&b_tfull[ib]);
+          }
+          if (ok) umma_commit(&b_empty[La % kTbStages]);   // the pair's UMMAs were anchor La's last readers
+        }
+        if (ok) umma_commit(&b_empty[(L + n_anc - 1) % kTbStages]);   // the item's last anchor
+      }
+      if (s_abort && n > 0) mbar_wait(&b_tfull[(n - 1) & 1], (uint32_t)((n - 1) >> 1) & 1u, lim);
+    }
+  } else if (warp >= 2 && warp <= 5) {
+    // ---------------------------------------------------------------- epilogue warps 2-5
+    // (warp 6 has no role: it goes straight to the final barrier)
+    const int ctid = tid - 64;                 // 0..127
+    const int q = warp & 3;                    // TMEM lanes 32 q .. 32 q + 31
+    const int ts = q >> 1;                     // target slot of this warp
+    const int o = 32 * (q & 1) + lane;         // output token 8 y + x
+    const int yo = o >> 3, xo = o & 7;
+    const bool valid = yo < a.th && xo < a.tw;
+    const int sr = yo * a.tw + xo;             // row inside the store box
+    uint8_t* out = s_out + ts * kTbPlane;
+    bool fail = false;
+    int n = 0;
+    for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+      const int tile = item / nck, c0 = (item - tile * nck) * kTbNC;
+      const TileGeom g = tile_geom(a, tile, FULL);
+      for (int j = 1; j < n_anc; ++j)
+        for (int t0 = a.pair_tbeg[j]; t0 < a.pair_tbeg[j + 1]; t0 += 2, ++n) {
+          const int ib = n & 1, nt = min(2, a.pair_tbeg[j + 1] - t0);
+          if (!fail && !wait(&b_tfull[ib], (uint32_t)(n >> 1) & 1u)) fail = true;
+          // the previous group's TMA stores have read the staging tiles
+          if (ctid == 0) bulk_wait_read_all();
+          if (bar_sync_or(1, 128, fail)) {
+            fail = true;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&b_tempty[ib]);
+            continue;
+          }
+          tc_fence_after();
+          const uint32_t ta = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(ib * kTbNC);
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            // 64 channels (one 128-byte box) at a time
+            uint32_t r[64];
+            tmem_ld_x64(ta + 64 * half, r);
+            if (half == 1) {   // the whole buffer is in registers: it goes back to the issuer
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&b_tempty[ib]);
+            }
+            if (ts < nt && valid) {
+#pragma unroll
+              for (int c8 = 0; c8 < 8; ++c8) {
+                uint32_t pk[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                  const __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(r[8 * c8 + 2 * u]),
+                                                                  __uint_as_float(r[8 * c8 + 2 * u + 1]));
+                  pk[u] = *reinterpret_cast<const uint32_t*>(&b2);
+                }
+                *reinterpret_cast<uint4*>(out + half * 8192 + sr * 128 + ((c8 ^ (sr & 7)) << 4)) =
+                    make_uint4(pk[0], pk[1], pk[2], pk[3]);
+              }
+            }
+          }
+          fence_proxy_async_smem();
+          bar_sync_or(1, 128, false);
+          if (ctid == 0) {
+            for (int u = 0; u < nt; ++u)
+              for (int b = 0; b < 2; ++b)
+                if (c0 + 64 * b < a.C)
+                  tma_store_4d(&tm_out, s_out + u * kTbPlane + b * 8192, c0 + 64 * b, g.x0, g.y0,
+                               a.target_frame[t0 + u]);
+            bulk_commit();
+          }
+        }
+    }
+    if (ctid == 0) bulk_wait_all();
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, 2 * kTbNC);
+}
+
+// 4-D map [F][Hg][Wg][C] with a 128-byte-swizzled box (64 bf16 channels, bw, bh, 1)
+bool make_r_map_sw(CUtensorMap* m, const cast_par_args& a, int bw, int bh) {
+  EncodeTiledFn fn = tensor_map_encoder();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.Wg, (cuuint64_t)a.Hg, (cuuint64_t)a.F};
+  cuuint64_t strides[3] = {a.C * 2ull, (cuuint64_t)a.Wg * a.C * 2, (cuuint64_t)a.Hg * a.Wg * a.C * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)bw, (cuuint32_t)bh, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, a.r, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // 4-D map [F][Hg][Wg][C], box (cc channels, tw, th, 1), zero fill out of range
@@ -630,14 +975,17 @@ bool make_r_map(CUtensorMap* m, const cast_par_args& a, int cc) {
 
 // One tile kind on one stream: K_stats, then K_transport and K_blend as programmatic dependents.
 template <typename T, bool FULL>
-cast_status launch_kind(const CUtensorMap& tm, const ParKArgs& k, int n_tiles, cudaStream_t st) {
+cast_status launch_kind(const CUtensorMap& tm, const CUtensorMap* tm_sw, const CUtensorMap* tm_out,
+                        const ParKArgs& k, int n_tiles, cudaStream_t st) {
   const size_t smem = par_dyn_smem<T>(kCC);
   static std::atomic<uint64_t> attr_done{0};
   if (!once_per_device(attr_done, [smem] {
         return cudaFuncSetAttribute(k_par<T, kCC, FULL, true>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess &&
                cudaFuncSetAttribute(k_par<T, kCC, FULL, false>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess;
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess &&
+               cudaFuncSetAttribute(k_par_blend_tc<FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    kTbSmem) == cudaSuccess;
       }))
     return check_launch("PAR kernel attributes");
   cudaLaunchAttribute pdl[1];
@@ -660,8 +1008,24 @@ cast_status launch_kind(const CUtensorMap& tm, const ParKArgs& k, int n_tiles, c
     return check_launch("PAR transport kernel");
   cfg.attrs = pdl;
   cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, k_par<T, kCC, FULL, false>, tm, k) != cudaSuccess)
+  if (k.img) {
+    // bf16: the blend as tensor-core GEMMs over the matrices K_transport wrote
+    // persistent: one CTA per SM over the (tile, 128-channel chunk) items of this kind
+    int dev = 0, nsm = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    const int items = ((k.C + kTbNC - 1) / kTbNC) * n_tiles;
+    cudaLaunchConfig_t bc{};
+    bc.gridDim = dim3(items < nsm ? items : nsm, 1, 1);
+    bc.blockDim = dim3(kTbThreads, 1, 1);
+    bc.dynamicSmemBytes = kTbSmem;
+    bc.stream = st;
+    bc.attrs = pdl;
+    bc.numAttrs = 1;
+    if (cudaLaunchKernelEx(&bc, k_par_blend_tc<FULL>, *tm_sw, *tm_out, k, n_tiles) != cudaSuccess)
+      return check_launch("PAR tensor-core blend kernel");
+  } else if (cudaLaunchKernelEx(&cfg, k_par<T, kCC, FULL, false>, tm, k) != cudaSuccess) {
     return check_launch("PAR blend kernel");
+  }
   return check_launch("PAR kernels");
 }
 
@@ -705,21 +1069,22 @@ ParKArgs with_segments(const ParKArgs& k0, int nseg) {
 }
 
 template <typename T>
-cast_status launch_typed(const CUtensorMap& tm, const ParKArgs& k0, const ParPlan& p, cudaStream_t st) {
+cast_status launch_typed(const CUtensorMap& tm, const CUtensorMap* tm_sw, const CUtensorMap* tm_out,
+                         const ParKArgs& k0, const ParPlan& p, cudaStream_t st) {
   ParKArgs kf = with_segments(k0, p.n_tseg_full), ke = with_segments(k0, p.n_tseg_edge);
   kf.tile_base = 0;
   ke.tile_base = p.n_full;
-  if (p.n_edge == 0) return launch_kind<T, true>(tm, kf, p.n_full, st);
-  if (p.n_full == 0) return launch_kind<T, false>(tm, ke, p.n_edge, st);
+  if (p.n_edge == 0) return launch_kind<T, true>(tm, tm_sw, tm_out, kf, p.n_full, st);
+  if (p.n_full == 0) return launch_kind<T, false>(tm, tm_sw, tm_out, ke, p.n_edge, st);
   // full tiles on the caller's stream, edge tiles concurrently on the side stream
   ForkStream* f = nullptr;
   cast_status s = fork_stream(f);
   if (s != CAST_OK) return s;
   if (cudaEventRecord(f->fork, st) != cudaSuccess || cudaStreamWaitEvent(f->side, f->fork, 0) != cudaSuccess)
     return check_launch("PAR fork");
-  s = launch_kind<T, false>(tm, ke, p.n_edge, f->side);
+  s = launch_kind<T, false>(tm, tm_sw, tm_out, ke, p.n_edge, f->side);
   if (s != CAST_OK) return s;
-  s = launch_kind<T, true>(tm, kf, p.n_full, st);
+  s = launch_kind<T, true>(tm, tm_sw, tm_out, kf, p.n_full, st);
   if (cudaEventRecord(f->join, f->side) != cudaSuccess || cudaStreamWaitEvent(st, f->join, 0) != cudaSuccess)
     return check_launch("PAR join");
   return s;
@@ -769,7 +1134,9 @@ ParPlan par_plan(const cast_par_args& a) {
   // workspace: the chunk records [tile][pair][chunk][kRec] and theta, g [tile][pair][2][kNB]
   p.rec_bytes = align_up((size_t)p.n_tile * (na > 0 ? na : 1) * p.n_chunk * kRec * sizeof(float));
   p.trans_bytes = align_up((size_t)p.n_tile * (na > 0 ? na : 1) * 2 * kNB * sizeof(float));
-  p.total_bytes = p.n_target > 0 ? p.rec_bytes + p.trans_bytes : 0;
+  // bf16: the blend matrices of every (tile, target)
+  p.img_bytes = a.dtype == CAST_BF16 ? align_up((size_t)p.n_tile * (p.n_target > 0 ? p.n_target : 1) * kImgBytes) : 0;
+  p.total_bytes = p.n_target > 0 ? p.rec_bytes + p.trans_bytes + p.img_bytes : 0;
   return p;
 }
 
@@ -791,6 +1158,8 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
   k.n_chunk = p.n_chunk;
   k.rec = static_cast<float*>(ws);
   k.trans = reinterpret_cast<float*>(static_cast<char*>(ws) + p.rec_bytes);
+  k.img = p.img_bytes ? static_cast<char*>(ws) + p.rec_bytes + p.trans_bytes : nullptr;
+  k.n_target = p.n_target;
   int anchors[CAST_MAX_FRAMES];
   int na = 0;
   for (int f = 0; f < a.F; ++f)
@@ -847,8 +1216,13 @@ cast_status launch_par(const cast_par_args& a, void* ws, cudaStream_t st) {
 
   CUtensorMap tm;
   if (!make_r_map(&tm, a, p.chunk)) return fail(CAST_ERR_CUDA, "PAR: cuTensorMapEncodeTiled failed");
-  if (a.dtype == CAST_BF16) return launch_typed<__nv_bfloat16>(tm, k, p, st);
-  return launch_typed<float>(tm, k, p, st);
+  if (a.dtype == CAST_BF16) {
+    CUtensorMap tm_sw, tm_out;
+    if (!make_r_map_sw(&tm_sw, a, 8, 8) || !make_r_map_sw(&tm_out, a, k.tw, k.th))
+      return fail(CAST_ERR_CUDA, "PAR: cuTensorMapEncodeTiled failed");
+    return launch_typed<__nv_bfloat16>(tm, &tm_sw, &tm_out, k, p, st);
+  }
+  return launch_typed<float>(tm, nullptr, nullptr, k, p, st);
 }
 
 unsigned int par_error_word(cudaStream_t st, bool clear) {

@@ -130,3 +130,27 @@ def test_par_sweep_full_size_sampled(lib, dtype, spacing):
             continue
         sl = (slice(y0, y0 + h), slice(x0, x0 + ww))
         par_check(gpu[:, sl[0], sl[1]], ref[:, sl[0], sl[1]], targets, dtype)
+
+
+def test_par_tensor_core_blend_edge_shapes(lib):
+    """bf16 with enough (tile, 128-channel chunk) items per tile kind that both the full 8x8
+    tiles and the truncated edge tiles (8x4 right column, 6x8 bottom row, 6x4 corner of a 30x52
+    grid) take the tensor-core blend; one pair carries five targets (two stacked groups and a
+    single), frames 5 and 6 extrapolated.  Every output of the edge tiles and of two full tiles
+    against the oracle."""
+    F, Hg, Wg, Cc, anchors = 7, 30, 52, 4096, (0, 4)
+    R, _ = G.grf_sequence(np.random.SeedSequence([F, Hg, Wg, Cc, 7]), F, Hg, Wg, Cc, ell=3.0)
+    mask = W.anchor_mask(F, anchors)
+    gpu = _run(lib, R, mask, "bf16")
+    tiles_all = O.tiles_of(Hg, Wg, 8, 8)
+    sample = [i for i, (y0, h, x0, w) in enumerate(tiles_all) if h < 8 or w < 8] + [0, 8]
+    ref, info, _ = _oracle(R, mask, "bf16", tiles=sample)
+    amb = _ambiguous_tiles(info, tiles_all)
+    assert len(amb) <= 1
+    targets = [t for t in range(F) if not mask[t]]
+    for ti in sample:
+        y0, h, x0, w = tiles_all[ti]
+        if (y0, x0) in amb:
+            continue
+        sl = (slice(y0, y0 + h), slice(x0, x0 + w))
+        par_check(gpu[:, sl[0], sl[1]], ref[:, sl[0], sl[1]], targets, "bf16")
