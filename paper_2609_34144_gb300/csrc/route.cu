@@ -595,6 +595,236 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const __grid_constant__ H
   }
 }
 
+// ---------------------------------------------------------------------- small per-head kernel
+// The same statistics, TopK and refinement for the common small case (no Gram matrix, no
+// candidate sets, M <= 32 blocks, at most 8 anchors), with one warp per anchor and lane m =
+// block m, so that the phases need no block-wide barriers: lane m forms s_m, the warp's
+// shuffles give the softmax, lanes split o_bar by dimensions, lane m forms u_m and its rank.
+// The refinement passes (Alg. routing) run in warp 0 with every anchor's u, sqrt(u u) of the
+// adjacent pairs and the masks (ballots) in registers, TopK(G) ranked by shuffles.
+constexpr int kSmallMaxM = 32, kSmallMaxAnchors = 8;
+
+// shared memory (floats): qb[na][d], ob[na][d], kb[M][d + 4], vb[M][d + 4] (rows padded so
+// that lane m's 16-byte reads of row m fall in distinct bank groups), key[na][32]
+size_t small_head_bytes(const cast_route_args& a) {
+  const int dp = a.d + 4;
+  return ((size_t)2 * a.n_anchors * a.d + (size_t)2 * a.M * dp + (size_t)a.n_anchors * kSmallMaxM) * sizeof(float);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kHeadThreads) k_head_small(const __grid_constant__ HeadArgs a) {
+  extern __shared__ float sm[];
+  constexpr int d = HD, dp = d + 4, d4 = d / 4;
+  const int h = blockIdx.x, na = a.n_anchors, M = a.M, K = a.K_eff;
+  const int D = a.H * d;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  float* qb = sm;
+  float* ob = qb + na * d;
+  float* kb = ob + na * d;
+  float* vb = kb + M * dp;
+  float* key = vb + M * dp;
+  __shared__ uint32_t s_mask[kSmallMaxAnchors];
+  launch_dependents();
+  grid_dependency_wait();   // the pooled means come from the preceding kernel
+  {
+    // q_bar rows of every anchor, then k_bar and v_bar rows; up to 8 loads in flight per thread
+    const int n_q = na * d4, n_all = n_q + 2 * M * d4;
+    for (int e0 = tid; e0 < n_all; e0 += 8 * kHeadThreads) {
+      float4 v[8];
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const int e = e0 + t * kHeadThreads;
+        if (e < n_q) {
+          const int i = e / d4, c = (e - i * d4) * 4;
+          v[t] = __ldcg(reinterpret_cast<const float4*>(a.qbar + (int64_t)i * D + h * d + c));
+        } else if (e < n_all) {
+          const int f = e - n_q, m = (f >> 1) / d4, c = ((f >> 1) - m * d4) * 4;
+          v[t] = __ldcg(reinterpret_cast<const float4*>(((f & 1) ? a.vbar : a.kbar) + (int64_t)m * D + h * d + c));
+        }
+      }
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const int e = e0 + t * kHeadThreads;
+        if (e < n_q) {
+          const int i = e / d4, c = (e - i * d4) * 4;
+          *reinterpret_cast<float4*>(qb + i * d + c) = v[t];
+        } else if (e < n_all) {
+          const int f = e - n_q, m = (f >> 1) / d4, c = ((f >> 1) - m * d4) * 4;
+          *reinterpret_cast<float4*>(((f & 1) ? vb : kb) + m * dp + c) = v[t];
+        }
+      }
+    }
+  }
+  __syncthreads();
+  const bool live = lane < M;
+  if (warp < na) {
+    const int i = warp;
+    // s_m = q_bar_i . k_bar_m / sqrt(d)   (Eq. pooled)
+    const float4* q4 = reinterpret_cast<const float4*>(qb + i * d);
+    const float4* k4 = reinterpret_cast<const float4*>(kb + (live ? lane : 0) * dp);
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < d4; ++c) {
+      const float4 x = q4[c], y = k4[c];
+      acc[c & 3] = fmaf(x.x, y.x, fmaf(x.y, y.y, fmaf(x.z, y.z, fmaf(x.w, y.w, acc[c & 3]))));
+    }
+    const float s = live ? ((acc[0] + acc[1]) + (acc[2] + acc[3])) * rsqrtf((float)d) : -FLT_MAX;
+    float u;
+    if (a.mode == CAST_ROUTE_OMISSION) {
+      // pi = softmax over blocks; o_bar = sum pi_m v_bar_m; u_m = (pi_m / (1 - pi_m + eps))^2 |o_bar - v_bar_m|^2
+      const float mx = warp_max(s);
+      const float e = live ? expf(s - mx) : 0.f;
+      const float pi = e / warp_sum(e);
+      // pi through shared memory (this anchor's key row, rewritten with u below): the
+      // dimension loop below runs on d / 4 lanes only
+      if (live) key[i * kSmallMaxM + lane] = pi;
+      __syncwarp();
+      if (lane < d4) {
+        const int c = lane;
+        float4 o[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+#pragma unroll
+        for (int m = 0; m < kSmallMaxM; ++m) {
+          if (m < M) {
+            const float pm = key[i * kSmallMaxM + m];
+            const float4 v = *reinterpret_cast<const float4*>(vb + m * dp + 4 * c);
+            float4& t = o[m & 1];
+            t.x = fmaf(pm, v.x, t.x);
+            t.y = fmaf(pm, v.y, t.y);
+            t.z = fmaf(pm, v.z, t.z);
+            t.w = fmaf(pm, v.w, t.w);
+          }
+        }
+        *reinterpret_cast<float4*>(ob + i * d + 4 * c) =
+            make_float4(o[0].x + o[1].x, o[0].y + o[1].y, o[0].z + o[1].z, o[0].w + o[1].w);
+      }
+      __syncwarp();
+      const float4* o4 = reinterpret_cast<const float4*>(ob + i * d);
+      const float4* v4 = reinterpret_cast<const float4*>(vb + (live ? lane : 0) * dp);
+      float dist[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < d4; ++c) {
+        const float4 x = o4[c], y = v4[c];
+        const float t0 = x.x - y.x, t1 = x.y - y.y, t2 = x.z - y.z, t3 = x.w - y.w;
+        dist[c & 3] = fmaf(t0, t0, fmaf(t1, t1, fmaf(t2, t2, fmaf(t3, t3, dist[c & 3]))));
+      }
+      const float coef = pi / (1.f - pi + a.eps);
+      u = live ? coef * coef * ((dist[0] + dist[1]) + (dist[2] + dist[3])) : 0.f;
+    } else {
+      u = live ? s : 0.f;   // SIMILARITY: TopK on the pooled score
+    }
+    if (live) {
+      key[i * kSmallMaxM + lane] = u;
+      if (a.u_out) a.u_out[((int64_t)i * a.H + h) * M + lane] = u;
+    }
+    // initial mask: TopK of u (Eq. topk), ties to the lower block index
+    const float uk = live ? u : -INFINITY;
+    int rank = 0;
+    for (int l = 0; l < M; ++l) {
+      const float w = __shfl_sync(0xffffffffu, uk, l);
+      rank += (w > uk) || (w == uk && l < lane);
+    }
+    const uint32_t mask = __ballot_sync(0xffffffffu, live && rank < K);
+    if (lane == 0) s_mask[i] = mask;
+  }
+  if (K == 0) return;
+  __syncthreads();
+  if (warp == 0) {
+    uint32_t mk[kSmallMaxAnchors];
+    float uu[kSmallMaxAnchors], sq[kSmallMaxAnchors];
+#pragma unroll
+    for (int k = 0; k < kSmallMaxAnchors; ++k) {
+      mk[k] = k < na ? s_mask[k] : 0u;
+      uu[k] = (k < na && live) ? key[k * kSmallMaxM + lane] : 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < kSmallMaxAnchors; ++k) sq[k] = (k >= 1 && k < na) ? sqrtf(uu[k - 1] * uu[k]) : 0.f;
+    if (a.passes > 0 && K < M) {
+      auto xb = [&](int k) -> float {   // 1 - x_{k, lane} (omission indicator), k < na
+        uint32_t v = 0u;
+#pragma unroll
+        for (int t = 0; t < kSmallMaxAnchors; ++t)
+          if (t == k) v = mk[t];
+        return ((v >> lane) & 1u) ? 0.f : 1.f;
+      };
+      auto pick = [&](const float* arr, int k) -> float {
+        float v = 0.f;
+#pragma unroll
+        for (int t = 0; t < kSmallMaxAnchors; ++t)
+          if (t == k) v = arr[t];
+        return v;
+      };
+      const float AL = a.AL, BL = a.BL, CL = a.CL, AR = a.AR, BR = a.BR, CR = a.CR;
+      const float lam_anc = a.lam_anc, lam_rec = a.lam_rec;
+      // J of the current masks (Eq. objective)
+      float Jl = 0.f;
+      if (live) {
+#pragma unroll
+        for (int k = 0; k < kSmallMaxAnchors; ++k)
+          if (k < na) Jl += lam_anc * xb(k) * uu[k];
+        float rec = 0.f;
+#pragma unroll
+        for (int j = 1; j < kSmallMaxAnchors; ++j)
+          if (j < na) {
+            const float xp = xb(j - 1), xq = xb(j);
+            rec += a.A[j] * xp * uu[j - 1] + a.B[j] * xq * uu[j] + 2.f * a.C[j] * xp * xq * sq[j];
+          }
+        if (na >= 2) {
+          const float x0 = xb(0), x1 = xb(1);
+          rec += AL * x0 * uu[0] + BL * x1 * uu[1] + 2.f * CL * x0 * x1 * sq[1];
+          const float y0 = xb(na - 2), y1 = xb(na - 1);
+          rec += AR * y0 * pick(uu, na - 2) + BR * y1 * pick(uu, na - 1) + 2.f * CR * y0 * y1 * pick(sq, na - 1);
+        }
+        Jl += lam_rec * rec;
+      }
+      float J = warp_sum(Jl);
+      for (int pass = 1; pass <= a.passes; ++pass) {
+        bool changed = false;
+        for (int step = 0; step < na; ++step) {
+          const int i = (pass & 1) ? step : na - 1 - step;
+          // retain gains, Eqs. (gain) and (boundarygain)
+          const float ui = pick(uu, i);
+          float rec = 0.f;
+          if (i >= 1) rec += a.B[i] * ui + 2.f * a.C[i] * xb(i - 1) * pick(sq, i);
+          if (i + 1 < na) rec += a.A[i + 1] * ui + 2.f * a.C[i + 1] * xb(i + 1) * pick(sq, i + 1);
+          if (na >= 2) {
+            if (i == 0) rec += AL * ui + 2.f * CL * xb(1) * sq[1];
+            if (i == 1) rec += BL * ui + 2.f * CL * xb(0) * sq[1];
+            if (i == na - 2) rec += AR * ui + 2.f * CR * xb(na - 1) * pick(sq, na - 1);
+            if (i == na - 1) rec += BR * ui + 2.f * CR * xb(na - 2) * pick(sq, na - 1);
+          }
+          const float G = live ? lam_anc * ui + lam_rec * rec : -INFINITY;
+          // best response TopK(G) and its gain sum_m G_m (x_new - x_i) (J is affine in x_i)
+          int rank = 0;
+          for (int l = 0; l < M; ++l) {
+            const float w = __shfl_sync(0xffffffffu, G, l);
+            rank += (w > G) || (w == G && l < lane);
+          }
+          const bool in = live && rank < K;
+          const float xi = 1.f - xb(i);
+          const float gain = warp_sum(live ? G * ((in ? 1.f : 0.f) - xi) : 0.f);
+          if (gain > a.tol * fmaxf(J, 1e-8f)) {   // uniform across the warp
+            const uint32_t nm = __ballot_sync(0xffffffffu, in);
+#pragma unroll
+            for (int t = 0; t < kSmallMaxAnchors; ++t)
+              if (t == i) mk[t] = nm;
+            J -= gain;
+            changed = true;
+          }
+        }
+        if (!changed) break;
+      }
+    }
+    // ascending block indices of every anchor's mask
+    for (int i = 0; i < na; ++i) {
+      uint32_t v = 0u;
+#pragma unroll
+      for (int t = 0; t < kSmallMaxAnchors; ++t)
+        if (t == i) v = mk[t];
+      if ((v >> lane) & 1u) a.idx[((int64_t)i * a.H + h) * K + __popc(v & ((1u << lane) - 1u))] = lane;
+    }
+  }
+}
+
 // ---------------------------------------------------------------------- wide per-head kernel
 // For many history blocks (k_bar, v_bar of a head too large for one CTA's shared memory) the
 // statistics of one head are spread over a cluster of cl CTAs, each owning a contiguous range
@@ -1293,8 +1523,12 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
            a.n_frames, ha.AR, ha.BR, ha.CR);
     }
   }
-  const size_t hsm = route_head_smem_bytes(a);
-  auto head_fn = !p.wide ? k_head : (a.d == 128 ? k_head_wide<128> : k_head_wide<64>);
+  // the small per-head kernel for the common case; the staged or wide kernel otherwise
+  const bool small = !p.wide && a.gram == nullptr && a.candidates == nullptr && a.M <= kSmallMaxM &&
+                     a.n_anchors <= kSmallMaxAnchors;
+  const size_t hsm = small ? small_head_bytes(a) : route_head_smem_bytes(a);
+  auto head_fn = small ? (a.d == 128 ? k_head_small<128> : k_head_small<64>)
+                       : !p.wide ? k_head : (a.d == 128 ? k_head_wide<128> : k_head_wide<64>);
   if (hsm > 48 * 1024 &&
       cudaFuncSetAttribute(head_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)hsm) != cudaSuccess)
     return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory", hsm);
