@@ -26,6 +26,7 @@
 // pair and chunk).
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cmath>
 #include <mutex>
 
@@ -368,7 +369,7 @@ __device__ void tile_transport(const ParKArgs& a, const TileGeom& g, const BinIn
 constexpr int kImgTerm = 64 * 128 * 2;   // one bf16 piece of one target's [64][128] matrix, 16 KB
 constexpr int kImgBytes = 2 * kImgTerm;  // both pieces (hi, lo): 32 KB per (tile, target)
 
-// The blend matrices of every target t of one (tile, pair), written as UMMA operand images
+// The blend matrices of the targets t_begin <= t < t_end of one (tile, pair), written as UMMA operand images
 // (K-major, 128-byte swizzle, K-blocks of 64 tokens 8 KB apart, two bf16 pieces kImgTerm apart):
 // row m = output token 8 yo + xo, column 64 side + 8 yi + xi = input token of anchor a (side 0)
 // or b (side 1); entry h_side((yo - yi) mod h, (xo - xi) mod w) with
@@ -376,7 +377,8 @@ constexpr int kImgBytes = 2 * kImgTerm;  // both pieces (hi, lo): 32 KB per (til
 // kappa' = 1 on the kx = 0 and Nyquist columns (every ky stored), 2 elsewhere;
 // phi_a = (1 - alpha) e^{i g alpha theta}, phi_b = alpha e^{-i g (1 - alpha) theta}.  128 threads.
 __device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const BinInfo& bi,
-                                   const float* th, const float* gate, int tg, int j, int tid) {
+                                   const float* th, const float* gate, int tg, int t_begin, int t_end,
+                                   int tid) {
   __shared__ float2 s_cs[64];
   __shared__ unsigned char s_ym[8][8], s_xm[5][8];
   __shared__ float4 s_phi[kNB];
@@ -395,7 +397,7 @@ __device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const B
   }
   const float inv_n = 1.f / (float)n;
   const int side = tid >> 6, d = tid & 63, dy0 = d >> 3, dx0 = d & 7;
-  for (int t = a.pair_tbeg[j]; t < a.pair_tbeg[j + 1]; ++t) {
+  for (int t = t_begin; t < t_end; ++t) {
     const float al = a.target_alpha[t];
     if (tid < kNB) {
       const int b = tid, kx = b % 5;
@@ -672,7 +674,9 @@ __global__ void __launch_bounds__(CC, 3)
   }
 }
 
-// K_transport: grid (n_tiles_of_kind, n_anchor - 1), 128 threads; block y = pair j - 1.
+// K_transport: grid (n_tiles_of_kind, n_anchor - 1, z), 128 threads; block y = pair j - 1.  With
+// blend matrices (bf16) block z builds the matrix of the pair's target z (z < the largest target
+// count of a pair; every block of a (tile, pair) solves the same transport), else z = 0 only.
 template <bool FULL>
 __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ ParKArgs a) {
   __shared__ float s_zw[kNV];
@@ -681,8 +685,9 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
   __shared__ BinInfo s_bins;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int tile = blockIdx.x, j = blockIdx.y + 1, tg = a.tile_base + tile;
+  const int t = a.pair_tbeg[j] + (int)blockIdx.z;   // this block's target
   launch_dependents();
-  if (!(a.pair_tbeg[j + 1] > a.pair_tbeg[j])) return;   // no targets: no record
+  if (!(a.pair_tbeg[j + 1] > t)) return;   // no (further) target: no record
   const TileGeom g = tile_geom(a, tile, FULL);
   bin_info(a, g, s_bins, tid);
   grid_dependency_wait();   // the records come from the preceding K_stats
@@ -710,12 +715,12 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
   __syncthreads();
   if (warp == 0) tile_transport(a, g, s_bins, s_zw, s_th, s_g, s_own_th, s_own_rel, lane);
   __syncthreads();
-  if (tid < kNB) {
-    float* t = a.trans + ((int64_t)tg * a.n_anchor + j) * 2 * kNB;
-    t[tid] = s_th[tid];
-    t[kNB + tid] = s_g[tid];
+  if (tid < kNB && blockIdx.z == 0) {
+    float* tr = a.trans + ((int64_t)tg * a.n_anchor + j) * 2 * kNB;
+    tr[tid] = s_th[tid];
+    tr[kNB + tid] = s_g[tid];
   }
-  if (a.img) build_blend_images(a, g, s_bins, s_th, s_g, tg, j, tid);
+  if (a.img) build_blend_images(a, g, s_bins, s_th, s_g, tg, t, t + 1, tid);
 }
 
 // ------------------------------------------------------------------ K_blend_tc (bf16)
@@ -998,8 +1003,11 @@ cast_status launch_kind(const CUtensorMap& tm, const CUtensorMap* tm_sw, const C
   cfg.stream = st;
   if (cudaLaunchKernelEx(&cfg, k_par<T, kCC, FULL, true>, tm, k) != cudaSuccess)
     return check_launch("PAR statistics kernel");
+  int zmax = 1;   // one transport block per (tile, pair, target) when it writes blend matrices
+  if (k.img)
+    for (int j = 1; j < k.n_anchor; ++j) zmax = std::max(zmax, k.pair_tbeg[j + 1] - k.pair_tbeg[j]);
   cudaLaunchConfig_t tc{};
-  tc.gridDim = dim3(n_tiles, k.n_anchor - 1, 1);
+  tc.gridDim = dim3(n_tiles, k.n_anchor - 1, zmax);
   tc.blockDim = dim3(128, 1, 1);
   tc.stream = st;
   tc.attrs = pdl;
