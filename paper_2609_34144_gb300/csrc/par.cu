@@ -376,6 +376,9 @@ constexpr int kImgBytes = 2 * kImgTerm;  // both pieces (hi, lo): 32 KB per (til
 // h_side(d) = (1 / (h w)) sum over stored bins of kappa' Re(phi_side e^{2 pi i (ky dy / h + kx dx / w)}),
 // kappa' = 1 on the kx = 0 and Nyquist columns (every ky stored), 2 elsewhere;
 // phi_a = (1 - alpha) e^{i g alpha theta}, phi_b = alpha e^{-i g (1 - alpha) theta}.  128 threads.
+// FULL8: an 8x8 tile, where every twiddle is an 8th root of unity and every index a mask (the
+// same values, summed in the same order, as the general form).
+template <bool FULL8>
 __device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const BinInfo& bi,
                                    const float* th, const float* gate, int tg, int t_begin, int t_end,
                                    int tid) {
@@ -383,8 +386,15 @@ __device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const B
   __shared__ unsigned char s_ym[8][8], s_xm[5][8];
   __shared__ float4 s_phi[kNB];
   __shared__ float s_h[2][64];
-  const int h = g.h, w = g.w, n = h * w;
-  if (tid < 64) {
+  const int h = FULL8 ? 8 : g.h, w = FULL8 ? 8 : g.w, n = h * w;
+  if (FULL8) {
+    // e^{2 pi i q / 8} at s_cs[q]
+    if (tid < 8) {
+      float sv, cv;
+      sincospif((float)tid / 4.f, &sv, &cv);
+      s_cs[tid] = make_float2(cv, sv);
+    }
+  } else if (tid < 64) {
     if (tid < n) {
       float sv, cv;
       sincospif(2.f * (float)tid / (float)n, &sv, &cv);
@@ -414,7 +424,21 @@ __device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const B
       s_phi[b] = ph;
     }
     __syncthreads();
-    {
+    if (FULL8) {
+      float acc = 0.f;
+#pragma unroll
+      for (int ky = 0; ky < 8; ++ky) {
+        const int ry = ky * dy0;
+#pragma unroll
+        for (int kx = 0; kx < 5; ++kx) {
+          const float2 e = s_cs[(ry + kx * dx0) & 7];
+          const float4 ph = s_phi[ky * 5 + kx];
+          const float pr = side ? ph.z : ph.x, pi = side ? ph.w : ph.y;
+          acc = fmaf(pr, e.x, fmaf(-pi, e.y, acc));
+        }
+      }
+      s_h[side][d] = acc;
+    } else {
       float acc = 0.f;
       if (dy0 < h && dx0 < w) {
         for (int b = 0; b < kNB; ++b) {
@@ -431,18 +455,20 @@ __device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const B
       s_h[side][d] = acc;
     }
     __syncthreads();
-    // thread = (output token m, side): one 64-entry row segment, eight 16-byte chunks per piece
+    // 16-byte chunk q = 128 it + tid of a piece: side q >> 9, output token (row) m = (q >> 3) & 63,
+    // stored chunk q & 7 = input row yi ^ (m & 7); a warp writes 512 contiguous bytes per piece
     uint8_t* img = reinterpret_cast<uint8_t*>(a.img) + ((int64_t)tg * a.n_target + t) * kImgBytes;
-    const int m = tid & 63, yo = m >> 3, xo = m & 7;
-    const bool row_ok = yo < h && xo < w;
 #pragma unroll
-    for (int yi = 0; yi < 8; ++yi) {
+    for (int it = 0; it < 8; ++it) {
+      const int q = it * 128 + tid, sd = q >> 9, m = (q >> 3) & 63, yi = (q & 7) ^ (m & 7);
+      const int yo = m >> 3, xo = m & 7;
+      const bool row_ok = FULL8 || (yo < h && xo < w && yi < h);
+      const int dy = FULL8 ? (yo - yi) & 7 : yo - yi + (yo < yi ? h : 0);
       float v[8];
-      const int dy = yo - yi + (yo < yi ? h : 0);
 #pragma unroll
       for (int xi = 0; xi < 8; ++xi) {
-        const int dx = xo - xi + (xo < xi ? w : 0);
-        v[xi] = (row_ok && yi < h && xi < w) ? s_h[side][dy * 8 + dx] : 0.f;
+        const int dx = FULL8 ? (xo - xi) & 7 : xo - xi + (xo < xi ? w : 0);
+        v[xi] = (FULL8 || (row_ok && xi < w)) ? s_h[sd][dy * 8 + dx] : 0.f;
       }
       uint32_t hi[4], lo[4];
 #pragma unroll
@@ -452,7 +478,7 @@ __device__ void build_blend_images(const ParKArgs& a, const TileGeom& g, const B
         hi[u / 2] = *reinterpret_cast<const uint32_t*>(&b1);
         lo[u / 2] = *reinterpret_cast<const uint32_t*>(&b2);
       }
-      const int off = side * 8192 + m * 128 + ((yi ^ (m & 7)) << 4);
+      const int off = q << 4;   // side * 8192 + m * 128 + ((yi ^ (m & 7)) << 4)
       *reinterpret_cast<uint4*>(img + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
       *reinterpret_cast<uint4*>(img + kImgTerm + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
     }
@@ -686,8 +712,10 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int tile = blockIdx.x, j = blockIdx.y + 1, tg = a.tile_base + tile;
   const int t = a.pair_tbeg[j] + (int)blockIdx.z;   // this block's target
-  launch_dependents();
-  if (!(a.pair_tbeg[j + 1] > t)) return;   // no (further) target: no record
+  if (!(a.pair_tbeg[j + 1] > t)) {   // no (further) target: no record
+    launch_dependents();
+    return;
+  }
   const TileGeom g = tile_geom(a, tile, FULL);
   bin_info(a, g, s_bins, tid);
   grid_dependency_wait();   // the records come from the preceding K_stats
@@ -700,14 +728,14 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
     }
     float sum = 0.f;
     if (k >= 0) {
-      // chunk order; eight loads in flight per round
+      // chunk order; twelve loads in flight per round
       const float* r = a.rec + ((int64_t)tg * a.n_anchor + j) * a.n_chunk * kRec + k;
-      for (int ch0 = 0; ch0 < a.n_chunk; ch0 += 8) {
-        float v[8];
+      for (int ch0 = 0; ch0 < a.n_chunk; ch0 += 12) {
+        float v[12];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) v[u] = ch0 + u < a.n_chunk ? __ldcg(r + (int64_t)(ch0 + u) * kRec) : 0.f;
+        for (int u = 0; u < 12; ++u) v[u] = ch0 + u < a.n_chunk ? __ldcg(r + (int64_t)(ch0 + u) * kRec) : 0.f;
 #pragma unroll
-        for (int u = 0; u < 8; ++u) sum += v[u];
+        for (int u = 0; u < 12; ++u) sum += v[u];
       }
     }
     s_zw[tid] = sign < 0 ? -sum : sum;
@@ -720,7 +748,10 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
     tr[tid] = s_th[tid];
     tr[kNB + tid] = s_g[tid];
   }
-  if (a.img) build_blend_images(a, g, s_bins, s_th, s_g, tg, t, t + 1, tid);
+  if (a.img) build_blend_images<FULL>(a, g, s_bins, s_th, s_g, tg, t, t + 1, tid);
+  // the blend is released only now: a tensor-core blend CTA takes a whole SM's shared memory,
+  // and released early it would leave room for too few of this grid's blocks
+  launch_dependents();
 }
 
 // ------------------------------------------------------------------ K_blend_tc (bf16)
