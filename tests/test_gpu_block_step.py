@@ -114,15 +114,16 @@ def test_block_step_degenerate(lib, wl):
     _check(wl, inp, out)
 
 
-def test_block_step_refined_mg_full_size(lib):
-    """The bench configuration: the Matrix-Game-shaped block step with the paper's two
-    refinement passes (Alg. routing).  The omission scores are compared with the oracle's,
-    the refined block sets with Alg. routing run by the oracle on those scores, and the
-    attention rows and PAR outputs with the oracle fed the GPU's routed blocks / anchor rows
-    (sampled rows on both sides of query-tile boundaries; every tile shape of the grid)."""
+@pytest.mark.parametrize("wl", [W.MG, W.HY], ids=lambda w: w.name)
+def test_block_step_refined_full_size(lib, wl):
+    """The bench configurations: the Matrix-Game- and HY-World-shaped block steps with the
+    paper's two refinement passes (Alg. routing).  The omission scores are compared with the
+    oracle's, the refined block sets with Alg. routing run by the oracle on those scores, and
+    the attention rows and PAR outputs with the oracle fed the GPU's routed blocks / anchor
+    rows (sampled rows on both sides of query-tile boundaries, the first and last tile pair
+    included; every tile shape of the grid)."""
     from tests.test_gpu_par_configs import edge_kind_sample
     from tests.test_gpu_refine import PAPER, check_refined
-    wl = W.MG
     inp = W.block_step_inputs(wl)
     out = _run_block(lib, wl, inp, refine=PAPER)
     anchors = list(wl.anchors)
@@ -136,6 +137,9 @@ def test_block_step_refined_mg_full_size(lib):
     changed, amb = check_refined(out["idx"], ug, anchors, wl.n_cur, wl.K, PAPER)
     assert amb < wl.H
     rng = np.random.default_rng(wl.seed + 1)
-    rows = np.unique(np.concatenate([[0, 127, 128, 1535, 1536, wl.S - 1], rng.integers(0, wl.S, 4)]))
-    tiles = edge_kind_sample(wl.grid[0], wl.grid[1], extra=(int(rng.integers(0, 28)),))
+    last = wl.S - wl.S % 256 if wl.S % 256 else wl.S - 256   # first row of the last tile pair
+    bounds = [0, 127, 128, 255, 256, last - 1, last, last + 127, last + 128, wl.S - 1]
+    rows = np.unique(np.concatenate([[b for b in bounds if 0 <= b < wl.S], rng.integers(0, wl.S, 4)]))
+    ntile = len(O.tiles_of(wl.grid[0], wl.grid[1], 8, 8))
+    tiles = edge_kind_sample(wl.grid[0], wl.grid[1], extra=(int(rng.integers(0, ntile)),))
     _check(wl, inp, out, rows=rows, tiles=tiles, routing=False)
