@@ -636,7 +636,7 @@ cast_status cast_check_device(void* stream) {
   const unsigned int wp = par_error_word(st, true);
   const unsigned int wr = route_error_word(st, true);
   const unsigned int wd = dense_error_word(st, true);
-  if (wa == 1u || wp || wd) return fail(CAST_ERR_DEVICE_TIMEOUT, "a kernel gave up on a bounded wait");
+  if (wa == 1u || wp || wd || wr == 2u) return fail(CAST_ERR_DEVICE_TIMEOUT, "a kernel gave up on a bounded wait");
   if (wa == 2u) return fail(CAST_ERR_INVALID_ARG, "attention: a routed block index was outside [0, M)");
   if (wr) return fail(CAST_ERR_INVALID_ARG, "routing: a candidate index was outside [0, M) or repeated");
   return check_launch("cast_check_device");

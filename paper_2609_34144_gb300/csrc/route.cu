@@ -24,6 +24,7 @@
 #include <cmath>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace cast {
 namespace {
@@ -31,6 +32,16 @@ namespace {
 constexpr int kPoolMaxThreads = 512;
 constexpr int kPoolUnroll = 8;     // 16-byte loads in flight per thread
 constexpr int kMaxClusterSplit = 8;
+// bulk-copy pooling of contiguous segments: a ring of kPoolStages copies of about
+// kPoolStageBytes (whole rows) per CTA, two CTAs per SM
+constexpr int kPoolStages = 3;
+constexpr int kPoolStageBytes = 32 * 1024;
+// bulk-copy pooling only where a CTA streams at least this much: measured on GB300, 0.245 vs
+// 0.253 ms for HY-World routing (2.7 MB per CTA) and 0.84 vs 0.89 ms for the stress history
+// (7 MB), but 0.052 vs 0.047 ms for Matrix-Game (0.6 MB), where the ring's per-CTA latency
+// chain is longer than that of eight register loads in flight per thread
+constexpr int64_t kPoolBulkMinBytes = 1 << 20;
+constexpr uint64_t kPoolWaitNs = 2000000000ull;
 
 // Thread layout of the pooling CTA: cgs 16-byte column groups side by side, lanes_r row lanes.
 struct PoolShape {
@@ -54,6 +65,7 @@ struct PoolArgs {
   int64_t q_row_stride, hist_row_stride;   // elements
   int n_anchors, M, S, B_v, D, nsplit, elt;
   int seg_base;           // segment of blockIdx.y == 0 (anchor frames first, then K, then V blocks)
+  int bulk_rows;          // bulk-copy pooling: rows per ring stage
   int Hg, Wg, nby, nbx;   // CAST_HIST_FRAMES: history frame grid and its 8x8 block grid
   int anchors[CAST_MAX_ANCHORS];
 };
@@ -104,11 +116,39 @@ __device__ __forceinline__ void launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+__device__ unsigned int g_pool_error;   // 1: a bulk-copy wait of the pooling gave up
+
+// Offset of the bulk-copy ring in the pooling kernel's dynamic shared memory (after colsum and
+// the per-lane rows), 128-byte aligned.
+__host__ __device__ inline size_t pool_ring_offset(int lanes_r, int D) {
+  return ((size_t)lanes_r * D * sizeof(float) + 127) & ~(size_t)127;
+}
+
+template <typename T>
+__device__ __forceinline__ void load_vec_smem(const uint8_t* p, float (&x)[16 / sizeof(T)]) {
+  const uint4 v = *reinterpret_cast<const uint4*>(p);
+  if (sizeof(T) == 4) {
+    x[0] = __uint_as_float(v.x);
+    x[1] = __uint_as_float(v.y);
+    x[2] = __uint_as_float(v.z);
+    x[3] = __uint_as_float(v.w);
+  } else {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      x[2 * k] = __uint_as_float(w[k] << 16);
+      x[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+    }
+  }
+}
+
 // grid (nsplit, n_seg), cluster (nsplit, 1, 1), cgs * lanes_r threads.  Dynamic smem:
-// colsum[D] and (lanes_r - 1) rows of per-lane sums.  SPATIAL: the history segments are
-// (1, 8, 8) blocks of frames [frames][Hg][Wg] (hv runs of wv consecutive tokens, Wg tokens
-// apart); the anchor-frame segments stay contiguous.
-template <typename T, bool SPATIAL>
+// colsum[D] and (lanes_r - 1) rows of per-lane sums (then, BULK, the copy ring).  SPATIAL: the
+// history segments are (1, 8, 8) blocks of frames [frames][Hg][Wg] (hv runs of wv consecutive
+// tokens, Wg tokens apart); the anchor-frame segments stay contiguous.  BULK (contiguous rows,
+// one 16-byte column group per thread): the CTA's rows arrive through a ring of bulk copies of
+// bulk_rows rows each, so that two CTAs keep about 190 KB of loads in flight per SM.
+template <typename T, bool SPATIAL, bool BULK>
 __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant__ PoolArgs a) {
   constexpr int VEC = 16 / sizeof(T);
   extern __shared__ float colsum[];
@@ -153,7 +193,64 @@ __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant_
   const int lanes_r = nthreads / cgs;                               // row lanes (>= 1)
   const int tcg = threadIdx.x % cgs, trl = threadIdx.x / cgs;
   float* lane_sum = colsum + a.D;                               // [lanes_r - 1][D] when lanes_r > 1
-  for (int cg = tcg; cg < ncg; cg += cgs) {
+  if constexpr (BULK) {
+    __shared__ __align__(8) uint64_t full[kPoolStages];
+    __shared__ int s_fail;
+    uint8_t* ring = reinterpret_cast<uint8_t*>(colsum) + pool_ring_offset(lanes_r, a.D);
+    const int row_bytes = a.D * a.elt, rps = a.bulk_rows, stage_bytes = rps * row_bytes;
+    const int nst = r1 > r0 ? (r1 - r0 + rps - 1) / rps : 0;
+    if (threadIdx.x == 0) {
+      for (int st = 0; st < kPoolStages; ++st) mbar_init(&full[st], 1);
+      fence_barrier_init();
+      s_fail = 0;
+    }
+    __syncthreads();
+    auto issue = [&](int it) {   // thread 0: rows r0 + it * rps .. into stage it % kPoolStages
+      const int st = it % kPoolStages, rr = r0 + it * rps, n = min(rps, r1 - rr);
+      mbar_arrive_expect_tx(&full[st], (uint32_t)(n * row_bytes));
+      bulk_load(ring + st * stage_bytes, base + (int64_t)rr * row_bytes, (uint32_t)(n * row_bytes), &full[st]);
+    };
+    int issued = 0;
+    if (threadIdx.x == 0)
+      for (; issued < kPoolStages && issued < nst; ++issued) issue(issued);
+    float acc[VEC];
+#pragma unroll
+    for (int k = 0; k < VEC; ++k) acc[k] = 0.f;
+    int it = 0;
+    for (; it < nst; ++it) {
+      const int st = it % kPoolStages;
+      if (mbar_wait(&full[st], (uint32_t)(it / kPoolStages) & 1u, kPoolWaitNs)) {
+        const int n = min(rps, r1 - (r0 + it * rps));
+        const uint8_t* sp = ring + st * stage_bytes + tcg * 16;
+        for (int q = trl; q < n; q += lanes_r) {
+          float x[VEC];
+          load_vec_smem<T>(sp + q * row_bytes, x);
+#pragma unroll
+          for (int k = 0; k < VEC; ++k) acc[k] += x[k];
+        }
+      } else {
+        s_fail = 1;
+      }
+      __syncthreads();   // stage st has been read by every thread
+      if (s_fail) break;
+      if (threadIdx.x == 0 && issued < nst) {
+        fence_proxy_async_smem();
+        issue(issued++);
+      }
+    }
+    if (s_fail && threadIdx.x == 0) {   // the copies in flight land before the memory is released
+      atomicExch(&g_pool_error, 1u);
+      for (int l = it; l < issued; ++l) mbar_wait(&full[l % kPoolStages], (uint32_t)(l / kPoolStages) & 1u, kPoolWaitNs);
+    }
+    if (trl == 0) {
+#pragma unroll
+      for (int k = 0; k < VEC; ++k) colsum[tcg * VEC + k] = acc[k];
+    } else if (trl < lanes_r) {
+#pragma unroll
+      for (int k = 0; k < VEC; ++k) lane_sum[(int64_t)(trl - 1) * a.D + tcg * VEC + k] = acc[k];
+    }
+  }
+  for (int cg = tcg; !BULK && cg < ncg; cg += cgs) {
     float acc[VEC];
 #pragma unroll
     for (int k = 0; k < VEC; ++k) acc[k] = 0.f;
@@ -241,8 +338,8 @@ __global__ void __launch_bounds__(kPoolMaxThreads) k_pool(const __grid_constant_
     out[c] = s * inv;
   }
   cluster_sync_all();   // no CTA leaves while a peer still reads its shared memory
-  // launched as a programmatic dependent of the anchor-frame pooling: this grid completes only
-  // after that one has, so its own dependents see every mean
+  // the second pooling launch is a programmatic dependent of the first: it completes only after
+  // the first has, so its own dependents see every mean
   grid_dependency_wait();
 }
 
@@ -719,6 +816,7 @@ __global__ void __launch_bounds__(kHeadThreads) k_head_small(const __grid_consta
     // initial mask: TopK of u (Eq. topk), ties to the lower block index
     const float uk = live ? u : -INFINITY;
     int rank = 0;
+#pragma unroll 4
     for (int l = 0; l < M; ++l) {
       const float w = __shfl_sync(0xffffffffu, uk, l);
       rank += (w > uk) || (w == uk && l < lane);
@@ -795,6 +893,7 @@ __global__ void __launch_bounds__(kHeadThreads) k_head_small(const __grid_consta
           const float G = live ? lam_anc * ui + lam_rec * rec : -INFINITY;
           // best response TopK(G) and its gain sum_m G_m (x_new - x_i) (J is affine in x_i)
           int rank = 0;
+#pragma unroll 4
           for (int l = 0; l < M; ++l) {
             const float w = __shfl_sync(0xffffffffu, G, l);
             rank += (w > G) || (w == G && l < lane);
@@ -1437,23 +1536,38 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
   for (int k = 0; k < a.n_anchors; ++k) pa.anchors[k] = a.anchors[k];
 
   const size_t psm = route_pool_smem_bytes(a);
-  auto pool_fn = a.dtype == CAST_BF16 ? (hg.spatial ? k_pool<__nv_bfloat16, true> : k_pool<__nv_bfloat16, false>)
-                                      : (hg.spatial ? k_pool<float, true> : k_pool<float, false>);
-  if (psm > 48 * 1024 &&
-      cudaFuncSetAttribute(pool_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psm) != cudaSuccess)
-    return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory for pooling", psm);
   const PoolShape ps = pool_shape(D, pa.elt);
-  // two launches of the pooling kernel, each with its own row split: the anchor frames (few
-  // long segments), then, as a programmatic dependent that fills the remaining SMs, the
-  // history blocks (it completes only after the first, see k_pool)
+  const int row_bytes = D * pa.elt;
+  // two launches of the pooling kernel, each with its own row split: the history blocks (the
+  // larger part), then, as a programmatic dependent that fills the remaining SMs, the anchor
+  // frames (few long segments; it completes only after the first, see k_pool).  A part whose
+  // rows are contiguous (row stride D), whose column groups fit one per thread and whose CTAs
+  // stream at least kPoolBulkMinBytes each is pooled through the bulk-copy ring.
   for (int part = 0; part < 2; ++part) {
-    const int nsplit = part == 0 ? p.nsplit_q : p.nsplit_kv;
+    const bool hist = part == 0;
+    const int nsplit = hist ? p.nsplit_kv : p.nsplit_q;
+    const bool contiguous = hist ? (!hg.spatial && a.hist_row_stride == D) : a.q_row_stride == D;
+    const int rows = hist ? a.B_v : a.S;
+    const int64_t cta_bytes = (int64_t)((rows + nsplit - 1) / nsplit) * row_bytes;
+    const bool bulk = contiguous && ps.cgs * (16 / pa.elt) == D && row_bytes <= kPoolStageBytes &&
+                      cta_bytes >= kPoolBulkMinBytes;
     pa.nsplit = nsplit;
-    pa.seg_base = part == 0 ? 0 : a.n_anchors;
+    pa.seg_base = hist ? a.n_anchors : 0;
+    pa.bulk_rows = bulk ? kPoolStageBytes / row_bytes : 0;
+    const size_t smem = bulk ? pool_ring_offset(ps.lanes_r, D) + (size_t)kPoolStages * pa.bulk_rows * row_bytes : psm;
+    void (*fn)(PoolArgs);
+    if (a.dtype == CAST_BF16)
+      fn = bulk ? k_pool<__nv_bfloat16, false, true>
+                : (hist && hg.spatial ? k_pool<__nv_bfloat16, true, false> : k_pool<__nv_bfloat16, false, false>);
+    else
+      fn = bulk ? k_pool<float, false, true> : (hist && hg.spatial ? k_pool<float, true, false> : k_pool<float, false, false>);
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+      return fail(CAST_ERR_CUDA, "routing: cannot reserve %zu B of shared memory for pooling", smem);
     cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3(nsplit, part == 0 ? a.n_anchors : 2 * a.M, 1);
+    cfg.gridDim = dim3(nsplit, hist ? 2 * a.M : a.n_anchors, 1);
     cfg.blockDim = dim3(ps.cgs * ps.lanes_r, 1, 1);
-    cfg.dynamicSmemBytes = psm;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cudaLaunchAttribute at[2];
     at[0].id = cudaLaunchAttributeClusterDimension;
@@ -1464,7 +1578,7 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
     at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = at;
     cfg.numAttrs = part == 0 ? 1 : 2;
-    if (cudaLaunchKernelEx(&cfg, pool_fn, pa) != cudaSuccess) return check_launch("routing pool kernel");
+    if (cudaLaunchKernelEx(&cfg, fn, pa) != cudaSuccess) return check_launch("routing pool kernel");
     const cast_status s = check_launch("routing pool kernel");
     if (s != CAST_OK) return s;
   }
@@ -1551,15 +1665,17 @@ cast_status launch_route(const cast_route_args& a, void* ws, cudaStream_t st) {
 }
 
 unsigned int route_error_word(cudaStream_t st, bool clear) {
-  unsigned int v = 0;
+  unsigned int v = 0, vp = 0;
   cudaMemcpyFromSymbolAsync(&v, g_route_error, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  cudaMemcpyFromSymbolAsync(&vp, g_pool_error, sizeof(vp), 0, cudaMemcpyDeviceToHost, st);
   cudaStreamSynchronize(st);
-  if (clear && v) {
+  if (clear && (v || vp)) {
     const unsigned int z = 0;
     cudaMemcpyToSymbolAsync(g_route_error, &z, sizeof(z), 0, cudaMemcpyHostToDevice, st);
+    cudaMemcpyToSymbolAsync(g_pool_error, &z, sizeof(z), 0, cudaMemcpyHostToDevice, st);
     cudaStreamSynchronize(st);
   }
-  return v;
+  return vp ? 2u : v;   // 2: a pooling wait gave up; 1: a candidate index outside [0, M) or repeated
 }
 
 }  // namespace cast

@@ -61,6 +61,25 @@ def test_route_small(lib, dtype, d):
     assert amb == 0
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_route_bulk_pooling(lib, dtype):
+    """Long contiguous segments (at least 1 MB per pooling CTA in both launches), which the
+    pooling streams through its bulk-copy ring: pooled means, u and TopK against the oracle."""
+    N, S, H, d, M, Bv, K = 3, 2048, 12, 128, 4, 4096, 2
+    q, k, v = _inputs(31, N, S, H, d, M, Bv, dtype)
+    anchors = [0, 2]
+    idx, u, (qb, kb, vb) = lib.cast_route_topk(to_dev(q, dtype), anchors, to_dev(k, dtype),
+                                                to_dev(v, dtype), K, want_u=True, want_pooled=True)
+    torch.cuda.synchronize()
+    lib.cast_check_device()
+    rt = O.pooled_routing(q, anchors, k, v)
+    np.testing.assert_allclose(to_host(qb), rt.qbar, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(to_host(kb), rt.kbar, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(to_host(vb), rt.vbar, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(to_host(u), rt.u, rtol=2e-4, atol=1e-7 * rt.u.max())
+    check_idx(idx.cpu().numpy(), rt.u, K)
+
+
 def test_route_gram_projection(lib):
     """GPU with G = P^T P equals the oracle's literal ||P delta||^2 (Eq. omission)."""
     N, S, H, d, M, Bv, K = 2, 64, 2, 64, 9, 40, 4
