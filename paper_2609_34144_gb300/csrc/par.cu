@@ -7,9 +7,9 @@
 //       spectrum stays in shared memory) and, for every anchor pair with targets, reduces
 //       Z = sum_c w_c F_b conj(F_a) and W = sum_c w_c |F_b||F_a| over the chunk's channels
 //       (warp transpose reductions) into one record in the workspace.
-//   K_transport (tile, pair): sums the records of the tile's channel chunks in chunk order
-//       (deterministic) and derives eta, reliability, principal phases, the confidence c and
-//       the gate g per bin; writes theta and g.
+//   K_transport (tile, pair[, target]): sums the records of the tile's channel chunks in chunk
+//       order (deterministic) and derives eta, reliability, principal phases, the confidence c
+//       and the gate g per bin; writes theta and g (and, for bf16, one target's blend matrix).
 //   K_blend (tile, channel chunk): streams the anchors again (an L2 hit at these sizes), forms
 //       their spectra and writes every target straight from registers:
 //       R_t = IRFFT2((1-alpha) F_a e^{i g alpha theta} + alpha F_b e^{-i g (1-alpha) theta}).
@@ -21,9 +21,11 @@
 //       laid out as a swizzled UMMA operand) and one UMMA chain per pair of targets computes
 //       [H_t1 ; H_t2] [X_a ; X_b] for 128 channels (M = 128 output rows, K = 128 tokens).
 // The CTAs of a pass never wait on each other, so the passes fill the GPU whatever the number
-// of anchor pairs; the passes are chained as programmatic dependents.  Global traffic beyond
-// the algorithmic bytes: a second read of the anchors and the records (120 floats per tile,
-// pair and chunk).
+// of anchor pairs; the passes are chained as programmatic dependents (the transport releases
+// the blend at its end), the full-tile chain on the caller's stream and the edge-tile chain on
+// a second stream.  Global traffic beyond the algorithmic bytes: a second read of the anchors,
+// the records (120 floats per tile, pair and chunk) and, for bf16, the blend matrices (32 KB
+// per tile and target, read from L2 by every channel chunk).
 #include <cuda_bf16.h>
 
 #include <algorithm>

@@ -2,12 +2,15 @@
 //
 //   K_pool  : mean of every pooled segment (anchor query frames, history key blocks, history
 //             value blocks): HBM-bound streaming of (K_f S + 2 M B_v) H d elements with 16-byte
-//             loads.  A segment's rows are split over the CTAs of one thread-block cluster;
-//             the CTAs reduce their column sums through distributed shared memory in rank order
-//             (deterministic) and write q_bar, k_bar, v_bar in f32.  No partial sums leave the
-//             chip.  Two launches with their own row split: the anchor frames (few long
-//             segments), then the history blocks (with (1, 8, 8) spatial blocks of history
-//             frames, 8 runs of up to 8 tokens each).
+//             loads, or, for long contiguous segments, through a ring of bulk copies into
+//             shared memory.  A segment's rows are split over the CTAs of one thread-block
+//             cluster; the CTAs reduce their column sums through distributed shared memory in
+//             rank order (deterministic) and write q_bar, k_bar, v_bar in f32.  No partial sums
+//             leave the chip.  Two launches with their own row split: the history blocks (with
+//             (1, 8, 8) spatial blocks of history frames, 8 runs of up to 8 tokens each), then
+//             the anchor frames (few long segments).
+//   K_head_small : for M <= 32 blocks and up to 8 anchors, one CTA per head with one warp per
+//             anchor for the statistics and the refinement in warp 0's registers.
 //   K_head  : one CTA per head, every anchor at once, with the head's k_bar and v_bar staged in
 //             shared memory: s, pi, o_bar, delta, u (Eq. omission, with an optional Gram matrix
 //             G = P^T P of the output projection), the TopK mask of each anchor (ties to the
