@@ -26,7 +26,9 @@ Readings of points where the paper is silent, ambiguous or garbled:
 Parity unpinned: the full paper gate of PAR on data that is not a translation.  The
 paper prints no worked example for it; the pins fix its pieces (the transform, the
 confidence bounds and closed forms, the gate's limits g = 0 / g = 1, exact translations
-and Prop. 1), and beyond them the oracle is the definition itself.
+and Prop. 1) and one property of the whole (time reversal: swapping a pair's anchors with
+alpha -> 1 - alpha reconstructs the same frames), and beyond them the oracle is the
+definition itself.
 """
 from __future__ import annotations
 

@@ -308,6 +308,24 @@ def check_par_weights_scale_invariant():
     assert np.allclose(c, d, atol=1e-12)
 
 
+def check_par_time_reversal():
+    """Reversing the frames swaps the two anchors of every pair and maps alpha to 1 - alpha
+    (Eq. block); the pooled Z becomes conj(Z) while W, c and g stay the same (Eqs. cross,
+    confidence, gate), and Eq. (fcpasm) with theta -> -theta then reconstructs the same frames.
+    So PAR of the reversed sequence, reversed back, equals PAR of the sequence: the paper's
+    gate on non-translating fields, interpolated and extrapolated frames, ragged edge tiles and
+    channel weights."""
+    r = _rng(32)
+    R = r.standard_normal((9, 11, 13, 6))
+    mask = [0, 1, 0, 0, 1, 0, 1, 0, 0]
+    wc = r.uniform(0.5, 2.0, 6)
+    fwd, info = O.par_reconstruct(R, np.asarray(mask, dtype=np.uint8), wc, O.ParParams(),
+                                  with_info=True)
+    assert not any(tt.branch_ambiguous for tt in info.values())   # theta away from +-pi
+    rev = _par(R[::-1].copy(), mask[::-1], wch=wc)[::-1]
+    assert np.allclose(fwd, rev, atol=1e-10)
+
+
 # ---------------------------------------------------------------------------
 # Routing (Section 4.4, Eqs. pooled, omission; App. B.1 Eq. omissionexact)
 # ---------------------------------------------------------------------------

@@ -41,6 +41,37 @@ def _transport_mirror_same_sign(Fa, Fb, wch, p, bins, amb_tol=1e-5):
     return tt
 
 
+def _transport_w_one_sided(Fa, Fb, wch, p, bins, amb_tol=1e-5):
+    # Eq. (cross) with W = sum_c w_c |F_b|^2 (one anchor's power) instead of |F_b| |F_a|
+    wc = np.ones(Fa.shape[0]) if wch is None else np.asarray(wch, dtype=np.float64)
+    Z = np.einsum("c,cij->ij", wc, Fb * np.conj(Fa))
+    W = np.einsum("c,cij->ij", wc, np.abs(Fb) ** 2)
+    eta = p.eta_rel * W.max() + p.eta_abs
+    Zabs = np.abs(Z)
+    rel_bin = (W > eta) & (Zabs > eta)
+    ry, rx = bins.rep[..., 0], bins.rep[..., 1]
+    reliable = rel_bin[ry, rx]
+    theta_rep = np.angle(Z[ry, rx])
+    theta_rep = np.where(theta_rep <= -np.pi, np.pi, theta_rep)
+    theta = np.where(bins.mirror, -theta_rep, theta_rep)
+    theta = np.where(reliable & ~bins.selfconj, theta, 0.0)
+    omega_plus = reliable & ~bins.dc
+    if omega_plus.any():
+        c = float(np.sum(bins.kappa * Zabs * omega_plus) / (np.sum(bins.kappa * W * omega_plus) + p.eps))
+    else:
+        c = 0.0
+        theta = np.zeros_like(theta)
+    tau = p.tau_low + (p.tau_high - p.tau_low) * bins.nu ** p.q
+    g = 1.0 / (1.0 + np.exp(-(c - tau) / p.T))
+    if p.gate_mode == "zero":
+        g = np.zeros_like(g)
+    elif p.gate_mode == "one":
+        g = np.ones_like(g)
+    if p.band_radius >= 0:
+        g = np.where(bins.rho > p.band_radius, 0.0, g)
+    return O.TileTransport(Z, W, eta, reliable, theta, c, g, False, False)
+
+
 def _bins_kappa_one(h, w):
     b = _orig_bins(h, w)
     b.kappa = np.ones_like(b.kappa)
@@ -250,6 +281,7 @@ MUTATIONS = {
     "blend_gate_dropped": ("blend", _blend_no_gate),
     "dft_exponent_sign": ("rfft2_ortho", _rfft2_transposed),
     "mirror_not_negated": ("tile_transport", _transport_mirror_same_sign),
+    "cross_amplitude_one_sided": ("tile_transport", _transport_w_one_sided),
     "kappa_dropped": ("tile_bins", _bins_kappa_one),
     "nu_not_normalised": ("tile_bins", _bins_nu_unnormalised),
     "omission_renorm_dropped": ("pooled_routing", _pooled_no_renorm),
