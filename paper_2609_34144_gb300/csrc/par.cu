@@ -759,14 +759,15 @@ __global__ void __launch_bounds__(128) k_par_transport(const __grid_constant__ P
 // ------------------------------------------------------------------ K_blend_tc (bf16)
 // Persistent, one CTA per SM over the (tile, 128-channel chunk) items of one tile kind, 224
 // threads: warp 0 streams the anchors of each item ([8 x 8 tokens][channels] through a
-// 128-byte-swizzled TMA box, the MN-major UMMA operand) through three stages; warp 6 streams
+// 128-byte-swizzled TMA box, the MN-major UMMA operand) through four stages (an item's first
+// anchors load while the previous item's last pairs run); warp 6 streams
 // the blend matrices K_transport wrote, two targets of one pair stacked per group (rows 0-63
 // target 1, 64-127 target 2 of the M = 128 operand), two groups in flight;
 // warp 1 issues one UMMA chain per group (2 pieces x 8 K-steps, M = 128, N = 128) into one of
 // two TMEM buffers; warps 2-5 (one TMEM lane quadrant each: a target slot and 32 output tokens)
 // convert the result to bf16 into a swizzled staging tile that one thread stores with TMA.
 constexpr int kTbNC = 128;                      // channels per item
-constexpr int kTbStages = 3;
+constexpr int kTbStages = 4;                    // 225 KB of shared memory in all
 constexpr int kTbPlane = 64 * kTbNC * 2;        // one anchor tile, 16 KB
 constexpr int kTbPiece = 128 * 128 * 2;         // one bf16 piece of a group's [128][128] operand, 32 KB
 constexpr int kTbGroup = 2 * kTbPiece;          // both pieces, 64 KB
